@@ -1,0 +1,62 @@
+"""The pins must catch plausible mistakes in the oracle. Each case below
+plants one mistake in a copy of the oracle's C source (on the CPU, in a
+temporary directory), builds it, and runs the pin suite against it with the
+wrapper pointed at the broken library: at least one pin has to fail."""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "unif_moe_oracle.c")
+
+MUTANTS = {
+    # dropped factor (1 - 2 tau) in Eq. 18
+    "alpha_dropped_term": ("tau + (1.0 - 2.0 * tau) * sigmoid(z[0])", "tau + sigmoid(z[0])"),
+    # wrong sign inside the logistic function
+    "sigmoid_sign": ("return 1.0 / (1.0 + exp(-z));", "return 1.0 / (1.0 + exp(z));"),
+    # prototypes from the wrong expert's keys (Eq. 20 uses the shared expert)
+    "prototype_off_by_one": ("sum += w_up0[(size_t)h * d + i];",
+                             "sum += w_up0[(size_t)((h + 1) % H) * d + i];"),
+    # sum instead of mean in Eq. 20 (changes nothing under exact TopK, but the
+    # priorities pin sees it)
+    "prototype_sum": ("round_to(sum / (double)M, round_mode)", "round_to(sum, round_mode)"),
+    # transposed value matrix
+    "value_transposed": ("V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * d + i) * H + h];",
+                         "V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * H + h) * d + i];"),
+    # residual experts run the shared blocks instead of the complement (Eq. 23)
+    "residual_blocks": ("EXPERT_BLOCKS(1 + j, 0);", "EXPERT_BLOCKS(1 + j, 1);"),
+    # shared pathway weighted by beta instead of alpha (Eq. 30)
+    "shared_weight": ("yt[i] += alpha[t] * acc[i];", "yt[i] += (1.0 - alpha[t]) * acc[i];"),
+    # TopK of the smallest priorities (Eq. 22)
+    "topk_reversed": ("shr |= 1ull << (prefix_blocks ? r : uorder[r]);",
+                      "shr |= 1ull << (prefix_blocks ? r : uorder[B - 1 - r]);"),
+    # the selected prefix one expert too long (Eq. 27 asks for the smallest)
+    "k_plus_one": ("if (P >= beta) { k = n; break; }", "if (P >= beta) { k = n < K ? n + 1 : K; break; }"),
+    # affinity of the unsorted expert index used as the weight (Eq. 25)
+    "p_unsorted": ("for (int i = 0; i < K; ++i) { q[i] = order[i]; p[i] = s[order[i]]; }",
+                   "for (int i = 0; i < K; ++i) { q[i] = order[i]; p[i] = s[i]; }"),
+    # round() replaced by truncation (Eq. 19)
+    "b_truncated": ("int b = (int)nearbyint((double)B * alpha);", "int b = (int)((double)B * alpha);"),
+    # GeLU without the 1/sqrt(2) scaling
+    "gelu_scale": ("erf(v * M_SQRT1_2)", "erf(v)"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_catch_mutant(name, tmp_path):
+    old, new = MUTANTS[name]
+    src = open(SRC).read()
+    assert src.count(old) == 1, "mutation anchor not found: " + name
+    mutated = tmp_path / "mutant.c"
+    mutated.write_text(src.replace(old, new))
+    lib = tmp_path / "libmutant.so"
+    subprocess.run(["gcc", "-O2", "-ffp-contract=off", "-fopenmp", "-shared", "-fPIC", "-o",
+                    str(lib), str(mutated), "-lm"], check=True)
+    env = dict(os.environ, UNIF_MOE_ORACLE_LIB=str(lib), OMP_NUM_THREADS="2")
+    res = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+                          os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                         cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert res.returncode != 0, "no pin caught mutant %s:\n%s" % (name, res.stdout[-2000:])

@@ -1,0 +1,395 @@
+"""Pins for the CPU oracle: checks against facts the paper and the mathematics
+fix, computed here by other means than the oracle's own code (dense matrix
+products, exhaustive search over subsets, a hand derivation, library routines
+for the normal CDF and the logistic function).
+
+Each test names the passage it pins. None needs a GPU.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy.special import expit, softmax
+from scipy.stats import norm
+
+import oracle
+from oracle import Thresholds
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def gelu_ref(v):
+    # GeLU(v) = v * Phi(v), Phi the standard normal CDF (library routine).
+    return v * norm.cdf(v)
+
+
+def rand_layer(rng, d, H, K, B, router_scale=1.0, T=64):
+    x = rng.standard_normal((T, d))
+    w_router = rng.standard_normal((d, K + 1)) * router_scale / math.sqrt(d)
+    w_up = rng.standard_normal((K + 1, H, d)) / math.sqrt(d)
+    w_down = rng.standard_normal((K + 1, d, H)) / math.sqrt(H)
+    return x, w_router, w_up, w_down
+
+
+def block_outputs_dense(x, w_up, w_down, B):
+    """All (K+1)*B block outputs E_e^(b)(x) for every token, by dense matrix
+    products: [T][K+1][B][d] (Eq. 16)."""
+    T = x.shape[0]
+    E1, H, d = w_up.shape
+    M = H // B
+    out = np.zeros((T, E1, B, d))
+    for e in range(E1):
+        act = gelu_ref(x @ w_up[e].T)  # [T][H]
+        for blk in range(B):
+            sl = slice(blk * M, (blk + 1) * M)
+            out[:, e, blk, :] = act[:, sl] @ w_down[e][:, sl].T
+    return out
+
+
+# --------------------------------------------------------------------------
+# Hand-derived example (Sec. III, Eqs. 16-30 and 35)
+# --------------------------------------------------------------------------
+
+def _num(v):
+    if isinstance(v, str):
+        return {"ln3/2": math.log(3) / 2}[v]
+    return float(v)
+
+
+def load_hand():
+    g = json.load(open(os.path.join(GOLDEN, "hand_example.json")))
+    x = np.array(g["x"], dtype=np.float64)
+    w_router = np.array([[_num(v) for v in row] for row in g["w_router"]])
+    w_up = np.array(g["w_up"], dtype=np.float64)
+    vr = np.array(g["value_rows"], dtype=np.float64)  # [K+1][H][d]
+    w_down = np.ascontiguousarray(vr.transpose(0, 2, 1))  # [K+1][d][H]
+    mask = np.array(g["mask"], dtype=np.uint8)
+    return g, x, w_router, w_up, w_down, mask
+
+
+def test_hand_example_decisions_and_output(oracle_mod):
+    g, x, w_router, w_up, w_down, mask = load_hand()
+    B = g["B"]
+    y, r = oracle.layer(x, w_router, w_up, w_down, B, mask=mask)
+    exp = g["expected"]
+    assert r.b.tolist() == exp["b"]
+    assert r.k.tolist() == exp["k"]
+    for t in range(3):
+        blocks = [blk for blk in range(B) if (int(r.shr_mask[t]) >> blk) & 1]
+        assert blocks == exp["shared_blocks"][t]
+        experts = sorted(int(r.q[t, i]) + 1 for i in range(r.k[t]))
+        assert experts == exp["experts"][t]
+    assert r.cb(B).tolist() == exp["C_B"]
+    alpha = [0.5, 0.25 + expit(-3.0) / 2, 0.0]
+    np.testing.assert_allclose(r.alpha, alpha, rtol=0, atol=1e-15)
+    s = {0: (0.75, 0.25), 1: (math.sqrt(3) / (1 + math.sqrt(3)), 1 / (1 + math.sqrt(3)))}
+    for t in range(3):
+        want = np.zeros(2)
+        for coef, pre, val in exp["output_terms"][t]:
+            c = {"alpha": alpha[t], "s1": s.get(t, (0, 0))[0], "s2": s.get(t, (0, 0))[1]}[coef]
+            want += c * gelu_ref(pre) * np.array(val, dtype=np.float64)
+        np.testing.assert_allclose(y[t], want, rtol=1e-13, atol=1e-15)
+
+
+def test_hand_example_groups(oracle_mod):
+    g, x, w_router, w_up, w_down, mask = load_hand()
+    B, K = g["B"], g["K"]
+    _, r = oracle.layer(x, w_router, w_up, w_down, B, mask=mask)
+    counts, tok, w = oracle.groups(r, K, B, mask)
+    assert counts.tolist() == g["expected"]["groups"]["counts"]
+    assert tok.tolist() == g["expected"]["groups"]["tokens"]
+    # weights: alpha on shared groups, p on residual groups
+    sA, sB = 0.75, math.sqrt(3) / (1 + math.sqrt(3))
+    np.testing.assert_allclose(w, [0.5, 0.25 + expit(-3.0) / 2, sB, sA, 1 - sB], atol=1e-15)
+
+
+# --------------------------------------------------------------------------
+# Exhaustive search on tiny layers (Eqs. 18-30 by enumeration)
+# --------------------------------------------------------------------------
+
+def brute_force(x, w_router, w_up, w_down, B, th: Thresholds):
+    """Decisions by exhaustive search and the output as a masked sum of dense
+    block outputs. No sorting: the shared set is the b-subset with the
+    largest total priority, the residual set the smallest subset of experts
+    whose affinity mass reaches beta (largest mass among subsets of that
+    size)."""
+    T, d = x.shape
+    K = w_up.shape[0] - 1
+    H = w_up.shape[1]
+    M = H // B
+    tau = (B - 1) / B**2 if math.isnan(th.tau) else th.tau
+    mu = np.stack([w_up[0, blk * M:(blk + 1) * M, :].mean(axis=0) for blk in range(B)])
+    blocks = block_outputs_dense(x, w_up, w_down, B)
+    ys, bs, ks, shr_sets, exp_sets = [], [], [], [], []
+    for t in range(T):
+        z = x[t] @ w_router
+        alpha = tau + (1 - 2 * tau) * expit(z[0]) if math.isnan(th.alpha_fixed) else th.alpha_fixed
+        b = int(np.rint(B * alpha))
+        u = mu @ x[t]
+        best = max(itertools.combinations(range(B), b), key=lambda S: sum(u[i] for i in S))
+        shr = set(best)
+        s = softmax(z[1:])
+        beta = 1 - alpha if math.isnan(th.beta_fixed) else th.beta_fixed
+        chosen = None
+        for n in range(1, K + 1):
+            S = max(itertools.combinations(range(K), n), key=lambda S: sum(s[j] for j in S))
+            if sum(s[j] for j in S) >= beta or n == K:
+                chosen = S
+                break
+        y = alpha * sum(blocks[t, 0, blk] for blk in shr) if shr else np.zeros(d)
+        for j in chosen:
+            y = y + s[j] * sum((blocks[t, 1 + j, blk] for blk in range(B) if blk not in shr),
+                               np.zeros(d))
+        ys.append(y)
+        bs.append(b)
+        ks.append(len(chosen))
+        shr_sets.append(shr)
+        exp_sets.append(set(chosen))
+    return np.array(ys), np.array(bs), np.array(ks), shr_sets, exp_sets
+
+
+@pytest.mark.parametrize("d,H,K,B", [(4, 8, 3, 2), (8, 16, 4, 4), (5, 12, 2, 4), (6, 16, 4, 2)])
+@pytest.mark.parametrize("seed", [0, 1])
+def test_brute_force_tiny(oracle_mod, d, H, K, B, seed):
+    rng = np.random.default_rng(100 * seed + d)
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, router_scale=3.0, T=48)
+    th = Thresholds()
+    y, r = oracle.layer(x, w_router, w_up, w_down, B, th)
+    yb, bb, kb, shr, exps = brute_force(x, w_router, w_up, w_down, B, th)
+    assert r.b.tolist() == bb.tolist()
+    assert r.k.tolist() == kb.tolist()
+    em = r.expert_mask()
+    for t in range(x.shape[0]):
+        assert {blk for blk in range(B) if (int(r.shr_mask[t]) >> blk) & 1} == shr[t]
+        assert {j for j in range(K) if (int(em[t]) >> j) & 1} == exps[t]
+    np.testing.assert_allclose(y, yb, rtol=1e-11, atol=1e-13)
+
+
+@pytest.mark.parametrize("th", [Thresholds(beta_fixed=0.7), Thresholds(alpha_fixed=0.4),
+                                Thresholds(tau=0.1)])
+def test_brute_force_threshold_variants(oracle_mod, th):
+    rng = np.random.default_rng(7)
+    x, w_router, w_up, w_down = rand_layer(rng, 6, 16, 4, 4, router_scale=3.0, T=40)
+    y, r = oracle.layer(x, w_router, w_up, w_down, 4, th)
+    yb, bb, kb, _, _ = brute_force(x, w_router, w_up, w_down, 4, th)
+    assert r.b.tolist() == bb.tolist() and r.k.tolist() == kb.tolist()
+    np.testing.assert_allclose(y, yb, rtol=1e-11, atol=1e-13)
+
+
+# --------------------------------------------------------------------------
+# Special cases that reduce to textbook layers
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("B", [2, 4, 8])
+def test_alpha_one_is_dense_ffn(oracle_mod, B):
+    """alpha fixed at 1: b = B, every block shared, I_res empty (Eqs. 19,
+    22-23), so y = E_shr(x), the plain FFN of Eq. 4."""
+    rng = np.random.default_rng(B)
+    x, w_router, w_up, w_down = rand_layer(rng, 16, 64, 4, B)
+    y, r = oracle.layer(x, w_router, w_up, w_down, B, Thresholds(alpha_fixed=1.0))
+    assert (r.b == B).all()
+    dense = gelu_ref(x @ w_up[0].T) @ w_down[0].T
+    np.testing.assert_allclose(y, dense, rtol=1e-12, atol=1e-13)
+
+
+@pytest.mark.parametrize("th", [Thresholds(alpha_fixed=0.0, beta_fixed=1.0),
+                                Thresholds(alpha_fixed=0.0, topk_fixed=5)])
+def test_alpha_zero_all_experts_is_soft_moe(oracle_mod, th):
+    """alpha = 0 and all K experts selected: y = sum_j s_j E_j(x), the
+    conventional MoE output of Eq. 5 with k = K (softmax gate of Eq. 2)."""
+    rng = np.random.default_rng(3)
+    K, B = 5, 4
+    x, w_router, w_up, w_down = rand_layer(rng, 12, 32, K, B, router_scale=4.0)
+    y, r = oracle.layer(x, w_router, w_up, w_down, B, th)
+    assert (r.b == 0).all() and (r.k == K).all()
+    s = softmax(x @ w_router[:, 1:], axis=1)
+    want = sum(s[:, [j]] * (gelu_ref(x @ w_up[1 + j].T) @ w_down[1 + j].T) for j in range(K))
+    np.testing.assert_allclose(y, want, rtol=1e-12, atol=1e-13)
+
+
+def test_two_blocks_share_exactly_one(oracle_mod):
+    """B = 2 gives tau = 1/4, alpha in (1/4, 3/4), so b = 1 always (Eqs. 18-19)."""
+    rng = np.random.default_rng(11)
+    x, w_router, w_up, w_down = rand_layer(rng, 8, 16, 3, 2, router_scale=6.0, T=400)
+    _, r = oracle.layer(x, w_router, w_up, w_down, 2)
+    assert (r.alpha > 0.25).all() and (r.alpha < 0.75).all()
+    assert r.alpha.min() < 0.27 and r.alpha.max() > 0.73  # the range is exercised
+    assert (r.b == 1).all()
+
+
+def test_top1_covers_one_full_ffn(oracle_mod):
+    """k = 1: shared plus residual blocks are exactly one FFN's B blocks,
+    C_B = B (Eq. 35 and the remark after it)."""
+    rng = np.random.default_rng(5)
+    x, w_router, w_up, w_down = rand_layer(rng, 8, 32, 4, 8)
+    _, r = oracle.layer(x, w_router, w_up, w_down, 8, Thresholds(topk_fixed=1))
+    assert (r.k == 1).all() and (r.cb(8) == 8).all()
+
+
+# --------------------------------------------------------------------------
+# Invariants stated in the paper, on realistic random layers
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("B,K", [(4, 4), (8, 8), (16, 16), (16, 32)])
+def test_invariants(oracle_mod, B, K):
+    rng = np.random.default_rng(B * 100 + K)
+    d = 32
+    x, w_router, w_up, w_down = rand_layer(rng, d, 16 * B, K, B, router_scale=8.0, T=500)
+    y, r = oracle.layer(x, w_router, w_up, w_down, B)
+    T = x.shape[0]
+    # Eq. 19 remark: b in {1..B-1}
+    assert r.b.min() >= 1 and r.b.max() <= B - 1
+    pc = np.array([bin(int(v)).count("1") for v in r.shr_mask])
+    assert (pc == r.b).all()  # |I_shr| = b (Eq. 22)
+    for t in range(T):
+        inside = [r.u[t, blk] for blk in range(B) if (int(r.shr_mask[t]) >> blk) & 1]
+        outside = [r.u[t, blk] for blk in range(B) if not (int(r.shr_mask[t]) >> blk) & 1]
+        assert min(inside) >= max(outside)  # TopK of priorities (Eq. 22)
+        # p sorted, a permutation of s (Eq. 25)
+        assert (np.diff(r.p[t]) <= 0).all()
+        np.testing.assert_allclose(np.sort(r.s[t]), np.sort(r.p[t]), rtol=0, atol=0)
+        kk = r.k[t]
+        Pk = r.p[t, :kk].sum()
+        Pk1 = r.p[t, :kk - 1].sum()
+        # Eq. 31-32: beta <= P_k < beta + p_k, and 1 <= alpha + P_k < 1 + p_k
+        assert r.beta[t] <= Pk + 1e-15 and Pk < r.beta[t] + r.p[t, kk - 1] + 1e-15
+        assert 1 - 1e-15 <= r.alpha[t] + Pk < 1 + r.p[t, kk - 1] + 1e-15
+        assert Pk1 < r.beta[t]  # minimality (Eq. 27)
+    np.testing.assert_allclose(r.alpha + r.beta, 1.0, atol=1e-15)  # Eq. 26
+    # The spread of decisions is exercised
+    assert len(set(r.b.tolist())) > 1 and len(set(r.k.tolist())) > 1
+
+
+def test_priorities_are_block_mean_preactivations(oracle_mod):
+    """u_b = x mu_b equals the mean over block b of the shared expert's
+    pre-activations x K_shr[:, h] (Eqs. 20-21)."""
+    rng = np.random.default_rng(9)
+    B, K, d, H = 8, 4, 24, 96
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, T=50)
+    mu = oracle.prototypes(w_up, B, oracle.ROUND_NONE)
+    r = oracle.route(x, w_router, mu, K, B)
+    pre = x @ w_up[0].T
+    want = pre.reshape(50, B, H // B).mean(axis=2)
+    np.testing.assert_allclose(r.u, want, rtol=1e-12, atol=1e-14)
+
+
+def test_block_decomposition_sums_to_expert(oracle_mod):
+    """E_j = sum_b E_j^(b) (Eq. 16): with every block shared and alpha = 1 the
+    oracle's blockwise sum equals the full FFN for every B dividing H."""
+    rng = np.random.default_rng(2)
+    x, w_router, w_up, w_down = rand_layer(rng, 8, 48, 2, 2, T=16)
+    outs = [oracle.layer(x, w_router, w_up, w_down, B, Thresholds(alpha_fixed=1.0))[0]
+            for B in (2, 3, 4, 6, 8, 12)]
+    for o in outs[1:]:
+        np.testing.assert_allclose(o, outs[0], rtol=1e-12, atol=1e-14)
+
+
+def test_permuting_tokens_permutes_outputs(oracle_mod):
+    rng = np.random.default_rng(4)
+    x, w_router, w_up, w_down = rand_layer(rng, 16, 64, 4, 4, router_scale=4.0, T=80)
+    y, r = oracle.layer(x, w_router, w_up, w_down, 4)
+    perm = rng.permutation(80)
+    y2, r2 = oracle.layer(x[perm], w_router, w_up, w_down, 4)
+    assert np.array_equal(y2, y[perm])
+    assert np.array_equal(r2.shr_mask, r.shr_mask[perm]) and np.array_equal(r2.k, r.k[perm])
+
+
+def test_padding_tokens(oracle_mod):
+    rng = np.random.default_rng(6)
+    x, w_router, w_up, w_down = rand_layer(rng, 8, 32, 4, 4, T=20)
+    mask = (np.arange(20) % 3 != 0).astype(np.uint8)
+    x[mask == 0] = np.nan
+    y, r = oracle.layer(x, w_router, w_up, w_down, 4, mask=mask)
+    assert np.isfinite(y).all()
+    assert (y[mask == 0] == 0).all() and (r.b[mask == 0] == 0).all() and (r.k[mask == 0] == 0).all()
+    counts, tok, _ = oracle.groups(r, 4, 4, mask)
+    assert not set(tok.tolist()) & set(np.nonzero(mask == 0)[0].tolist())
+    assert counts.sum() == r.cb(4)[mask == 1].sum()
+
+
+def test_group_table_matches_decisions(oracle_mod):
+    """Each token appears in exactly C_B(t) groups (Eq. 35): the b shared
+    blocks of expert 0 and the B-b residual blocks of each of its k experts."""
+    rng = np.random.default_rng(8)
+    B, K = 8, 6
+    x, w_router, w_up, w_down = rand_layer(rng, 16, 64, K, B, router_scale=6.0, T=200)
+    _, r = oracle.layer(x, w_router, w_up, w_down, B)
+    counts, tok, w = oracle.groups(r, K, B)
+    assert np.bincount(tok, minlength=200).tolist() == r.cb(B).tolist()
+    start = np.concatenate([[0], np.cumsum(counts)])
+    em = r.expert_mask()
+    for g in range(len(counts)):
+        e, blk = divmod(g, B)
+        rows = tok[start[g]:start[g + 1]]
+        assert (np.diff(rows) > 0).all()  # increasing token order
+        for t, wt in zip(rows, w[start[g]:start[g + 1]]):
+            shared = (int(r.shr_mask[t]) >> blk) & 1
+            if e == 0:
+                assert shared and wt == r.alpha[t]
+            else:
+                assert not shared and (int(em[t]) >> (e - 1)) & 1
+                assert wt == r.s[t, e - 1]
+
+
+# --------------------------------------------------------------------------
+# Readings: ties, rounding of Eq. 19 and of the stored prototypes
+# --------------------------------------------------------------------------
+
+def test_ties_break_to_lower_index(oracle_mod):
+    d, K, B = 4, 4, 4
+    x = np.array([[1.0, 0.0, 0.0, 0.0]])
+    w_router = np.zeros((d, K + 1))
+    w_router[0, 2] = w_router[0, 3] = 1.0  # experts 1 and 2 tie on top
+    w_up = np.zeros((K + 1, 16, d))
+    w_up[0, :, 0] = 1.0  # all block priorities equal
+    w_down = np.zeros((K + 1, d, 16))
+    _, r = oracle.layer(x, w_router, w_up, w_down, B, Thresholds(alpha_fixed=0.5))
+    assert r.q[0, :2].tolist() == [1, 2] and r.q[0, 2:].tolist() == [0, 3]
+    assert int(r.shr_mask[0]) == 0b0011  # b = 2 of 4 equal priorities: blocks 0, 1
+
+
+@pytest.mark.parametrize("alpha,b", [(0.3125, 2), (0.4375, 4), (0.5625, 4), (0.6875, 6)])
+def test_round_half_to_even(oracle_mod, alpha, b):
+    """B alpha exactly halfway between integers (B = 8): round half to even."""
+    rng = np.random.default_rng(0)
+    x, w_router, w_up, w_down = rand_layer(rng, 4, 16, 2, 8, T=1)
+    _, r = oracle.layer(x, w_router, w_up, w_down, 8, Thresholds(alpha_fixed=alpha))
+    assert r.b[0] == b
+
+
+def test_prototype_rounding(oracle_mod):
+    """With M = 1 the prototype is the key itself, so the rounding to the
+    router's storage precision is seen directly: bf16 keeps 8 significant
+    bits, ties go to the even neighbour; fp32 is the IEEE single rounding."""
+    vals = np.array([1 + 2**-8, 1 + 3 * 2**-8, 1 + 2**-8 + 2**-30, -(1 + 2**-8),
+                     3.0, 0.1, 2**-130 * 1.5])
+    want_bf16 = np.array([1.0, 1 + 2**-6, 1 + 2**-7, -1.0, 3.0, 0.10009765625,
+                          2**-130 * 1.5])
+    w = np.zeros((len(vals), 1))
+    w[:, 0] = vals
+    mu = oracle.prototypes(w, len(vals), oracle.ROUND_BF16)[:, 0]
+    np.testing.assert_array_equal(mu, want_bf16)
+    mu32 = oracle.prototypes(w, len(vals), oracle.ROUND_F32)[:, 0]
+    np.testing.assert_array_equal(mu32, vals.astype(np.float32).astype(np.float64))
+    # The mean over a block is exact before the single rounding.
+    w2 = np.array([[1.0], [2**-9], [0.0], [0.0]])  # mean of first block = (1 + 2^-9)/2
+    mu2 = oracle.prototypes(w2, 2, oracle.ROUND_BF16)[:, 0]
+    assert mu2[0] == 0.5  # (1+2^-9)/2 = 0.5 + 2^-10, below the halfway point 0.5 + 2^-9
+
+
+def test_margins_flag_near_ties(oracle_mod):
+    """Margin (iv) is p_k - p_{k+1}; margin (i) is the distance of B alpha to
+    the nearest half-integer, divided by B."""
+    rng = np.random.default_rng(12)
+    x, w_router, w_up, w_down = rand_layer(rng, 16, 64, 8, 8, router_scale=2.0, T=300)
+    _, r = oracle.layer(x, w_router, w_up, w_down, 8)
+    for t in range(300):
+        kk = r.k[t]
+        if kk < 8:
+            assert r.margin[t, 3] == pytest.approx(r.p[t, kk - 1] - r.p[t, kk], abs=1e-15)
+        frac = 8 * r.alpha[t] - math.floor(8 * r.alpha[t])
+        assert r.margin[t, 0] == pytest.approx(abs(frac - 0.5) / 8, abs=1e-15)
+        assert (r.margin[t] >= 0).all()
