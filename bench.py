@@ -1,0 +1,370 @@
+#!/usr/bin/env python
+"""Benchmark of the UniF-MoE layer forward pass on GB300.
+
+One step = one forward of the whole layer (router, permute, grouped up and
+down GEMMs, combine; Sec. III, Eqs. 16-30) over one batch of seeded
+synthetic tokens. Default workload: ViT-S-like vision tokens (64 images x 197
+tokens, d=384, H=1536 in 8 blocks, 8 upcycled residual experts + 1 shared
+expert, bf16), the stand-in for the paper's DeiT-S/DomainBed setting.
+
+Prints one JSON line (rank 0). Multi-GPU (torchrun): every rank runs its own
+batch (weak scaling, no data-path collective); value = tokens of all ranks /
+max over ranks of the timed device time.
+
+--impl reference times the CPU oracle (the plain fp64 restatement of the
+paper) on the host cores instead, on bounded token samples of the same
+workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "UniF-MoE layer fwd tokens/s & activated TFLOP/s (% of GB300 bf16 peak), 1 GPU"
+UNIT = "tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+KERNELS_PER_FORWARD = 7  # router, count, scan, scatter, up GEMM, down GEMM, combine
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload_desc(s, T_valid):
+    return {"workload": "%s: %d tokens (%d valid), d=%d, H=%d in B=%d blocks of %d, K=%d residual "
+                        "experts + 1 shared, %s" % (s.name, s.tokens, T_valid, s.d_model, s.d_ff,
+                                                    s.n_blocks, s.block_width, s.n_experts, s.dtype),
+            "tokens": s.tokens, "valid_tokens": T_valid, "d_model": s.d_model, "d_ff": s.d_ff,
+            "n_blocks": s.n_blocks, "n_experts": s.n_experts,
+            "thresholds": "adaptive (Eqs. 18-27)" if math.isnan(s.beta_fixed) else
+                          "beta fixed %.2f" % s.beta_fixed}
+
+
+# ----------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, interval_ms=50):
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", "clocks_bench.csv")
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", str(interval_ms)],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self, gpu_index=0):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9 or not parts[0].isdigit() or int(parts[0]) != gpu_index:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, v in zip(("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                                "sw_power_cap"), parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------- oracle
+
+class OracleRunner:
+    """The CPU oracle, as it stands, on the first `tokens` token slots of a
+    workload (inputs converted to fp64 once, outside the timing)."""
+
+    def __init__(self, wl):
+        import oracle
+        s = wl.spec
+        self.o, self.wl, self.s = oracle, wl, s
+        self.rm = oracle.ROUND_BF16 if s.dtype == "bf16" else oracle.ROUND_F32
+        self.th = oracle.Thresholds(s.tau, s.alpha_fixed, s.beta_fixed, s.topk_fixed,
+                                    s.prefix_blocks)
+        self.wu, self.wd = oracle._f64(wl.w_up), oracle._f64(wl.w_down)
+        self.wr, self.xa = oracle._f64(wl.w_router), oracle._f64(wl.x)
+
+    def time(self, tokens, repeat=1):
+        m = None if self.wl.mask is None else self.wl.mask[:tokens]
+        x = self.xa[:tokens]
+        t0 = time.perf_counter()
+        for _ in range(repeat):
+            self.o.layer(x, self.wr, self.wu, self.wd, self.s.n_blocks, self.th, m,
+                         self.wl.router_bias, self.rm)
+        dt = time.perf_counter() - t0
+        valid = tokens if m is None else int(m.sum())
+        return valid * repeat / dt, dt, valid * repeat
+
+
+def oracle_cores():
+    import oracle
+    return oracle.threads()
+
+
+# ----------------------------------------------------------------- main
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="vit_s")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=50)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    import torch
+    import workloads
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    s = workloads.spec(args.workload)
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        run_reference(args, s)
+        return 0
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_10392_gb300 import Layer
+
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+
+    # every rank draws its own batch of tokens (same layer weights)
+    w_router, w_up, w_down, bias = workloads.make_weights(s)
+    x, mask = workloads.make_tokens(s, w_router, seed=None if rank == 0 else s.index * 1000 + 1 + 7919 * rank)
+    T = s.tokens
+    T_valid = T if mask is None else int(mask.sum())
+    layer = Layer(s.d_model, s.d_ff, s.n_experts, s.n_blocks, dtype=s.dtype, max_tokens=T,
+                  tau=s.tau, alpha_fixed=s.alpha_fixed, beta_fixed=s.beta_fixed,
+                  topk_fixed=s.topk_fixed, prefix_blocks=s.prefix_blocks)
+    layer.load_weights(w_router.to(dev), w_up.to(dev), w_down.to(dev),
+                       None if bias is None else bias.to(dev))
+    xd = x.to(dev)
+    md = None if mask is None else mask.to(dev)
+    out = torch.empty_like(xd)
+    bcnt = torch.empty(T, dtype=torch.int32, device=dev)
+    kcnt = torch.empty(T, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > 129 MB L2
+
+    for _ in range(args.warmup):
+        layer.forward(xd, out=out, mask=md, shared_counts=bcnt, residual_counts=kcnt)
+    torch.cuda.synchronize(dev)
+    if layer.sync_status() != 0:
+        raise RuntimeError("device status word set during warm-up")
+    b_h, k_h = bcnt.cpu().long(), kcnt.cpu().long()
+    B, M, d = s.n_blocks, s.block_width, s.d_model
+    cb = b_h + k_h * (B - b_h)
+    if mask is not None:
+        cb = cb * mask.long()
+    sum_cb = int(cb.sum())
+    gemm_flops = 2.0 * d * M * sum_cb  # one of the two grouped GEMMs (Eq. 16)
+    act_flops = 2.0 * gemm_flops       # activated FLOPs of the layer (Eq. 35 blocks)
+
+    K = args.steps
+    mk = lambda: torch.cuda.Event(enable_timing=True)
+    starts = [mk() for _ in range(K)]
+    ends = [mk() for _ in range(K)]
+    stage_ev = [[mk() for _ in range(6)] for _ in range(K)]
+    for evs in stage_ev:  # create the CUDA events
+        for e in evs:
+            e.record(stream)
+    torch.cuda.synchronize(dev)
+
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    sampler = ClockSampler() if rank == 0 else None
+    for i in range(K):
+        flush.zero_()  # L2 flush between steps (outside the timed events)
+        layer.set_stage_events(stage_ev[i])
+        starts[i].record(stream)
+        layer.forward(xd, out=out, mask=md, shared_counts=bcnt, residual_counts=kcnt)
+        ends[i].record(stream)
+    torch.cuda.synchronize(dev)
+    if dist:
+        dist.barrier()
+    clocks = sampler.stop(0) if sampler else None
+    layer.set_stage_events(None)
+    if layer.sync_status() != 0:
+        raise RuntimeError("device status word set during the timed region")
+
+    step_ms = [starts[i].elapsed_time(ends[i]) for i in range(K)]
+    total_ms = sum(step_ms)
+    names = ["router", "permute", "up_gemm", "down_gemm", "combine"]
+    stage_ms = {n: statistics.fmean(stage_ev[i][j].elapsed_time(stage_ev[i][j + 1]) for i in range(K))
+                for j, n in enumerate(names)}
+    if dist:
+        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+
+    # e2e through the C ABI with host buffers (copies inside the timed region)
+    xh = x.pin_memory()
+    oh = torch.empty_like(xh).pin_memory()
+    mh = None if mask is None else mask.pin_memory()
+    bh = torch.empty(T, dtype=torch.int32).pin_memory()
+    kh = torch.empty(T, dtype=torch.int32).pin_memory()
+    for _ in range(3):
+        layer.forward_host(xh, oh, mh, bh, kh)
+    e2e_ms = []
+    for _ in range(args.e2e_steps):
+        a, b = mk(), mk()
+        a.record(stream)
+        layer.forward_host(xh, oh, mh, bh, kh)
+        b.record(stream)
+        b.synchronize()
+        e2e_ms.append(a.elapsed_time(b))
+    elt = 2 if s.dtype == "bf16" else 4
+    h2d = T * d * elt + (0 if mask is None else T)
+    d2h = T * d * elt + 2 * 4 * T
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return 0
+
+    peaks, peak_kind = load_peaks()
+    ms = total_ms / K
+    value = world * T_valid / (ms / 1e3)
+    tflops = act_flops / (ms / 1e3) / 1e12
+    peak_tf = peaks["bf16_tflops_sustained"]
+    hbm = peaks["hbm_gbs"]
+    # roofline of the dominant kernel (the larger grouped GEMM), timed live
+    dom = "up_gemm" if stage_ms["up_gemm"] >= stage_ms["down_gemm"] else "down_gemm"
+    ach = gemm_flops / (stage_ms[dom] / 1e3) / 1e12
+    traffic = None
+    tr_path = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tr_path):
+        tr = json.load(open(tr_path)).get(s.name, {})
+        traffic = tr.get(dom)
+    router_bytes = T * d * elt + T * (4 * 3 + 8 * 2 + 12 * s.n_experts)
+    combine_bytes = T * d * (4 + elt)
+    permute_bytes = sum_cb * 8
+    stages = {
+        "router": {"ms": stage_ms["router"], "GB/s": router_bytes / stage_ms["router"] / 1e6},
+        "permute": {"ms": stage_ms["permute"], "GB/s": permute_bytes / stage_ms["permute"] / 1e6},
+        "up_gemm": {"ms": stage_ms["up_gemm"],
+                    "TFLOP/s": gemm_flops / stage_ms["up_gemm"] / 1e9},
+        "down_gemm": {"ms": stage_ms["down_gemm"],
+                      "TFLOP/s": gemm_flops / stage_ms["down_gemm"] / 1e9},
+        "combine": {"ms": stage_ms["combine"], "GB/s": combine_bytes / stage_ms["combine"] / 1e6},
+    }
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": s.dtype, "data": "synthetic (seeded; stands in for DeiT-S "
+        "tokens on DomainBed, which are not available)",
+        "config": dict(workload_desc(s, T_valid), parallelism="dp%d (independent batches)" % world,
+                       l2="flushed between steps (512 MB write outside the timed events)"),
+        "activated_tflops": tflops,
+        "activated_frac_of_bf16_peak": tflops / peak_tf,
+        "mean_C_B": sum_cb / T_valid,
+        "roofline": {"bound": "tensor", "kernel": dom, "achieved": ach, "peak": peak_tf,
+                     "unit": "TFLOP/s", "frac": ach / peak_tf, "traffic": traffic,
+                     "peak_kind": "%s bf16 sustained" % peak_kind},
+        "stages": stages,
+        "hbm_peak_gbs": hbm,
+        "e2e": {"value": T_valid / (statistics.fmean(e2e_ms) / 1e3), "unit": UNIT,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": statistics.fmean(e2e_ms)},
+        "gpu_launches": KERNELS_PER_FORWARD * K,
+        "clocks": clocks,
+    }
+    if not args.no_cpu_baseline and world >= 1:
+        tokens = min(T, 2048)
+        wl = workloads.Workload(s, w_router, w_up, w_down, bias, x, mask)
+        v, dt, n = OracleRunner(wl).time(tokens)
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": oracle_cores(), "kind": "oracle",
+                                "sample": "first %d token slots of the same workload, one pass "
+                                          "(%d valid tokens, %.1f s)" % (tokens, n, dt)}
+    print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_reference(args, s):
+    """The reference arm: the CPU oracle as it stands, on the host cores, each
+    step a bounded token sample of the same workload."""
+    import workloads
+    wl = workloads.make_workload(s)
+    runner = OracleRunner(wl)
+    # size the per-step sample so that warm-up + steps stay within ~2 minutes
+    probe_tokens = 64
+    v, dt, _ = runner.time(probe_tokens)
+    budget = 120.0 / (args.steps + args.warmup)
+    tokens = int(max(16, min(s.tokens, probe_tokens * budget / max(dt, 1e-6))))
+    for _ in range(args.warmup):
+        runner.time(tokens)
+    total_t, total_n = 0.0, 0
+    for _ in range(args.steps):
+        _, dt, n = runner.time(tokens)
+        total_t += dt
+        total_n += n
+    value = total_n / total_t
+    T_valid = s.tokens if wl.mask is None else int(wl.mask.sum())
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total_t / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded)",
+        "config": dict(workload_desc(s, T_valid), parallelism="host cores"),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle_cores(), "kind": "oracle",
+                         "sample": "first %d token slots of the workload per step" % tokens},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,186 @@
+/*
+ * unif_moe.h - C ABI of the GB300 (sm_103a) UniF-MoE layer forward pass.
+ *
+ * The layer ("Share First, Route What Remains", Sec. III) holds one shared
+ * expert and K residual experts, each an FFN of width H = d_ff split into B
+ * aligned blocks of width M = H / B (Sec. III-A, Eq. 16). For every token x:
+ *   alpha = tau + (1 - 2 tau) sigmoid(x W_shr), tau = (B-1)/B^2    (Eq. 18)
+ *   b     = round(B alpha) shared blocks                          (Eq. 19)
+ *   I_shr = the b blocks of largest priority u_b = x mu_b, where
+ *           mu_b is the mean of the shared keys of block b         (Eqs. 20-23)
+ *   s     = softmax(x W_g) over the K residual experts, sorted as
+ *           p_1 >= ... >= p_K with experts q_1..q_K                (Eqs. 24-25)
+ *   k     = smallest n with p_1 + ... + p_n >= beta = 1 - alpha    (Eqs. 26-27)
+ *   y     = alpha * sum_{b in I_shr} E_shr^(b)(x)
+ *           + sum_{i<=k} p_i * sum_{b not in I_shr} E_{q_i}^(b)(x)   (Eqs. 28-30)
+ * and it activates C_B = b + k (B - b) blocks (Eq. 35).
+ *
+ * Conventions for every call below:
+ *   - Pointers named *_dev are device pointers; the caller owns them. Pointers
+ *     named *_host are host pointers (pinned memory gives the fastest copies).
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream). Work is
+ *     enqueued on it; calls return without synchronising unless stated.
+ *   - Return value: UNIF_MOE_OK (0) or a negative UNIF_MOE_ERR_* code; the
+ *     message of the last failure on the calling thread is returned by
+ *     unif_moe_last_error().
+ *   - Rows are row-major and densely packed; element type is the layer dtype
+ *     (float for UNIF_MOE_F32, bfloat16 for UNIF_MOE_BF16) unless stated.
+ *   - Device pointers handed to unif_moe_forward must be 16-byte aligned.
+ * A handle may be used from one host thread at a time; forwards on one
+ * handle share its workspace, so they must be ordered on a single stream.
+ */
+#ifndef UNIF_MOE_H
+#define UNIF_MOE_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define UNIF_MOE_API __attribute__((visibility("default")))
+#else
+#define UNIF_MOE_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct unif_moe_layer* unif_moe_t;
+
+enum {
+  UNIF_MOE_OK = 0,
+  UNIF_MOE_ERR_ARG = -1,      /* null or misaligned pointer, value out of range */
+  UNIF_MOE_ERR_SHAPE = -2,    /* layer shape the kernels do not support */
+  UNIF_MOE_ERR_CAPACITY = -3, /* T larger than max_tokens of the handle */
+  UNIF_MOE_ERR_CUDA = -4,     /* a CUDA runtime or driver call failed */
+  UNIF_MOE_ERR_TIMEOUT = -5,  /* a kernel gave up waiting (see sync_status) */
+  UNIF_MOE_ERR_STATE = -6     /* call out of order, e.g. forward before load */
+};
+
+typedef enum { UNIF_MOE_F32 = 0, UNIF_MOE_BF16 = 1 } unif_moe_dtype;
+
+/* Routing thresholds. NaN / 0 select the paper's adaptive rule; the other
+ * values are the non-adaptive replacements the paper ablates (Table IV). */
+typedef struct {
+  float tau;         /* NaN: (B-1)/B^2 (Eq. 18); else this tau */
+  float alpha_fixed; /* NaN: adaptive alpha (Eq. 18); else this constant alpha,
+                        which sets b (Eq. 19) and the shared weight */
+  float beta_fixed;  /* NaN: beta = 1 - alpha (Eq. 26); else this constant
+                        cumulative-mass threshold theta */
+  int topk_fixed;    /* 0: cumulative count (Eq. 27); else k = topk_fixed */
+  int prefix_blocks; /* 0: TopK of prototype priorities (Eq. 22); 1: the
+                        first b blocks */
+} unif_moe_thresholds;
+
+/* Fills *th with the paper's adaptive settings (all NaN / 0). */
+UNIF_MOE_API void unif_moe_default_thresholds(unif_moe_thresholds* th);
+
+/* Creates a layer (Sec. III-A): d_model = d, d_ff = H, n_experts = K residual
+ * experts (one shared expert is added), n_blocks = B, max_tokens = largest T
+ * a forward will be given. th may be NULL (adaptive defaults).
+ * Limits: 2 <= B <= 64, 1 <= K <= 64, H % B == 0, d % 8 == 0; for
+ * UNIF_MOE_BF16 also d % 64 == 0 and M = H/B a multiple of 64.
+ * Device workspace for max_tokens is allocated here, sized for the largest
+ * possible C_B (Eq. 35) under th; nothing is allocated by later calls.
+ * Errors: ERR_ARG (out == NULL, bad values), ERR_SHAPE, ERR_CUDA (allocation). */
+UNIF_MOE_API int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n_blocks,
+                    const unif_moe_thresholds* th, unif_moe_dtype dtype, int max_tokens);
+
+/* Loads weights from device memory (copied into the handle; the caller may
+ * free its buffers once `stream` has passed this call):
+ *   w_router_dev [d][K+1]    column 0 = W_shr, columns 1..K = W_g (Eq. 17)
+ *   w_up_dev     [K+1][H][d] expert 0 = shared; row h = key K_e[:, h] (Eq. 4)
+ *   w_down_dev   [K+1][d][H] column h = value V_e[h, :] (Eq. 4)
+ *   router_bias_dev [K+1] float or NULL: added to the router logits. The
+ *                paper has no bias (Sec. II-A); NULL reproduces it.
+ * Also forms the block prototypes mu_b (Eq. 20) from the shared keys, exactly
+ * (fp64 sums) and rounded once to the layer dtype.
+ * Errors: ERR_ARG (NULL weight), ERR_CUDA. */
+UNIF_MOE_API int unif_moe_load_weights(unif_moe_t h, const void* w_router_dev, const void* w_up_dev,
+                          const void* w_down_dev, const float* router_bias_dev, void* stream);
+
+/* One forward pass over T tokens (Eqs. 17-30):
+ *   x_dev   [T][d] input tokens
+ *   out_dev [T][d] output y (layer dtype); padding tokens give 0
+ *   token_mask_dev [T] uint8 or NULL: 0 marks padding, which takes no routing
+ *                decision, no expert work and outputs 0
+ *   shared_counts_dev [T] int32 or NULL: receives b(x) (Eq. 19), 0 for padding
+ *   residual_counts_dev [T] int32 or NULL: receives k(x) (Eq. 27), 0 for padding
+ * T = 0 is a no-op. The decisions of the last forward stay in the handle for
+ * unif_moe_get_routing / unif_moe_get_groups.
+ * Errors: ERR_ARG, ERR_CAPACITY (T > max_tokens), ERR_STATE (no weights),
+ * ERR_CUDA (launch failure). Kernel timeouts surface through sync_status. */
+UNIF_MOE_API int unif_moe_forward(unif_moe_t h, const void* x_dev, void* out_dev, int T,
+                     const uint8_t* token_mask_dev, int32_t* shared_counts_dev,
+                     int32_t* residual_counts_dev, void* stream);
+
+/* The same forward from host buffers: copies x_host (and token_mask_host if
+ * not NULL) to the handle's device staging buffers, runs the forward, copies
+ * the output to out_host and the counts to shared_counts_host /
+ * residual_counts_host (each may be NULL), and synchronises `stream` before
+ * returning. Host buffers should be pinned for asynchronous copies. */
+UNIF_MOE_API int unif_moe_forward_host(unif_moe_t h, const void* x_host, void* out_host, int T,
+                          const uint8_t* token_mask_host, int32_t* shared_counts_host,
+                          int32_t* residual_counts_host, void* stream);
+
+/* Copies the decisions of the last forward (T tokens) to device buffers; any
+ * pointer may be NULL:
+ *   alpha_dev [T] float          shared demand alpha (Eq. 18)
+ *   shared_mask_dev [T] uint64   bit b set = block b in I_shr (Eq. 22)
+ *   expert_mask_dev [T] uint64   bit j set = residual expert j selected
+ *   q_dev [T][K] int32           experts by decreasing affinity (Eq. 25)
+ *   p_dev [T][K] float           their affinities p_1 >= ... >= p_K
+ * Synchronises `stream`. Errors: ERR_ARG, ERR_STATE (no forward yet). */
+UNIF_MOE_API int unif_moe_get_routing(unif_moe_t h, float* alpha_dev, uint64_t* shared_mask_dev,
+                         uint64_t* expert_mask_dev, int32_t* q_dev, float* p_dev,
+                         void* stream);
+
+/* Copies the (expert, block) group table of the last forward to host memory.
+ * Group g = e*B + b for e = 0 (shared expert) or e = 1+j (residual expert j),
+ * G = (K+1)*B groups. counts_host [G] receives each group's row count; the
+ * rows of group g are listed in increasing token order at
+ * [offsets_host[g], offsets_host[g] + counts_host[g]) of row_token_host /
+ * row_weight_host (weight = alpha for e = 0, p_i for e = 1+q_i). offsets_host
+ * [G+1] (offsets_host[G] = total padded rows). Rows past a group's count up to
+ * the next offset are padding (token -1). *n_rows receives offsets_host[G];
+ * row buffers must hold max_rows entries, where unif_moe_max_rows() gives
+ * the bound. Synchronises `stream`. */
+UNIF_MOE_API int unif_moe_get_groups(unif_moe_t h, int32_t* counts_host, int32_t* offsets_host,
+                        int32_t* row_token_host, float* row_weight_host, int64_t* n_rows,
+                        void* stream);
+
+/* Optional stage timing. events points to 6 cudaEvent_t handles created by
+ * the caller (with timing enabled); each later forward records them on its
+ * stream at the stage boundaries: [0] before the router, [1] after the
+ * router (Eqs. 17-27), [2] after the permute (grouping of Eqs. 28-29),
+ * [3] after the up-projection GEMM + GeLU, [4] after the down-projection
+ * GEMM (Eq. 16), [5] after the combine (Eq. 30). NULL stops the recording.
+ * The caller keeps the events alive while they are set. */
+UNIF_MOE_API int unif_moe_set_stage_events(unif_moe_t h, void* const* events);
+
+/* Upper bound on group-table rows (padded) of a forward at max_tokens. */
+UNIF_MOE_API int64_t unif_moe_max_rows(unif_moe_t h);
+
+/* Waits for `stream`, then reads and clears the handle's device status word.
+ * Returns UNIF_MOE_OK, UNIF_MOE_ERR_TIMEOUT if a kernel abandoned a bounded
+ * wait since the last call, or UNIF_MOE_ERR_CUDA. */
+UNIF_MOE_API int unif_moe_sync_status(unif_moe_t h, void* stream);
+
+/* Diagnostic: launches one kernel that waits, with its bounded wait, on a
+ * barrier nothing ever completes, giving up after about `timeout_us`
+ * microseconds (capped at 1 s) and recording ERR_TIMEOUT in the status word
+ * exactly as the GEMM kernels would. Used to test the timeout path without
+ * hanging the GPU. */
+UNIF_MOE_API int unif_moe_selftest_timeout(unif_moe_t h, int timeout_us, void* stream);
+
+/* Frees the handle and its device memory (synchronises the device first).
+ * NULL is ignored. */
+UNIF_MOE_API void unif_moe_destroy(unif_moe_t h);
+
+/* Message of the last error on the calling thread ("" if none). */
+UNIF_MOE_API const char* unif_moe_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* UNIF_MOE_H */

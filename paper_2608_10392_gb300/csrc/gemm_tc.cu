@@ -1,0 +1,504 @@
+// Grouped expert GEMMs on the sm_103a tensor cores (tcgen05 + TMEM, fed by
+// TMA) for bf16 layers.
+//
+// Every (expert e, block b) pair of Eqs. 28-29 is one group; the permute step
+// lists each group's rows (token, weight) contiguously, padded to 128-row
+// tiles. Two persistent, warp-specialised kernels walk that tile list:
+//   up   : h[row]  = GeLU(x[tok(row)] K_e[:, H_b])        128 x M  per tile
+//   down : y[tok] += w(row) * h[row] V_e[H_b, :]          128 x d  per tile
+// (Eq. 16 split at the activation; w = alpha for the shared expert and p_i
+// for residual expert q_i, Eq. 30).
+//
+// Roles inside one CTA (one CTA per SM, 384 threads):
+//   warp 0      TMA producer: A tile (gathered x rows with tile::gather4, or
+//               a plain 2-D tile of h) and B tile (a weight slice) per stage
+//   warp 1      TMEM allocator and MMA issuer (one lane): 128 x BN x 16
+//               kind::f16 MMAs, fp32 accumulators in TMEM
+//   warps 4-11  epilogue: tcgen05.ld of the accumulator, GeLU -> bf16 h
+//               (up), or weight-scale -> fp32 atomic add into y (down)
+// Shared-memory stages are a 4-deep ring (full/empty mbarriers); the TMEM
+// accumulator is double-buffered (2 x 256 columns) so the epilogue of one
+// tile overlaps the MMAs of the next.
+//
+// Operands use the 128-byte-swizzled K-major layout: a stage row holds 64
+// bf16 (128 bytes) of the reduction dimension, 8-row groups are 1024 bytes
+// apart, and the MMA's 16-element K steps advance the descriptor start
+// address by 32 bytes inside the swizzle atom.
+//
+// Every wait on an mbarrier is bounded; a wait that runs out records
+// kStatusTimeout in the handle's status word and the CTA unwinds.
+#include <stdio.h>
+
+#include "internal.cuh"
+
+namespace unif {
+namespace tc {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kStages = 4;
+constexpr int kThreads = 384;
+constexpr int kEpiWarps = 8;
+constexpr int kFirstEpiWarp = 4;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kAccStride = 256;  // TMEM columns per accumulator buffer
+constexpr int kMaxBN = 256;
+constexpr uint32_t kStageA = kBM * kBK * 2;      // 16 KB
+constexpr uint32_t kStageB = kMaxBN * kBK * 2;   // 32 KB
+constexpr size_t kSmemBytes = 1024 + kStages * (kStageA + kStageB) + 256;
+
+struct Params {
+  const int32_t* n_tiles;
+  const int32_t* tile_group;
+  const int32_t* tile_row0;
+  const int32_t* row_tok;
+  const float* row_w;
+  int n_sub;       // N sub-tiles per 128-row tile
+  int bn;          // N per sub-tile (multiple of 32, <= 256)
+  int num_kb;      // reduction steps of 64
+  int B, M, H, d;
+  __nv_bfloat16* h;  // up: [rows][M]
+  float* y32;        // down: [T][d]
+  int* status;
+  long long wait_limit;  // clock cycles before a wait gives up
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// ---- mbarrier ----
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0u;
+}
+
+// Bounded wait: gives up after `limit` cycles (or once another role of the
+// CTA has given up), recording the timeout in the status word.
+__device__ __noinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          int* status, long long limit) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (clock64() - t0 > limit) {
+      *abort_flag = 1;
+      atomicOr(status, kStatusTimeout);
+      return false;
+    }
+  }
+}
+
+// ---- TMA ----
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
+      : "memory");
+}
+__device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int col, int r0, int r1, int r2, int r3) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(col), "r"(r0), "r"(r1), "r"(r2),
+      "r"(r3)
+      : "memory");
+}
+
+// ---- tcgen05 ----
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+// 32 lanes x 16 consecutive 32-bit TMEM columns; thread i holds lane base+i.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32"
+      " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (stride-dimension offset), leading offset unused (1),
+// descriptor version 1 at bit 46, swizzle mode 2 (128 B) at bits 61-63.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) |
+         ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1),
+// A and B bf16 (bits 7-9 = 1, 10-12 = 1), both K-major, N>>3 at bits 17-22,
+// M>>4 at bits 24-28.
+__device__ __forceinline__ uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ float gelu_erf(float v) {
+  return 0.5f * v * (1.0f + erff(v * 0.70710678118654752f));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&p);
+}
+
+// MODE 0 = up-projection (+GeLU), MODE 1 = down-projection (+weighted add).
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sA = smem_u32(smem);
+  const uint32_t sB = sA + kStages * kStageA;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * (kStageA + kStageB));
+  const uint32_t bar0 = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
+  auto accf_bar = [&](int a) { return bar0 + 8u * (2 * kStages + a); };
+  auto acce_bar = [&](int a) { return bar0 + 8u * (2 * kStages + 2 + a); };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 4);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(accf_bar(a), 1);
+      mbar_init(acce_bar(a), kEpiWarps);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int n_items = p.n_tiles[0] * p.n_sub;
+  const uint32_t stage_bytes = kStageA + (uint32_t)p.bn * kBK * 2;
+
+  if (warp == 0) {
+    // ------------------------------ producer ------------------------------
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      const int tile = item / p.n_sub, ns = item % p.n_sub;
+      const int g = p.tile_group[tile], row0 = p.tile_row0[tile];
+      const int e = g / p.B, blk = g % p.B;
+      int tok[4] = {0, 0, 0, 0};
+      if (MODE == 0) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int t = p.row_tok[row0 + 4 * lane + j];
+          tok[j] = t < 0 ? 0 : t;  // padding rows read token 0; never reduced
+        }
+      }
+      // B rows: w_up viewed [(K+1)H][d] or w_down viewed [(K+1)d][H].
+      const int brow = (MODE == 0) ? e * p.H + blk * p.M + ns * p.bn : e * p.d + ns * p.bn;
+      for (int kb = 0; kb < p.num_kb; ++kb) {
+        bool w = true;
+        if (lane == 0) w = wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
+        ok = __shfl_sync(0xffffffffu, w, 0);
+        if (!ok) break;
+        if (lane == 0) mbar_expect_tx(full_bar(stage), stage_bytes);
+        __syncwarp();
+        const uint32_t a_dst = sA + stage * kStageA, b_dst = sB + stage * kStageB;
+        if (MODE == 0) {
+          tma_gather4(a_dst + lane * 512u, &tmA, full_bar(stage), kb * kBK, tok[0], tok[1], tok[2],
+                      tok[3]);
+          if (lane == 0) tma_load_2d(b_dst, &tmB, full_bar(stage), kb * kBK, brow);
+        } else if (lane == 0) {
+          tma_load_2d(a_dst, &tmA, full_bar(stage), kb * kBK, row0);
+          tma_load_2d(b_dst, &tmB, full_bar(stage), blk * p.M + kb * kBK, brow);
+        }
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------ MMA issuer ----------------------------
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(kBM, p.bn);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        if (!wait_bounded(acce_bar(acc), acc_phase ^ 1u, abort_flag, p.status, p.wait_limit)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)acc * kAccStride;
+        for (int kb = 0; kb < p.num_kb; ++kb) {
+          if (!wait_bounded(full_bar(stage), phase, abort_flag, p.status, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = sA + stage * kStageA, b_base = sB + stage * kStageB;
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            umma_bf16(d_tmem, sw128_desc(a_base + k * 32), sw128_desc(b_base + k * 32), idesc,
+                      (kb | k) != 0 ? 1u : 0u);
+          umma_commit(empty_bar(stage));
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        umma_commit(accf_bar(acc));
+        if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+      }
+    }
+    __syncwarp();
+  } else if (warp >= kFirstEpiWarp) {
+    // ------------------------------ epilogue ------------------------------
+    const int q = warp & 3;                        // TMEM lane quarter of this warp
+    const int half = (warp - kFirstEpiWarp) >> 2;  // which half of the columns
+    const int cols = p.bn / 2;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
+      const int tile = item / p.n_sub, ns = item % p.n_sub;
+      const int row0 = p.tile_row0[tile];
+      bool w = true;
+      if (lane == 0) w = wait_bounded(accf_bar(acc), acc_phase, abort_flag, p.status, p.wait_limit);
+      if (!__shfl_sync(0xffffffffu, w, 0)) break;
+      tc_fence_after();
+      const int row = row0 + q * 32 + lane;
+      const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)acc * kAccStride;
+      const int c_begin = half * cols;
+      if (MODE == 0) {
+        __nv_bfloat16* dst = p.h + (size_t)row * p.M + ns * p.bn + c_begin;
+        for (int c = 0; c < cols; c += 16) {
+          float v[16];
+          tmem_ld16(t_row + c_begin + c, v);
+          uint4 o0, o1;
+          o0.x = pack_bf16(gelu_erf(v[0]), gelu_erf(v[1]));
+          o0.y = pack_bf16(gelu_erf(v[2]), gelu_erf(v[3]));
+          o0.z = pack_bf16(gelu_erf(v[4]), gelu_erf(v[5]));
+          o0.w = pack_bf16(gelu_erf(v[6]), gelu_erf(v[7]));
+          o1.x = pack_bf16(gelu_erf(v[8]), gelu_erf(v[9]));
+          o1.y = pack_bf16(gelu_erf(v[10]), gelu_erf(v[11]));
+          o1.z = pack_bf16(gelu_erf(v[12]), gelu_erf(v[13]));
+          o1.w = pack_bf16(gelu_erf(v[14]), gelu_erf(v[15]));
+          *reinterpret_cast<uint4*>(dst + c) = o0;
+          *reinterpret_cast<uint4*>(dst + c + 8) = o1;
+        }
+      } else {
+        const int t = p.row_tok[row];
+        const float wt = p.row_w[row];
+        float* dst = p.y32 + (size_t)(t < 0 ? 0 : t) * p.d + ns * p.bn + c_begin;
+        for (int c = 0; c < cols; c += 16) {
+          float v[16];
+          tmem_ld16(t_row + c_begin + c, v);
+          if (t >= 0) {
+#pragma unroll
+            for (int j = 0; j < 16; j += 4)
+              atomicAdd(reinterpret_cast<float4*>(dst + c + j),
+                        make_float4(wt * v[j], wt * v[j + 1], wt * v[j + 2], wt * v[j + 3]));
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acce_bar(acc));
+      if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+// A kernel that waits, with the same bounded wait, on a barrier that nothing
+// completes: exercises the timeout path without hanging.
+__global__ void timeout_probe_kernel(int* status, long long limit) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    mbar_init(smem_u32(&bar), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    wait_bounded(smem_u32(&bar), 0u, &abort_flag, status, limit);
+  }
+}
+
+// ---- host side ----
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor map [rows][cols] (cols contiguous), 128-byte swizzle.
+bool encode_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
+               uint32_t box_cols, uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// N split into n_sub sub-tiles of bn columns: bn <= 256, bn % 32 == 0.
+bool pick_split(int n, int* bn, int* nsub) {
+  for (int s = 1; s <= n / 32; ++s) {
+    if (n % s) continue;
+    const int b = n / s;
+    if (b <= kMaxBN && b % 32 == 0) {
+      *bn = b;
+      *nsub = s;
+      return true;
+    }
+  }
+  return false;
+}
+
+long long g_wait_limit = 4000000000ll;  // ~2 s of SM clock
+
+}  // namespace tc
+
+int gemm_tc_setup(unif_moe_layer* L) {
+  if (!tc::pick_split(L->M, &L->up_bn, &L->up_nsub) ||
+      !tc::pick_split(L->d, &L->down_bn, &L->down_nsub)) {
+    set_error("no tensor-core tile split for M=%d or d=%d", L->M, L->d);
+    return UNIF_MOE_ERR_SHAPE;
+  }
+  const uint64_t E = (uint64_t)L->K + 1;
+  if (!tc::encode_2d(&L->tm_wup, L->w_up, L->d, E * L->H, tc::kBK, L->up_bn) ||
+      !tc::encode_2d(&L->tm_wdown, L->w_down, L->H, E * L->d, tc::kBK, L->down_bn) ||
+      !tc::encode_2d(&L->tm_h, L->ws.hbuf, L->M, (uint64_t)L->max_rows, tc::kBK, tc::kBM)) {
+    set_error("cuTensorMapEncodeTiled failed for the weight or activation maps");
+    return UNIF_MOE_ERR_CUDA;
+  }
+  for (auto fn : {tc::grouped_gemm_kernel<0>, tc::grouped_gemm_kernel<1>}) {
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)tc::kSmemBytes);
+    if (e != cudaSuccess) {
+      set_error("cudaFuncSetAttribute: %s", cudaGetErrorString(e));
+      return UNIF_MOE_ERR_CUDA;
+    }
+  }
+  return UNIF_MOE_OK;
+}
+
+cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
+                            cudaStream_t s) {
+  CUtensorMap tm_x;
+  if (!tc::encode_2d(&tm_x, x, L->d, (uint64_t)T, tc::kBK, 1)) return cudaErrorInvalidValue;
+  tc::Params p;
+  p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group; p.tile_row0 = L->ws.tile_row0;
+  p.row_tok = L->ws.row_tok; p.row_w = L->ws.row_w;
+  p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;
+  p.h = static_cast<__nv_bfloat16*>(L->ws.hbuf);
+  p.y32 = L->ws.y32;
+  p.status = L->ws.status;
+  p.wait_limit = tc::g_wait_limit;
+  // up: N = M (block width), reduction over d
+  p.n_sub = L->up_nsub; p.bn = L->up_bn; p.num_kb = L->d / tc::kBK;
+  tc::grouped_gemm_kernel<0><<<L->n_sm, tc::kThreads, tc::kSmemBytes, s>>>(tm_x, L->tm_wup, p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (mid) cudaEventRecord(mid, s);
+  // down: N = d, reduction over the block's M channels
+  p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
+  tc::grouped_gemm_kernel<1><<<L->n_sm, tc::kThreads, tc::kSmemBytes, s>>>(L->tm_h, L->tm_wdown, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_timeout_probe(unif_moe_layer* L, int timeout_us, cudaStream_t s) {
+  int khz = 0;
+  cudaError_t e = cudaDeviceGetAttribute(&khz, cudaDevAttrClockRate, L->device);
+  if (e != cudaSuccess) return e;
+  if (timeout_us > 1000000) timeout_us = 1000000;
+  if (timeout_us < 1) timeout_us = 1;
+  const long long limit = (long long)timeout_us * (long long)khz / 1000ll;
+  tc::timeout_probe_kernel<<<1, 32, 0, s>>>(L->ws.status, limit);
+  return cudaGetLastError();
+}
+
+}  // namespace unif

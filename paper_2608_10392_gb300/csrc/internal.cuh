@@ -1,0 +1,109 @@
+// Internal declarations shared by the translation units of the UniF-MoE
+// library: the handle layout and the kernel launchers. Not part of the ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/unif_moe.h"
+
+namespace unif {
+
+// Rows per tile of the grouped GEMMs (the tcgen05 MMA M).
+constexpr int kTileRows = 128;
+// Tokens per block in the router and in the permute kernels.
+constexpr int kRouterTokens = 64;
+constexpr int kChunkTokens = 256;
+// Status-word bits written by kernels.
+constexpr int kStatusTimeout = 1;
+constexpr int kStatusBadIndex = 2;
+
+struct Workspace {
+  // Routing records of the last forward (one entry per token slot).
+  float* alpha = nullptr;        // [T]
+  int32_t* b = nullptr;          // [T]
+  int32_t* k = nullptr;          // [T]
+  uint64_t* shr_mask = nullptr;  // [T]
+  uint64_t* exp_mask = nullptr;  // [T] selected residual experts
+  int32_t* q = nullptr;          // [T][K]
+  float* p = nullptr;            // [T][K] sorted affinities
+  float* s = nullptr;            // [T][K] affinities by expert index
+  // Group table.
+  int32_t* chunk_cnt = nullptr;  // [G][n_chunks]: counts, then exclusive offsets
+  int32_t* grp_cnt = nullptr;    // [G]
+  int32_t* grp_off = nullptr;    // [G+1] padded offsets
+  int32_t* n_tiles = nullptr;    // [1]
+  int32_t* tile_group = nullptr; // [max_tiles]
+  int32_t* tile_row0 = nullptr;  // [max_tiles]
+  int32_t* row_tok = nullptr;    // [max_rows] (-1 = padding row)
+  float* row_w = nullptr;        // [max_rows]
+  // Intermediate activations h = GeLU(x K_e[:, H_b]) per row, and the fp32
+  // output accumulator.
+  void* hbuf = nullptr;          // [max_rows][M] (layer dtype)
+  float* y32 = nullptr;          // [max_tokens][d]
+  // Host-buffer forward staging.
+  void* x_stage = nullptr;
+  void* out_stage = nullptr;
+  uint8_t* mask_stage = nullptr;
+  int32_t* b_stage = nullptr;
+  int32_t* k_stage = nullptr;
+  int* status = nullptr;         // device status word
+};
+
+}  // namespace unif
+
+struct unif_moe_layer {
+  int d = 0, H = 0, K = 0, B = 0, M = 0, G = 0;
+  int dtype = 0;
+  int max_tokens = 0;
+  unif_moe_thresholds th{};
+  float tau = 0.f;
+  int cb_max = 0;
+  int64_t max_rows = 0;
+  int64_t max_tiles = 0;
+  int max_chunks = 0;
+  int router_cols = 0;      // 1 + K + B
+  int router_cols_pad = 0;  // padded to 16
+  int n_sm = 0;
+  int device = 0;
+  bool loaded = false;
+  int last_T = -1;
+  // Weights (device, owned).
+  float* wr_t = nullptr;    // [router_cols_pad][d]: W_shr, W_g, mu_1..mu_B (fp32)
+  float* bias = nullptr;    // [K+1]
+  void* w_up = nullptr;     // [K+1][H][d]
+  void* w_down = nullptr;   // [K+1][d][H]
+  unif::Workspace ws;
+  // tcgen05 path: tensor maps of the weights and of h (encoded once).
+  CUtensorMap tm_wup;
+  CUtensorMap tm_wdown;
+  CUtensorMap tm_h;
+  int up_bn = 0, up_nsub = 0, down_bn = 0, down_nsub = 0;
+  // Optional caller-owned timing events recorded at the stage boundaries.
+  cudaEvent_t stage_ev[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+};
+
+namespace unif {
+
+void set_error(const char* fmt, ...);
+
+// Load time.
+cudaError_t launch_prototypes(unif_moe_layer* L, const void* w_router, const float* bias,
+                              cudaStream_t s);
+// Forward steps.
+cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
+                          int32_t* b_out, int32_t* k_out, cudaStream_t s);
+cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s);
+cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s);
+cudaError_t launch_gemms_simt(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
+                              cudaStream_t s);
+cudaError_t router_setup(unif_moe_layer* L);
+// tcgen05 path.
+int gemm_tc_setup(unif_moe_layer* L);  // tensor maps of weights and h; returns UNIF_MOE_* code
+cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
+                            cudaStream_t s);
+cudaError_t launch_timeout_probe(unif_moe_layer* L, int timeout_us, cudaStream_t s);
+
+}  // namespace unif

@@ -1,0 +1,397 @@
+// Host side of the UniF-MoE C ABI declared in include/unif_moe.h: argument
+// checks, workspace allocation at create time, and the launch sequence of a
+// forward pass
+//   router (Eqs. 17-27) -> permute (groups of Eqs. 28-29) ->
+//   grouped up/down GEMMs (Eq. 16) -> combine (Eq. 30).
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <new>
+
+#include "internal.cuh"
+
+namespace unif {
+
+static thread_local char g_err[512] = "";
+
+void set_error(const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+}
+
+}  // namespace unif
+
+using unif::set_error;
+
+namespace {
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+    else prev = -1;
+  }
+  ~DeviceGuard() {
+    if (prev >= 0) cudaSetDevice(prev);
+  }
+};
+
+#define CK(call)                                                              \
+  do {                                                                        \
+    cudaError_t e_ = (call);                                                  \
+    if (e_ != cudaSuccess) {                                                  \
+      set_error("%s failed: %s", #call, cudaGetErrorString(e_));              \
+      return UNIF_MOE_ERR_CUDA;                                               \
+    }                                                                         \
+  } while (0)
+
+template <typename T>
+int dalloc(T** p, size_t count) {
+  *p = nullptr;
+  if (count == 0) count = 1;
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), sizeof(T) * count);
+  if (e != cudaSuccess) {
+    set_error("cudaMalloc of %zu bytes failed: %s", sizeof(T) * count, cudaGetErrorString(e));
+    return UNIF_MOE_ERR_CUDA;
+  }
+  return UNIF_MOE_OK;
+}
+
+void free_all(unif_moe_layer* L) {
+  void* ptrs[] = {L->wr_t, L->bias, L->w_up, L->w_down, L->ws.alpha, L->ws.b, L->ws.k,
+                  L->ws.shr_mask, L->ws.exp_mask, L->ws.q, L->ws.p, L->ws.s, L->ws.chunk_cnt,
+                  L->ws.grp_cnt, L->ws.grp_off, L->ws.n_tiles, L->ws.tile_group,
+                  L->ws.tile_row0, L->ws.row_tok, L->ws.row_w, L->ws.hbuf, L->ws.y32,
+                  L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
+                  L->ws.k_stage, L->ws.status};
+  for (void* q : ptrs)
+    if (q) cudaFree(q);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t elt_size(const unif_moe_layer* L) { return L->dtype == UNIF_MOE_BF16 ? 2 : 4; }
+
+}  // namespace
+
+extern "C" {
+
+void unif_moe_default_thresholds(unif_moe_thresholds* th) {
+  if (!th) return;
+  th->tau = NAN;
+  th->alpha_fixed = NAN;
+  th->beta_fixed = NAN;
+  th->topk_fixed = 0;
+  th->prefix_blocks = 0;
+}
+
+const char* unif_moe_last_error(void) { return unif::g_err; }
+
+int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n_blocks,
+                    const unif_moe_thresholds* th, unif_moe_dtype dtype, int max_tokens) {
+  unif::g_err[0] = 0;
+  if (!out) { set_error("out is NULL"); return UNIF_MOE_ERR_ARG; }
+  *out = nullptr;
+  if (dtype != UNIF_MOE_F32 && dtype != UNIF_MOE_BF16) { set_error("bad dtype"); return UNIF_MOE_ERR_ARG; }
+  if (d_model <= 0 || d_ff <= 0 || n_experts < 1 || n_experts > 64 || n_blocks < 2 ||
+      n_blocks > 64 || max_tokens < 1) {
+    set_error("bad sizes: d=%d H=%d K=%d B=%d max_tokens=%d (need K in [1,64], B in [2,64])",
+              d_model, d_ff, n_experts, n_blocks, max_tokens);
+    return UNIF_MOE_ERR_ARG;
+  }
+  if (d_ff % n_blocks != 0 || d_model % 8 != 0) {
+    set_error("need d_ff %% n_blocks == 0 and d_model %% 8 == 0");
+    return UNIF_MOE_ERR_SHAPE;
+  }
+  const int M = d_ff / n_blocks;
+  if (dtype == UNIF_MOE_BF16 && (d_model % 64 != 0 || M % 64 != 0)) {
+    set_error("bf16 layers need d_model %% 64 == 0 and block width %% 64 == 0 (d=%d, M=%d)",
+              d_model, M);
+    return UNIF_MOE_ERR_SHAPE;
+  }
+  unif_moe_thresholds t;
+  unif_moe_default_thresholds(&t);
+  if (th) t = *th;
+  if (t.topk_fixed < 0 || t.topk_fixed > n_experts) {
+    set_error("topk_fixed=%d outside [0, K]", t.topk_fixed);
+    return UNIF_MOE_ERR_ARG;
+  }
+  if (!isnan(t.alpha_fixed) && !(t.alpha_fixed >= 0.f && t.alpha_fixed <= 1.f)) {
+    set_error("alpha_fixed outside [0, 1]");
+    return UNIF_MOE_ERR_ARG;
+  }
+  if (!isnan(t.tau) && !(t.tau >= 0.f && t.tau <= 0.5f)) {
+    set_error("tau outside [0, 1/2]");
+    return UNIF_MOE_ERR_ARG;
+  }
+
+  unif_moe_layer* L = new (std::nothrow) unif_moe_layer();
+  if (!L) { set_error("out of host memory"); return UNIF_MOE_ERR_ARG; }
+  L->d = d_model; L->H = d_ff; L->K = n_experts; L->B = n_blocks; L->M = M;
+  L->G = (n_experts + 1) * n_blocks;
+  L->dtype = dtype; L->max_tokens = max_tokens; L->th = t;
+  L->tau = isnan(t.tau) ? (float)((double)(n_blocks - 1) / ((double)n_blocks * n_blocks)) : t.tau;
+  const int kmax = t.topk_fixed > 0 ? t.topk_fixed : n_experts;
+  L->cb_max = kmax * n_blocks;  // C_B = b + k (B - b) <= k B for every b >= 0 (Eq. 35)
+  const int64_t rows = (int64_t)max_tokens * L->cb_max + (int64_t)L->G * (unif::kTileRows - 1);
+  L->max_rows = (rows + unif::kTileRows - 1) / unif::kTileRows * unif::kTileRows;
+  if (L->max_rows >= (int64_t)1 << 31) {
+    set_error("max_tokens=%d needs %lld group rows, above the int32 row index", max_tokens,
+              (long long)L->max_rows);
+    delete L;
+    return UNIF_MOE_ERR_CAPACITY;
+  }
+  L->max_tiles = L->max_rows / unif::kTileRows;
+  L->max_chunks = (max_tokens + unif::kChunkTokens - 1) / unif::kChunkTokens;
+  L->router_cols = 1 + n_experts + n_blocks;
+  L->router_cols_pad = (L->router_cols + 15) / 16 * 16;
+  if (cudaGetDevice(&L->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&L->n_sm, cudaDevAttrMultiProcessorCount, L->device) != cudaSuccess) {
+    set_error("no CUDA device");
+    delete L;
+    return UNIF_MOE_ERR_CUDA;
+  }
+  int major = 0, minor = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, L->device);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, L->device);
+  if (major != 10 || minor != 3) {
+    set_error("this library is built for sm_103a (GB300); device is sm_%d%d", major, minor);
+    delete L;
+    return UNIF_MOE_ERR_CUDA;
+  }
+  const size_t es = elt_size(L);
+  const size_t T = (size_t)max_tokens, K = (size_t)n_experts, E = K + 1;
+  unif::Workspace& w = L->ws;
+  int rc = UNIF_MOE_OK;
+#define ALLOC(ptr, n)                          \
+  if (rc == UNIF_MOE_OK) rc = dalloc(&(ptr), (n));
+  ALLOC(L->wr_t, (size_t)L->router_cols_pad * d_model);
+  ALLOC(L->bias, E);
+  void* wup = nullptr;
+  void* wdn = nullptr;
+  if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&wup), es * E * d_ff * d_model);
+  if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&wdn), es * E * d_ff * d_model);
+  L->w_up = wup; L->w_down = wdn;
+  ALLOC(w.alpha, T); ALLOC(w.b, T); ALLOC(w.k, T); ALLOC(w.shr_mask, T); ALLOC(w.exp_mask, T);
+  ALLOC(w.q, T * K); ALLOC(w.p, T * K); ALLOC(w.s, T * K);
+  ALLOC(w.chunk_cnt, (size_t)L->G * L->max_chunks);
+  ALLOC(w.grp_cnt, (size_t)L->G); ALLOC(w.grp_off, (size_t)L->G + 1); ALLOC(w.n_tiles, 1);
+  ALLOC(w.tile_group, (size_t)L->max_tiles); ALLOC(w.tile_row0, (size_t)L->max_tiles);
+  ALLOC(w.row_tok, (size_t)L->max_rows); ALLOC(w.row_w, (size_t)L->max_rows);
+  void* hb = nullptr;
+  if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&hb), es * (size_t)L->max_rows * M);
+  w.hbuf = hb;
+  ALLOC(w.y32, T * d_model);
+  ALLOC(w.status, 1);
+#undef ALLOC
+  if (rc == UNIF_MOE_OK && cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess) {
+    set_error("cudaMemset failed");
+    rc = UNIF_MOE_ERR_CUDA;
+  }
+  if (rc == UNIF_MOE_OK && unif::router_setup(L) != cudaSuccess) {
+    set_error("router kernel attribute setup failed");
+    rc = UNIF_MOE_ERR_CUDA;
+  }
+  if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::gemm_tc_setup(L);
+  if (rc != UNIF_MOE_OK) {
+    free_all(L);
+    delete L;
+    return rc;
+  }
+  *out = L;
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_load_weights(unif_moe_t L, const void* w_router, const void* w_up,
+                          const void* w_down, const float* router_bias, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L || !w_router || !w_up || !w_down) { set_error("NULL handle or weight"); return UNIF_MOE_ERR_ARG; }
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t bytes = elt_size(L) * (size_t)(L->K + 1) * L->H * L->d;
+  CK(cudaMemcpyAsync(L->w_up, w_up, bytes, cudaMemcpyDeviceToDevice, s));
+  CK(cudaMemcpyAsync(L->w_down, w_down, bytes, cudaMemcpyDeviceToDevice, s));
+  CK(unif::launch_prototypes(L, w_router, router_bias, s));
+  L->loaded = true;
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_t* token_mask,
+                     int32_t* shared_counts, int32_t* residual_counts, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (T < 0) { set_error("T < 0"); return UNIF_MOE_ERR_ARG; }
+  if (T > L->max_tokens) {
+    set_error("T=%d exceeds max_tokens=%d", T, L->max_tokens);
+    return UNIF_MOE_ERR_CAPACITY;
+  }
+  if (!L->loaded) { set_error("forward before load_weights"); return UNIF_MOE_ERR_STATE; }
+  if (T == 0) return UNIF_MOE_OK;
+  if (!x || !out) { set_error("x or out is NULL"); return UNIF_MOE_ERR_ARG; }
+  if (!aligned16(x) || !aligned16(out)) {
+    set_error("x and out must be 16-byte aligned");
+    return UNIF_MOE_ERR_ARG;
+  }
+  if ((shared_counts && !aligned16(shared_counts)) || (residual_counts && !aligned16(residual_counts))) {
+    set_error("count buffers must be 16-byte aligned");
+    return UNIF_MOE_ERR_ARG;
+  }
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaEvent_t* ev = L->stage_ev;
+  if (ev[0]) CK(cudaEventRecord(ev[0], s));
+  CK(cudaMemsetAsync(L->ws.y32, 0, sizeof(float) * (size_t)T * L->d, s));
+  CK(unif::launch_router(L, x, token_mask, T, shared_counts, residual_counts, s));
+  if (ev[1]) CK(cudaEventRecord(ev[1], s));
+  CK(unif::launch_permute(L, T, s));
+  if (ev[2]) CK(cudaEventRecord(ev[2], s));
+  if (L->dtype == UNIF_MOE_BF16) {
+    CK(unif::launch_gemms_tc(L, x, T, ev[3], s));
+  } else {
+    CK(unif::launch_gemms_simt(L, x, T, ev[3], s));
+  }
+  if (ev[4]) CK(cudaEventRecord(ev[4], s));
+  CK(unif::launch_combine(L, out, T, s));
+  if (ev[5]) CK(cudaEventRecord(ev[5], s));
+  L->last_T = T;
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_forward_host(unif_moe_t L, const void* x_host, void* out_host, int T,
+                          const uint8_t* mask_host, int32_t* b_host, int32_t* k_host,
+                          void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (T < 0 || T > L->max_tokens) {
+    set_error("T=%d outside [0, max_tokens=%d]", T, L->max_tokens);
+    return T < 0 ? UNIF_MOE_ERR_ARG : UNIF_MOE_ERR_CAPACITY;
+  }
+  if (!L->loaded) { set_error("forward before load_weights"); return UNIF_MOE_ERR_STATE; }
+  if (T == 0) return UNIF_MOE_OK;
+  if (!x_host || !out_host) { set_error("x or out is NULL"); return UNIF_MOE_ERR_ARG; }
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unif::Workspace& w = L->ws;
+  const size_t es = elt_size(L);
+  const size_t n = (size_t)L->max_tokens;
+  if (!w.x_stage) {  // staging buffers are created on first use
+    int rc = dalloc(reinterpret_cast<char**>(&w.x_stage), es * n * L->d);
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.out_stage), es * n * L->d);
+    if (rc == UNIF_MOE_OK) rc = dalloc(&w.mask_stage, n);
+    if (rc == UNIF_MOE_OK) rc = dalloc(&w.b_stage, n);
+    if (rc == UNIF_MOE_OK) rc = dalloc(&w.k_stage, n);
+    if (rc != UNIF_MOE_OK) return rc;
+  }
+  const size_t xb = es * (size_t)T * L->d;
+  CK(cudaMemcpyAsync(w.x_stage, x_host, xb, cudaMemcpyHostToDevice, s));
+  if (mask_host) CK(cudaMemcpyAsync(w.mask_stage, mask_host, (size_t)T, cudaMemcpyHostToDevice, s));
+  int rc = unif_moe_forward(L, w.x_stage, w.out_stage, T, mask_host ? w.mask_stage : nullptr,
+                            b_host ? w.b_stage : nullptr, k_host ? w.k_stage : nullptr, stream);
+  if (rc != UNIF_MOE_OK) return rc;
+  CK(cudaMemcpyAsync(out_host, w.out_stage, xb, cudaMemcpyDeviceToHost, s));
+  if (b_host) CK(cudaMemcpyAsync(b_host, w.b_stage, sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
+  if (k_host) CK(cudaMemcpyAsync(k_host, w.k_stage, sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_get_routing(unif_moe_t L, float* alpha, uint64_t* shared_mask, uint64_t* expert_mask,
+                         int32_t* q, float* p, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (L->last_T < 0) { set_error("no forward has run"); return UNIF_MOE_ERR_STATE; }
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t T = (size_t)L->last_T, K = (size_t)L->K;
+  const cudaMemcpyKind dd = cudaMemcpyDeviceToDevice;
+  if (T > 0) {
+    if (alpha) CK(cudaMemcpyAsync(alpha, L->ws.alpha, sizeof(float) * T, dd, s));
+    if (shared_mask) CK(cudaMemcpyAsync(shared_mask, L->ws.shr_mask, sizeof(uint64_t) * T, dd, s));
+    if (expert_mask) CK(cudaMemcpyAsync(expert_mask, L->ws.exp_mask, sizeof(uint64_t) * T, dd, s));
+    if (q) CK(cudaMemcpyAsync(q, L->ws.q, sizeof(int32_t) * T * K, dd, s));
+    if (p) CK(cudaMemcpyAsync(p, L->ws.p, sizeof(float) * T * K, dd, s));
+  }
+  CK(cudaStreamSynchronize(s));
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t* row_token,
+                        float* row_weight, int64_t* n_rows, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (L->last_T < 0) { set_error("no forward has run"); return UNIF_MOE_ERR_STATE; }
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const cudaMemcpyKind dh = cudaMemcpyDeviceToHost;
+  int32_t total = 0;
+  if (L->last_T > 0) CK(cudaMemcpyAsync(&total, L->ws.grp_off + L->G, sizeof(int32_t), dh, s));
+  CK(cudaStreamSynchronize(s));
+  if (L->last_T > 0) {
+    if (counts) CK(cudaMemcpyAsync(counts, L->ws.grp_cnt, sizeof(int32_t) * L->G, dh, s));
+    if (offsets) CK(cudaMemcpyAsync(offsets, L->ws.grp_off, sizeof(int32_t) * (L->G + 1), dh, s));
+    if (row_token && total > 0) CK(cudaMemcpyAsync(row_token, L->ws.row_tok, sizeof(int32_t) * total, dh, s));
+    if (row_weight && total > 0) CK(cudaMemcpyAsync(row_weight, L->ws.row_w, sizeof(float) * total, dh, s));
+  } else {
+    if (counts) memset(counts, 0, sizeof(int32_t) * L->G);
+    if (offsets) memset(offsets, 0, sizeof(int32_t) * (L->G + 1));
+  }
+  if (n_rows) *n_rows = total;
+  CK(cudaStreamSynchronize(s));
+  return UNIF_MOE_OK;
+}
+
+int64_t unif_moe_max_rows(unif_moe_t L) { return L ? L->max_rows : -1; }
+
+int unif_moe_set_stage_events(unif_moe_t L, void* const* events) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  for (int i = 0; i < 6; ++i) {
+    L->stage_ev[i] = events ? static_cast<cudaEvent_t>(events[i]) : nullptr;
+    if (events && !events[i]) { set_error("event %d is NULL", i); return UNIF_MOE_ERR_ARG; }
+  }
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_sync_status(unif_moe_t L, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int st = 0;
+  CK(cudaMemcpyAsync(&st, L->ws.status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  CK(cudaMemsetAsync(L->ws.status, 0, sizeof(int), s));
+  CK(cudaStreamSynchronize(s));
+  if (st & unif::kStatusTimeout) {
+    set_error("a kernel gave up a bounded wait (status 0x%x)", st);
+    return UNIF_MOE_ERR_TIMEOUT;
+  }
+  if (st) {
+    set_error("kernel status 0x%x", st);
+    return UNIF_MOE_ERR_CUDA;
+  }
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_selftest_timeout(unif_moe_t L, int timeout_us, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  DeviceGuard dg(L->device);
+  CK(unif::launch_timeout_probe(L, timeout_us, static_cast<cudaStream_t>(stream)));
+  return UNIF_MOE_OK;
+}
+
+void unif_moe_destroy(unif_moe_t L) {
+  if (!L) return;
+  {
+    DeviceGuard dg(L->device);
+    cudaDeviceSynchronize();
+    free_all(L);
+  }
+  delete L;
+}
+
+}  // extern "C"

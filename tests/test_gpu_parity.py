@@ -1,0 +1,268 @@
+"""GPU parity: the CUDA layer (through the C ABI) against the CPU oracle on
+the five seeded workloads, on ragged and edge-case shapes, and on the
+ablation switches of Table IV. Rules in tests/gpu_helpers.py."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads
+from gpu_helpers import assert_parity, compare, make_layer, run_gpu, subset
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def small(dtype="bf16", **kw):
+    base = dict(tokens=300, d_model=128, d_ff=512, n_experts=4, n_blocks=4)
+    base.update(kw)
+    name = "tiny_f32" if dtype == "f32" else "vit_s"
+    return workloads.spec(name).with_(**base)
+
+
+# ---------------------------------------------------------------- workloads
+
+def test_tiny_f32_full():
+    wl = workloads.make_workload(workloads.spec("tiny_f32"))
+    g = run_gpu(wl)
+    rep = compare(wl, g)
+    assert_parity(wl, g, rep)
+
+
+def test_vit_s_full_size():
+    wl = workloads.make_workload(workloads.spec("vit_s"))
+    g = run_gpu(wl)
+    rep = compare(wl, g, sample=1500)
+    print(rep)
+    assert_parity(wl, g, rep)
+
+
+def test_bert_base_padding():
+    wl = workloads.make_workload(workloads.spec("bert_base"))
+    g = run_gpu(wl)
+    m = wl.mask.numpy()
+    assert (g.b[m == 0] == 0).all() and (g.k[m == 0] == 0).all()
+    assert (g.y[m == 0] == 0).all()
+    assert np.isfinite(g.y).all()
+    rep = compare(wl, g, sample=1000)
+    print(rep)
+    assert_parity(wl, g, rep)
+
+
+@pytest.mark.parametrize("theta", [math.nan, 0.5, 0.7, 0.9])
+def test_vit_b_thresholds(theta):
+    wl = workloads.make_workload(workloads.spec("vit_b", beta_fixed=theta))
+    g = run_gpu(wl)
+    rep = compare(wl, g, sample=400)
+    print(theta, rep)
+    assert_parity(wl, g, rep)
+
+
+def test_stress_full_size():
+    wl = workloads.make_workload(workloads.spec("stress"))
+    g = run_gpu(wl)
+    rep = compare(wl, g, sample=200)
+    print(rep, "b range", g.b.min(), g.b.max(), "k range", g.k.min(), g.k.max())
+    assert g.b.min() == 1 and g.b.max() == 15  # the mixture spans every shared count
+    assert_parity(wl, g, rep)
+
+
+# ------------------------------------------------------------- ragged sizes
+
+@pytest.mark.parametrize("T", [1, 7, 64, 129, 255, 257, 1000])
+def test_ragged_token_counts(T):
+    wl = workloads.make_workload(small(tokens=T))
+    g = run_gpu(wl)
+    assert_parity(wl, g, compare(wl, g))
+
+
+def test_zero_tokens_is_noop():
+    wl = workloads.make_workload(small(tokens=16))
+    layer = make_layer(wl.spec)
+    dev = torch.device("cuda")
+    layer.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
+    x = torch.empty(0, wl.spec.d_model, dtype=torch.bfloat16, device=dev)
+    y = layer.forward(x)
+    assert y.shape == (0, wl.spec.d_model)
+
+
+def test_all_tokens_masked():
+    wl = workloads.make_workload(small(tokens=200))
+    mask = torch.zeros(200, dtype=torch.uint8)
+    g = run_gpu(wl, mask=mask)
+    assert (g.y == 0).all() and (g.b == 0).all() and (g.k == 0).all()
+
+
+def test_max_tokens_and_reuse():
+    """T = max_tokens, then a smaller T on the same handle (workspace reuse)."""
+    wl = workloads.make_workload(small(tokens=1000))
+    g = run_gpu(wl)
+    assert_parity(wl, g, compare(wl, g))
+    x2 = wl.x[:333].clone()
+    g2 = run_gpu(wl, layer=g.layer, x=x2, mask=None)
+    np.testing.assert_allclose(g2.y, g.y[:333], rtol=1e-2, atol=1e-6)  # one bf16 ulp
+
+
+@pytest.mark.parametrize("shape", [
+    dict(d_model=64, d_ff=256, n_experts=2, n_blocks=2),     # B = 2: b = 1 always
+    dict(d_model=192, d_ff=768, n_experts=6, n_blocks=4),
+    dict(d_model=256, d_ff=2048, n_experts=3, n_blocks=8),   # M = 256
+    dict(d_model=384, d_ff=3072, n_experts=5, n_blocks=8),   # M = 384: two N sub-tiles
+    dict(d_model=320, d_ff=1280, n_experts=4, n_blocks=5),   # d = 5 x 64
+])
+def test_shapes(shape):
+    wl = workloads.make_workload(small(tokens=700, **shape))
+    g = run_gpu(wl)
+    if shape["n_blocks"] == 2:
+        assert (g.b == 1).all()
+    assert_parity(wl, g, compare(wl, g))
+
+
+# ------------------------------------------------- ablation switches (Table IV)
+
+@pytest.mark.parametrize("kw", [
+    dict(alpha_fixed=0.4),
+    dict(topk_fixed=2),
+    dict(prefix_blocks=1),
+    dict(beta_fixed=0.7),
+    dict(tau=0.05),
+])
+def test_threshold_variants(kw):
+    wl = workloads.make_workload(small(tokens=900, n_experts=6, n_blocks=8, d_ff=1024, **kw))
+    g = run_gpu(wl)
+    assert_parity(wl, g, compare(wl, g))
+
+
+def test_alpha_one_is_dense_ffn():
+    """alpha = 1: every block shared, y = E_shr(x) (Eq. 4)."""
+    wl = workloads.make_workload(small(tokens=500, alpha_fixed=1.0))
+    g = run_gpu(wl)
+    assert (g.b == wl.spec.n_blocks).all()
+    x = wl.x.double().numpy()
+    wu = wl.w_up[0].double().numpy()
+    wd = wl.w_down[0].double().numpy()
+    from scipy.stats import norm
+    a = x @ wu.T
+    dense = (a * norm.cdf(a)) @ wd.T
+    rel = np.abs(g.y - dense).max(axis=1) / np.abs(dense).max(axis=1)
+    assert rel.max() < 2e-2
+
+
+def test_alpha_zero_all_experts_is_soft_moe():
+    wl = workloads.make_workload(small(tokens=400, alpha_fixed=0.0, beta_fixed=1.0))
+    g = run_gpu(wl)
+    assert (g.b == 0).all() and (g.k == wl.spec.n_experts).all()
+    assert_parity(wl, g, compare(wl, g))
+
+
+def test_f32_variants():
+    wl = workloads.make_workload(workloads.spec("tiny_f32", tokens=1000, topk_fixed=2))
+    g = run_gpu(wl)
+    assert_parity(wl, g, compare(wl, g))
+
+
+# ------------------------------------------------------------ group table
+
+def test_group_table_matches_oracle():
+    wl = workloads.make_workload(small(tokens=1500, n_experts=6, n_blocks=8, d_ff=1024))
+    g = run_gpu(wl)
+    counts, offsets, tok, w = g.layer.groups()
+    r = oracle.with_decisions(compare_routing(wl), g.shr, g.em, wl.spec.n_blocks)
+    c_ref, tok_ref, w_ref = oracle.groups(r, wl.spec.n_experts, wl.spec.n_blocks)
+    assert counts.numpy().tolist() == c_ref.tolist()
+    offs = offsets.numpy()
+    assert (offs[1:] - offs[:-1]).tolist() == [(c + 127) // 128 * 128 for c in c_ref]
+    start = np.concatenate([[0], np.cumsum(c_ref)])
+    for gi in range(len(c_ref)):
+        got = tok.numpy()[offs[gi]:offs[gi] + c_ref[gi]]
+        assert got.tolist() == tok_ref[start[gi]:start[gi + 1]].tolist()
+        np.testing.assert_allclose(w.numpy()[offs[gi]:offs[gi] + c_ref[gi]],
+                                   w_ref[start[gi]:start[gi + 1]], rtol=1e-5, atol=1e-7)
+        assert (tok.numpy()[offs[gi] + c_ref[gi]:offs[gi + 1]] == -1).all()
+
+
+def compare_routing(wl):
+    from gpu_helpers import oracle_routing
+    return oracle_routing(wl)
+
+
+def test_permuting_tokens_permutes_outputs():
+    wl = workloads.make_workload(small(tokens=600))
+    g = run_gpu(wl)
+    perm = torch.from_numpy(np.random.default_rng(1).permutation(600))
+    g2 = run_gpu(wl, layer=g.layer, x=wl.x[perm], mask=None)
+    pn = perm.numpy()
+    assert np.array_equal(g2.b, g.b[pn]) and np.array_equal(g2.shr, g.shr[pn])
+    assert np.array_equal(g2.em, g.em[pn])
+    np.testing.assert_allclose(g2.y, g.y[pn], rtol=1e-2, atol=1e-6)  # one bf16 ulp
+
+
+# ------------------------------------------------------------- ABI behaviour
+
+def test_errors_are_reported():
+    from paper_2608_10392_gb300 import UnifMoeError
+    wl = workloads.make_workload(small(tokens=64))
+    layer = make_layer(wl.spec)
+    dev = torch.device("cuda")
+    x = wl.x.to(dev)
+    with pytest.raises(UnifMoeError) as e:
+        layer.forward(x)  # no weights yet
+    assert e.value.code == -6
+    layer.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
+    big = torch.zeros(65, wl.spec.d_model, dtype=torch.bfloat16, device=dev)
+    with pytest.raises(UnifMoeError) as e:
+        layer.forward(big)
+    assert e.value.code == -3
+    raw = torch.zeros(64 * wl.spec.d_model + 8, dtype=torch.bfloat16, device=dev)
+    mis = raw[1:1 + 64 * wl.spec.d_model].view(64, wl.spec.d_model)
+    with pytest.raises(UnifMoeError) as e:
+        layer.forward(mis)
+    assert e.value.code == -1
+    with pytest.raises(UnifMoeError):
+        make_layer(wl.spec.with_(d_ff=500))  # H % B != 0
+    with pytest.raises(UnifMoeError):
+        make_layer(wl.spec.with_(d_model=96))  # bf16 needs d % 64 == 0
+
+
+def test_output_guard_bands():
+    wl = workloads.make_workload(small(tokens=257))
+    layer = make_layer(wl.spec)
+    dev = torch.device("cuda")
+    layer.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
+    d = wl.spec.d_model
+    buf = torch.full((257 + 4, d), 7.0, dtype=torch.bfloat16, device=dev)
+    out = buf[2:2 + 257]
+    layer.forward(wl.x.to(dev), out=out)
+    torch.cuda.synchronize()
+    assert (buf[:2] == 7.0).all() and (buf[-2:] == 7.0).all()
+
+
+def test_timeout_status_path():
+    """A bounded wait that runs out is reported, and the context stays usable."""
+    wl = workloads.make_workload(small(tokens=128))
+    layer = make_layer(wl.spec)
+    assert layer.sync_status() == 0
+    layer.selftest_timeout(2000)
+    assert layer.sync_status() == -5
+    assert layer.sync_status() == 0  # cleared
+    g = run_gpu(wl, layer=None)
+    assert_parity(wl, g, compare(wl, g))
+
+
+def test_forward_host_matches_device():
+    wl = workloads.make_workload(small(tokens=500))
+    g = run_gpu(wl)
+    xh = wl.x.pin_memory()
+    out = torch.empty_like(xh).pin_memory()
+    b = torch.empty(500, dtype=torch.int32).pin_memory()
+    k = torch.empty(500, dtype=torch.int32).pin_memory()
+    g.layer.forward_host(xh, out, shared_counts_host=b, residual_counts_host=k)
+    np.testing.assert_allclose(out.float().numpy(), g.y, rtol=1e-2, atol=1e-6)  # one bf16 ulp
+    assert np.array_equal(b.numpy(), g.b) and np.array_equal(k.numpy(), g.k)
