@@ -314,9 +314,10 @@ def main():
                      "peak_kind": "%s bf16 sustained" % peak_kind},
         "stages": stages,
         "hbm_peak_gbs": hbm,
-        "e2e": {"value": T_valid / (statistics.fmean(e2e_ms) / 1e3), "unit": UNIT,
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "ms_per_step": statistics.fmean(e2e_ms)},
+        "e2e": None if not e2e_ms else {
+            "value": T_valid / (statistics.fmean(e2e_ms) / 1e3), "unit": UNIT,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": statistics.fmean(e2e_ms)},
         "gpu_launches": KERNELS_PER_FORWARD * K,
         "clocks": clocks,
     }
