@@ -172,6 +172,36 @@ UNIF_MOE_API int unif_moe_sync_status(unif_moe_t h, void* stream);
  * hanging the GPU. */
 UNIF_MOE_API int unif_moe_selftest_timeout(unif_moe_t h, int timeout_us, void* stream);
 
+/* Groups (expert, block) pairs by pair, like the grouping step inside
+ * unif_moe_forward, but allocates nothing and needs no handle. It is for
+ * callers that cannot call cudaMalloc: inference engines that plan all device
+ * memory up front and give plugins no allocator once set up, and
+ * latency-critical paths that cannot pay cudaMalloc's implicit device
+ * synchronisation. The paper has no counterpart; this is a deployment aid.
+ * Inputs (device, one entry per token, as unif_moe_get_routing returns them
+ * plus the per-expert affinities):
+ *   shared_mask_dev [T] uint64, expert_mask_dev [T] uint64, alpha_dev [T]
+ *   float, affinity_dev [T][K] float (s_j by expert index j).
+ * Outputs (device, caller-allocated): counts_dev [G], offsets_dev [G+1],
+ *   n_tiles_dev [1], tile_group_dev and tile_row0_dev [row_capacity/128],
+ *   row_token_dev and row_weight_dev [row_capacity]; G = (K+1)*B, layout as
+ *   in unif_moe_get_groups (groups padded to 128 rows, padding token -1).
+ * row_capacity must be at least T*K*B + G*127 (else ERR_CAPACITY).
+ * Scratch: a 1 MiB array inside the library (device memory every GPU that
+ * loads the library keeps until exit) holds the per-chunk counts, so
+ * (K+1)*B*ceil(T/256) must not exceed 262144 (else ERR_CAPACITY). The first
+ * call on each device looks up that array's device address; make that first
+ * call before any stream capture. Calls that overlap on the GPU share the
+ * array and race: order them on one stream. Enqueued on `stream`, no sync. */
+UNIF_MOE_API int unif_moe_group_noalloc(int T, int n_experts, int n_blocks,
+                                        const uint64_t* shared_mask_dev,
+                                        const uint64_t* expert_mask_dev, const float* alpha_dev,
+                                        const float* affinity_dev, int32_t* counts_dev,
+                                        int32_t* offsets_dev, int32_t* n_tiles_dev,
+                                        int32_t* tile_group_dev, int32_t* tile_row0_dev,
+                                        int32_t* row_token_dev, float* row_weight_dev,
+                                        int64_t row_capacity, void* stream);
+
 /* Frees the handle and its device memory (synchronises the device first).
  * NULL is ignored. */
 UNIF_MOE_API void unif_moe_destroy(unif_moe_t h);

@@ -31,8 +31,8 @@ ERR = {0: "OK", -1: "ERR_ARG", -2: "ERR_SHAPE", -3: "ERR_CAPACITY", -4: "ERR_CUD
 EXPORTS = ["unif_moe_default_thresholds", "unif_moe_create", "unif_moe_load_weights",
            "unif_moe_forward", "unif_moe_forward_host", "unif_moe_get_routing",
            "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_set_stage_events",
-           "unif_moe_sync_status",
-           "unif_moe_selftest_timeout", "unif_moe_destroy", "unif_moe_last_error"]
+           "unif_moe_sync_status", "unif_moe_selftest_timeout", "unif_moe_group_noalloc",
+           "unif_moe_destroy", "unif_moe_last_error"]
 
 
 class UnifMoeError(RuntimeError):
@@ -70,6 +70,7 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_set_stage_events.argtypes = [P, P]
         L.unif_moe_sync_status.argtypes = [P, P]
         L.unif_moe_selftest_timeout.argtypes = [P, I, P]
+        L.unif_moe_group_noalloc.argtypes = [I, I, I] + [P] * 11 + [C.c_int64, P]
         L.unif_moe_destroy.argtypes = [P]
         L.unif_moe_destroy.restype = None
         L.unif_moe_last_error.restype = C.c_char_p

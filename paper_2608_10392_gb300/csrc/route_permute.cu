@@ -584,3 +584,104 @@ cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s) 
 }
 
 }  // namespace unif
+
+// ---------------------------------------------------------------------------
+// Grouping without allocation (unif_moe_group_noalloc)
+// ---------------------------------------------------------------------------
+// Some callers cannot call cudaMalloc: inference engines that plan all
+// device memory up front and give plugins no allocator after setup, and
+// latency-critical paths that must not pay cudaMalloc's implicit device
+// synchronisation. For them the grouping step's only scratch, the per-chunk
+// group counts, lives in this file-scope device array, which every GPU that
+// loads the library holds (1 MiB) until the process exits. Its contents
+// persist between calls; the count kernel overwrites every entry a call
+// reads, so nothing needs clearing. Calls that overlap on the GPU share the
+// array and race.
+#include <mutex>
+
+namespace unif {
+
+constexpr int kNoAllocScratchInts = 1 << 18;  // 1 MiB of int32
+static __device__ __align__(256) int32_t g_group_scratch[kNoAllocScratchInts];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+int32_t* g_scratch_dev_ptr[kMaxDevices] = {};
+
+// The device address of g_group_scratch on the current device. In host code
+// the array's name is only a host-side stand-in, so the address is looked up
+// once per device (first call with that device current) and cached.
+int32_t* group_scratch_on_current_device(cudaError_t* err) {
+  int dev = -1;
+  *err = cudaGetDevice(&dev);
+  if (*err != cudaSuccess) return nullptr;
+  if (dev < 0 || dev >= kMaxDevices) {
+    *err = cudaErrorInvalidDevice;
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_dev_ptr[dev]) {
+    void* p = nullptr;
+    *err = cudaGetSymbolAddress(&p, g_group_scratch);
+    if (*err != cudaSuccess) return nullptr;
+    g_scratch_dev_ptr[dev] = static_cast<int32_t*>(p);
+  }
+  return g_scratch_dev_ptr[dev];
+}
+
+}  // namespace
+}  // namespace unif
+
+extern "C" UNIF_MOE_API int unif_moe_group_noalloc(
+    int T, int n_experts, int n_blocks, const uint64_t* shared_mask, const uint64_t* expert_mask,
+    const float* alpha, const float* affinity, int32_t* counts, int32_t* offsets,
+    int32_t* n_tiles, int32_t* tile_group, int32_t* tile_row0, int32_t* row_token,
+    float* row_weight, int64_t row_capacity, void* stream) {
+  using namespace unif;
+  if (T < 0 || n_experts < 1 || n_experts > 64 || n_blocks < 2 || n_blocks > 64) {
+    set_error("group_noalloc: bad sizes T=%d K=%d B=%d", T, n_experts, n_blocks);
+    return UNIF_MOE_ERR_ARG;
+  }
+  if (!counts || !offsets || !n_tiles || !tile_group || !tile_row0 || !row_token || !row_weight ||
+      (T > 0 && (!shared_mask || !expert_mask || !alpha || !affinity))) {
+    set_error("group_noalloc: NULL pointer");
+    return UNIF_MOE_ERR_ARG;
+  }
+  const int G = (n_experts + 1) * n_blocks;
+  const int n_chunks = (T + kChunkTokens - 1) / kChunkTokens;
+  if ((int64_t)G * n_chunks > kNoAllocScratchInts) {
+    set_error("group_noalloc: (K+1)*B*ceil(T/256) = %lld exceeds the built-in scratch of %d "
+              "entries; reduce T", (long long)G * n_chunks, kNoAllocScratchInts);
+    return UNIF_MOE_ERR_CAPACITY;
+  }
+  const int64_t need = (int64_t)T * n_experts * n_blocks + (int64_t)G * (kTileRows - 1);
+  if (row_capacity < need) {
+    set_error("group_noalloc: row_capacity %lld below the bound T*K*B + G*127 = %lld",
+              (long long)row_capacity, (long long)need);
+    return UNIF_MOE_ERR_CAPACITY;
+  }
+  cudaError_t e;
+  int32_t* scratch = group_scratch_on_current_device(&e);
+  if (!scratch) {
+    set_error("group_noalloc: scratch address lookup failed: %s", cudaGetErrorString(e));
+    return UNIF_MOE_ERR_CUDA;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (n_chunks > 0)
+    count_kernel<<<n_chunks, kPermThreads, 0, s>>>(shared_mask, expert_mask, T, n_experts,
+                                                   n_blocks, n_chunks, scratch);
+  scan_kernel<<<1, 1024, 0, s>>>(G, n_chunks, scratch, counts, offsets, n_tiles, tile_group,
+                                 tile_row0, row_token, row_weight);
+  if (n_chunks > 0)
+    scatter_kernel<<<n_chunks, kPermThreads, 0, s>>>(shared_mask, expert_mask, alpha, affinity, T,
+                                                     n_experts, n_blocks, n_chunks, scratch,
+                                                     offsets, row_token, row_weight);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_error("group_noalloc: launch failed: %s", cudaGetErrorString(e));
+    return UNIF_MOE_ERR_CUDA;
+  }
+  return UNIF_MOE_OK;
+}
