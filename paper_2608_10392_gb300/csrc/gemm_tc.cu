@@ -10,8 +10,10 @@
 // for residual expert q_i, Eq. 30).
 //
 // Roles inside one CTA (one CTA per SM, 384 threads):
-//   warp 0      TMA producer: A tile (gathered x rows with tile::gather4, or
-//               a plain 2-D tile of h) and B tile (a weight slice) per stage
+//   warps 0, 2  up kernel: gather the tile's 128 token rows of x with 16-byte
+//               cp.async into the swizzled operand layout; warp 0 lane 0 also
+//               loads the weight tile with TMA
+//   warp 0      down kernel: TMA of the h tile and the weight tile
 //   warp 1      TMEM allocator and MMA issuer (one lane): 128 x BN x 16
 //               kind::f16 MMAs, fp32 accumulators in TMEM
 //   warps 4-11  epilogue: tcgen05.ld of the accumulator, GeLU -> bf16 h
@@ -36,7 +38,6 @@ namespace tc {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;
-constexpr int kStages = 4;
 constexpr int kThreads = 384;
 constexpr int kEpiWarps = 8;
 constexpr int kFirstEpiWarp = 4;
@@ -45,7 +46,17 @@ constexpr uint32_t kAccStride = 256;  // TMEM columns per accumulator buffer
 constexpr int kMaxBN = 256;
 constexpr uint32_t kStageA = kBM * kBK * 2;      // 16 KB
 constexpr uint32_t kStageB = kMaxBN * kBK * 2;   // 32 KB
-constexpr size_t kSmemBytes = 1024 + kStages * (kStageA + kStageB) + 256;
+constexpr int kStageRow = 36;                    // fp32 per staged row (32 + 4 pad, 16 B aligned)
+
+// Per-kernel shared memory: the up kernel keeps 4 operand stages; the down
+// kernel keeps 3 and a per-warp 32 x 32 fp32 staging tile that turns its
+// row-per-thread accumulator into row-contiguous, coalesced atomic adds.
+template <int MODE>
+struct Cfg {
+  static constexpr int kStages = MODE == 0 ? 4 : 3;
+  static constexpr uint32_t kStaging = MODE == 0 ? 0u : kEpiWarps * 32u * kStageRow * 4u;
+  static constexpr size_t kSmem = 1024 + kStages * (kStageA + kStageB) + kStaging + 256;
+};
 
 struct Params {
   const int32_t* n_tiles;
@@ -54,9 +65,10 @@ struct Params {
   const int32_t* row_tok;
   const float* row_w;
   int n_sub;       // N sub-tiles per 128-row tile
-  int bn;          // N per sub-tile (multiple of 32, <= 256)
+  int bn;          // N per sub-tile (multiple of 64, <= 256)
   int num_kb;      // reduction steps of 64
   int B, M, H, d;
+  const __nv_bfloat16* x;  // up: tokens [T][d] (rows gathered with cp.async)
   __nv_bfloat16* h;  // up: [rows][M]
   float* y32;        // down: [T][d]
   int* status;
@@ -116,14 +128,19 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
       : "memory");
 }
-__device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap* map, uint32_t bar,
-                                            int col, int r0, int r1, int r2, int r3) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(col), "r"(r0), "r"(r1), "r"(r2),
-      "r"(r3)
-      : "memory");
+// ---- cp.async (row gather into the swizzled operand layout) ----
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // ---- tcgen05 ----
@@ -174,6 +191,86 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 32 lanes x 32 consecutive 32-bit TMEM columns; thread i holds lane base+i.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32"
+      " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15,"
+      " %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// ---- GeLU on pairs with packed fp32x2 arithmetic ----
+// GeLU(x) = x Phi(x) = max(x, 0) - |x| Q(|x|), Q(a) = Phi(-a) = exp(-a^2/2) R(a),
+// R(a) = erfcx(a / sqrt 2) / 2 (the exact erf form, rewritten through the
+// normal tail). R is a degree-12 polynomial in s = 0.4 min(a, 5) - 1, a
+// least-squares Chebyshev fit on [0, 5] (coefficients from gelu_coeffs.py):
+// GeLU relative error < 5e-6 for |x| <= 5, absolute error < 5e-7 everywhere,
+// far below the bf16 rounding h receives next.
+__device__ __forceinline__ uint64_t pk2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void upk2(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+#define UNIF_K2(bits) ((uint64_t)(bits##u) << 32 | (uint64_t)(bits##u))
+__device__ __forceinline__ uint32_t gelu2_bf16x2(float x0, float x1) {
+  const float a0 = fabsf(x0), a1 = fabsf(x1);
+  const uint64_t s = fma2(pk2(fminf(a0, 5.f), fminf(a1, 5.f)), UNIF_K2(0x3ecccccd),  // 0.4
+                          UNIF_K2(0xbf800000));                                      // -1
+  uint64_t r = UNIF_K2(0x3a5572c6);
+  r = fma2(r, s, UNIF_K2(0xbad23ee0));
+  r = fma2(r, s, UNIF_K2(0x3a403f1b));
+  r = fma2(r, s, UNIF_K2(0xbac3e363));
+  r = fma2(r, s, UNIF_K2(0x3bb29d94));
+  r = fma2(r, s, UNIF_K2(0xbc1d2cf5));
+  r = fma2(r, s, UNIF_K2(0x3c76a00d));
+  r = fma2(r, s, UNIF_K2(0xbccc3410));
+  r = fma2(r, s, UNIF_K2(0x3d22ed53));
+  r = fma2(r, s, UNIF_K2(0xbd754c1d));
+  r = fma2(r, s, UNIF_K2(0x3daeb1a7));
+  r = fma2(r, s, UNIF_K2(0xbde98aa9));
+  r = fma2(r, s, UNIF_K2(0x3e10b92a));
+  const uint64_t aa = pk2(a0, a1);
+  // exp(-a^2/2) = 2^(-a^2 log2(e) / 2)
+  const uint64_t t = mul2(mul2(aa, aa), UNIF_K2(0xbf38aa3b));  // -0.7213475
+  float t0, t1;
+  upk2(t, t0, t1);
+  const uint64_t q = mul2(mul2(pk2(ex2_approx(t0), ex2_approx(t1)), r), aa);
+  float q0, q1;
+  upk2(q, q0, q1);
+  const float g0 = fmaxf(x0, 0.f) - q0, g1 = fmaxf(x1, 0.f) - q1;
+  __nv_bfloat162 h = __floats2bfloat162_rn(g0, g1);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+#undef UNIF_K2
+
 // Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
 // 1024 bytes apart (stride-dimension offset), leading offset unused (1),
 // descriptor version 1 at bit 46, swizzle mode 2 (128 B) at bits 61-63.
@@ -190,14 +287,6 @@ __device__ __forceinline__ uint32_t idesc_bf16(int m, int n) {
          ((uint32_t)(m >> 4) << 24);
 }
 
-__device__ __forceinline__ float gelu_erf(float v) {
-  return 0.5f * v * (1.0f + erff(v * 0.70710678118654752f));
-}
-
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&p);
-}
 
 // MODE 0 = up-projection (+GeLU), MODE 1 = down-projection (+weighted add).
 template <int MODE>
@@ -207,9 +296,12 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
+  constexpr int kStages = Cfg<MODE>::kStages;
   const uint32_t sA = smem_u32(smem);
   const uint32_t sB = sA + kStages * kStageA;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * (kStageA + kStageB));
+  float* staging = reinterpret_cast<float*>(smem + kStages * (kStageA + kStageB));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * (kStageA + kStageB) +
+                                               Cfg<MODE>::kStaging);
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
   auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
@@ -221,7 +313,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(full_bar(s), 1);
+      mbar_init(full_bar(s), MODE == 0 ? 3 : 1);
       mbar_init(empty_bar(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -240,10 +332,69 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int n_items = p.n_tiles[0] * p.n_sub;
-  const uint32_t stage_bytes = kStageA + (uint32_t)p.bn * kBK * 2;
+  // Bytes the TMA brings per stage (the up kernel gathers A with cp.async).
+  const uint32_t stage_bytes = (MODE == 0 ? 0u : kStageA) + (uint32_t)p.bn * kBK * 2;
 
-  if (warp == 0) {
-    // ------------------------------ producer ------------------------------
+  if (MODE == 0 && (warp == 0 || warp == 2)) {
+    // ------------------- producer (up): gathered x rows ----------------------
+    // Warps 0 and 2 copy the 128 token rows of a stage with 16-byte cp.async
+    // into the 128-byte-swizzled layout (16-byte chunk j of row r lands at
+    // chunk j ^ (r mod 8)); lane 0 of warp 0 also brings the weight tile by TMA.
+    // A stage is signalled LAG stages after its copies were issued, once
+    // cp.async.wait_group shows them complete.
+    constexpr int LAG = 2;
+    const int rbase = (warp == 0 ? 0 : 64) + lane;  // rows rbase and rbase + 32
+    int stage = 0;
+    uint32_t phase = 0;
+    int issued = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      const int tile = item / p.n_sub, ns = item % p.n_sub;
+      const int g = p.tile_group[tile], row0 = p.tile_row0[tile];
+      const int e = g / p.B, blk = g % p.B;
+      int t0 = p.row_tok[row0 + rbase], t1 = p.row_tok[row0 + rbase + 32];
+      t0 = t0 < 0 ? 0 : t0;  // padding rows read token 0; their results are never used
+      t1 = t1 < 0 ? 0 : t1;
+      const __nv_bfloat16* src0 = p.x + (size_t)t0 * p.d;
+      const __nv_bfloat16* src1 = p.x + (size_t)t1 * p.d;
+      const int brow = e * p.H + blk * p.M + ns * p.bn;
+      for (int kb = 0; kb < p.num_kb; ++kb) {
+        bool w = true;
+        if (lane == 0) w = wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
+        ok = __shfl_sync(0xffffffffu, w, 0);
+        if (!ok) break;
+        const uint32_t a_dst = sA + stage * kStageA;
+        if (warp == 0 && lane == 0) {
+          mbar_expect_tx(full_bar(stage), stage_bytes);
+          tma_load_2d(sB + stage * kStageB, &tmB, full_bar(stage), kb * kBK, brow);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          cp_async16(a_dst + rbase * 128u + ((j ^ (rbase & 7)) << 4), src0 + kb * kBK + j * 8);
+          cp_async16(a_dst + (rbase + 32) * 128u + ((j ^ (rbase & 7)) << 4),
+                     src1 + kb * kBK + j * 8);
+        }
+        cp_async_commit();
+        ++issued;
+        if (issued >= LAG) {
+          cp_async_wait<LAG - 1>();
+          fence_proxy_async();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(full_bar((stage + kStages - (LAG - 1)) % kStages));
+        }
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+      }
+    }
+    // signal the stages still in flight
+    cp_async_wait<0>();
+    fence_proxy_async();
+    __syncwarp();
+    if (ok && lane == 0) {
+      for (int i = (issued < LAG - 1 ? issued : LAG - 1); i >= 1; --i)
+        mbar_arrive(full_bar((stage + kStages - i) % kStages));
+    }
+  } else if (MODE == 1 && warp == 0) {
+    // ------------------- producer (down): h tile and weight tile ------------
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
@@ -251,32 +402,18 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       const int tile = item / p.n_sub, ns = item % p.n_sub;
       const int g = p.tile_group[tile], row0 = p.tile_row0[tile];
       const int e = g / p.B, blk = g % p.B;
-      int tok[4] = {0, 0, 0, 0};
-      if (MODE == 0) {
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int t = p.row_tok[row0 + 4 * lane + j];
-          tok[j] = t < 0 ? 0 : t;  // padding rows read token 0; never reduced
-        }
-      }
-      // B rows: w_up viewed [(K+1)H][d] or w_down viewed [(K+1)d][H].
-      const int brow = (MODE == 0) ? e * p.H + blk * p.M + ns * p.bn : e * p.d + ns * p.bn;
+      const int brow = e * p.d + ns * p.bn;  // w_down viewed [(K+1)d][H]
       for (int kb = 0; kb < p.num_kb; ++kb) {
         bool w = true;
         if (lane == 0) w = wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
         ok = __shfl_sync(0xffffffffu, w, 0);
         if (!ok) break;
-        if (lane == 0) mbar_expect_tx(full_bar(stage), stage_bytes);
-        __syncwarp();
-        const uint32_t a_dst = sA + stage * kStageA, b_dst = sB + stage * kStageB;
-        if (MODE == 0) {
-          tma_gather4(a_dst + lane * 512u, &tmA, full_bar(stage), kb * kBK, tok[0], tok[1], tok[2],
-                      tok[3]);
-          if (lane == 0) tma_load_2d(b_dst, &tmB, full_bar(stage), kb * kBK, brow);
-        } else if (lane == 0) {
-          tma_load_2d(a_dst, &tmA, full_bar(stage), kb * kBK, row0);
-          tma_load_2d(b_dst, &tmB, full_bar(stage), blk * p.M + kb * kBK, brow);
+        if (lane == 0) {
+          mbar_expect_tx(full_bar(stage), stage_bytes);
+          tma_load_2d(sA + stage * kStageA, &tmA, full_bar(stage), kb * kBK, row0);
+          tma_load_2d(sB + stage * kStageB, &tmB, full_bar(stage), blk * p.M + kb * kBK, brow);
         }
+        __syncwarp();
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
       }
     }
@@ -331,35 +468,46 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)acc * kAccStride;
       const int c_begin = half * cols;
       if (MODE == 0) {
+        // h = bf16(GeLU(acc)), 32 columns per TMEM load, 64 B stores per row.
         __nv_bfloat16* dst = p.h + (size_t)row * p.M + ns * p.bn + c_begin;
-        for (int c = 0; c < cols; c += 16) {
-          float v[16];
-          tmem_ld16(t_row + c_begin + c, v);
-          uint4 o0, o1;
-          o0.x = pack_bf16(gelu_erf(v[0]), gelu_erf(v[1]));
-          o0.y = pack_bf16(gelu_erf(v[2]), gelu_erf(v[3]));
-          o0.z = pack_bf16(gelu_erf(v[4]), gelu_erf(v[5]));
-          o0.w = pack_bf16(gelu_erf(v[6]), gelu_erf(v[7]));
-          o1.x = pack_bf16(gelu_erf(v[8]), gelu_erf(v[9]));
-          o1.y = pack_bf16(gelu_erf(v[10]), gelu_erf(v[11]));
-          o1.z = pack_bf16(gelu_erf(v[12]), gelu_erf(v[13]));
-          o1.w = pack_bf16(gelu_erf(v[14]), gelu_erf(v[15]));
-          *reinterpret_cast<uint4*>(dst + c) = o0;
-          *reinterpret_cast<uint4*>(dst + c + 8) = o1;
+        for (int c = 0; c < cols; c += 32) {
+          float v[32];
+          tmem_ld32(t_row + c_begin + c, v);
+          uint32_t o[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) o[j] = gelu2_bf16x2(v[2 * j], v[2 * j + 1]);
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            *reinterpret_cast<uint4*>(dst + c + 8 * j) =
+                make_uint4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
         }
       } else {
+        // y[tok] += w * acc: each thread scales its row, the warp stages 32 rows x
+        // 32 columns in shared memory and adds them back row-contiguously (8 lanes
+        // x 16 B per row, 4 rows per instruction).
+        float* stg = staging + (size_t)(warp - kFirstEpiWarp) * 32 * kStageRow;
         const int t = p.row_tok[row];
         const float wt = p.row_w[row];
-        float* dst = p.y32 + (size_t)(t < 0 ? 0 : t) * p.d + ns * p.bn + c_begin;
-        for (int c = 0; c < cols; c += 16) {
-          float v[16];
-          tmem_ld16(t_row + c_begin + c, v);
-          if (t >= 0) {
+        const int r_sub = lane >> 3, c_sub = (lane & 7) * 4;
+        for (int c = 0; c < cols; c += 32) {
+          float v[32];
+          tmem_ld32(t_row + c_begin + c, v);
 #pragma unroll
-            for (int j = 0; j < 16; j += 4)
-              atomicAdd(reinterpret_cast<float4*>(dst + c + j),
-                        make_float4(wt * v[j], wt * v[j + 1], wt * v[j + 2], wt * v[j + 3]));
+          for (int j = 0; j < 32; j += 4)
+            *reinterpret_cast<float4*>(stg + lane * kStageRow + j) =
+                make_float4(wt * v[j], wt * v[j + 1], wt * v[j + 2], wt * v[j + 3]);
+          __syncwarp();
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int r = 4 * i + r_sub;
+            const int tr = __shfl_sync(0xffffffffu, t, r);
+            const float4 val = *reinterpret_cast<const float4*>(stg + r * kStageRow + c_sub);
+            if (tr >= 0)
+              atomicAdd(reinterpret_cast<float4*>(p.y32 + (size_t)tr * p.d + ns * p.bn + c_begin +
+                                                  c + c_sub),
+                        val);
           }
+          __syncwarp();
         }
       }
       tc_fence_before();
@@ -424,12 +572,14 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
   return r == CUDA_SUCCESS;
 }
 
-// N split into n_sub sub-tiles of bn columns: bn <= 256, bn % 32 == 0.
+// N split into n_sub sub-tiles of bn columns: bn <= 256 and bn % 64 == 0, so
+// that each of the two epilogue column halves is a whole number of 32-column
+// TMEM loads.
 bool pick_split(int n, int* bn, int* nsub) {
-  for (int s = 1; s <= n / 32; ++s) {
+  for (int s = 1; s <= n / 64; ++s) {
     if (n % s) continue;
     const int b = n / s;
-    if (b <= kMaxBN && b % 32 == 0) {
+    if (b <= kMaxBN && b % 64 == 0) {
       *bn = b;
       *nsub = s;
       return true;
@@ -455,38 +605,42 @@ int gemm_tc_setup(unif_moe_layer* L) {
     set_error("cuTensorMapEncodeTiled failed for the weight or activation maps");
     return UNIF_MOE_ERR_CUDA;
   }
-  for (auto fn : {tc::grouped_gemm_kernel<0>, tc::grouped_gemm_kernel<1>}) {
-    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)tc::kSmemBytes);
-    if (e != cudaSuccess) {
-      set_error("cudaFuncSetAttribute: %s", cudaGetErrorString(e));
-      return UNIF_MOE_ERR_CUDA;
-    }
+  cudaError_t e = cudaFuncSetAttribute(tc::grouped_gemm_kernel<0>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)tc::Cfg<0>::kSmem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc::grouped_gemm_kernel<1>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc::Cfg<1>::kSmem);
+  if (e != cudaSuccess) {
+    set_error("cudaFuncSetAttribute: %s", cudaGetErrorString(e));
+    return UNIF_MOE_ERR_CUDA;
   }
   return UNIF_MOE_OK;
 }
 
 cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
                             cudaStream_t s) {
-  CUtensorMap tm_x;
-  if (!tc::encode_2d(&tm_x, x, L->d, (uint64_t)T, tc::kBK, 1)) return cudaErrorInvalidValue;
+  (void)T;
   tc::Params p;
   p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group; p.tile_row0 = L->ws.tile_row0;
   p.row_tok = L->ws.row_tok; p.row_w = L->ws.row_w;
   p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;
+  p.x = static_cast<const __nv_bfloat16*>(x);
   p.h = static_cast<__nv_bfloat16*>(L->ws.hbuf);
   p.y32 = L->ws.y32;
   p.status = L->ws.status;
   p.wait_limit = tc::g_wait_limit;
   // up: N = M (block width), reduction over d
   p.n_sub = L->up_nsub; p.bn = L->up_bn; p.num_kb = L->d / tc::kBK;
-  tc::grouped_gemm_kernel<0><<<L->n_sm, tc::kThreads, tc::kSmemBytes, s>>>(tm_x, L->tm_wup, p);
+  tc::grouped_gemm_kernel<0><<<L->n_sm, tc::kThreads, tc::Cfg<0>::kSmem, s>>>(L->tm_h, L->tm_wup,
+                                                                             p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (mid) cudaEventRecord(mid, s);
   // down: N = d, reduction over the block's M channels
   p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
-  tc::grouped_gemm_kernel<1><<<L->n_sm, tc::kThreads, tc::kSmemBytes, s>>>(L->tm_h, L->tm_wdown, p);
+  tc::grouped_gemm_kernel<1><<<L->n_sm, tc::kThreads, tc::Cfg<1>::kSmem, s>>>(L->tm_h, L->tm_wdown,
+                                                                             p);
   return cudaGetLastError();
 }
 

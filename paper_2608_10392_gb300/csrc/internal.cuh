@@ -27,11 +27,9 @@ struct Workspace {
   int32_t* k = nullptr;          // [T]
   uint64_t* shr_mask = nullptr;  // [T]
   uint64_t* exp_mask = nullptr;  // [T] selected residual experts
-  int32_t* q = nullptr;          // [T][K]
-  float* p = nullptr;            // [T][K] sorted affinities
-  float* s = nullptr;            // [T][K] affinities by expert index
+  float* s = nullptr;            // [T][K] affinities by expert index (Eq. 24)
   // Group table.
-  int32_t* chunk_cnt = nullptr;  // [G][n_chunks]: counts, then exclusive offsets
+  int32_t* chunk_cnt = nullptr;  // [G][T/32]: counts, then exclusive offsets
   int32_t* grp_cnt = nullptr;    // [G]
   int32_t* grp_off = nullptr;    // [G+1] padded offsets
   int32_t* n_tiles = nullptr;    // [1]
@@ -65,13 +63,13 @@ struct unif_moe_layer {
   int64_t max_tiles = 0;
   int max_chunks = 0;
   int router_cols = 0;      // 1 + K + B
-  int router_cols_pad = 0;  // padded to 16
+  int router_cols_pad = 0;  // padded to a multiple of 32
   int n_sm = 0;
   int device = 0;
   bool loaded = false;
   int last_T = -1;
   // Weights (device, owned).
-  float* wr_t = nullptr;    // [router_cols_pad][d]: W_shr, W_g, mu_1..mu_B (fp32)
+  float* wr = nullptr;      // [d][router_cols_pad]: W_shr, W_g, mu_1..mu_B (fp32)
   float* bias = nullptr;    // [K+1]
   void* w_up = nullptr;     // [K+1][H][d]
   void* w_down = nullptr;   // [K+1][d][H]
@@ -97,6 +95,9 @@ cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask,
                           int32_t* b_out, int32_t* k_out, cudaStream_t s);
 cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s);
 cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s);
+cudaError_t launch_sort_affinities(unif_moe_layer* L, int T, int32_t* q, float* p,
+                                   cudaStream_t s);
+int forward_chunks(int T);
 cudaError_t launch_gemms_simt(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
                               cudaStream_t s);
 cudaError_t router_setup(unif_moe_layer* L);

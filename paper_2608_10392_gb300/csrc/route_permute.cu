@@ -35,26 +35,28 @@ __device__ __forceinline__ float round_f64_to_bf16(double v) {
 // Eq. 20: mu_b = (1/M) sum_{h in H_b} K_shr[:, h]. The sum of stored
 // (fp32/bf16) keys is exact in fp64 for these magnitudes, so the single
 // rounding below gives the same value on any summation order.
+// The router matrix is kept as [d][Cp] fp32: row i holds x_i's weights for
+// W_shr, W_g (columns 0..K) and mu_1..mu_B (columns K+1..K+B), zero padded.
 template <typename Tin>
 __global__ void prototypes_kernel(const Tin* __restrict__ w_up0, int d, int H, int B,
-                                  int round_bf16, float* __restrict__ mu_rows) {
+                                  int round_bf16, int Cp, int col0, float* __restrict__ wr) {
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= B * d) return;
   const int b = idx / d, i = idx % d, M = H / B;
   double sum = 0.0;
   for (int h = b * M; h < (b + 1) * M; ++h) sum += (double)to_f32(w_up0[(size_t)h * d + i]);
   const double m = sum / (double)M;
-  mu_rows[(size_t)b * d + i] = round_bf16 ? round_f64_to_bf16(m) : __double2float_rn(m);
+  wr[(size_t)i * Cp + col0 + b] = round_bf16 ? round_f64_to_bf16(m) : __double2float_rn(m);
 }
 
-// Router columns 0..K (Eq. 17) transposed to [column][d] in fp32.
+// Router columns 0..K (Eq. 17) into the [d][Cp] fp32 router matrix.
 template <typename Tin>
-__global__ void router_transpose_kernel(const Tin* __restrict__ w_router, int d, int C1,
-                                        float* __restrict__ wr_t) {
+__global__ void router_copy_kernel(const Tin* __restrict__ w_router, int d, int C1, int Cp,
+                                   float* __restrict__ wr) {
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= d * C1) return;
   const int i = idx / C1, c = idx % C1;
-  wr_t[(size_t)c * d + i] = to_f32(w_router[idx]);
+  wr[(size_t)i * Cp + c] = to_f32(w_router[idx]);
 }
 
 // ---------------------------------------------------------------------------
@@ -62,12 +64,13 @@ __global__ void router_transpose_kernel(const Tin* __restrict__ w_router, int d,
 // ---------------------------------------------------------------------------
 
 constexpr int kRouterThreads = 256;
-constexpr int kKc = 32;  // d-chunk of the router GEMM
+constexpr int kKc = 32;          // d-chunk of the router GEMM
+constexpr int kWarpChunk = 32;   // tokens per permute chunk on the forward path (one warp)
 
 struct RouterArgs {
   const uint8_t* mask;
-  int T, d, K, B, C, Cpad;
-  const float* wr_t;
+  int T, d, K, B;
+  const float* wr;  // [d][Cp] router matrix
   const float* bias;
   float tau, alpha_fixed, beta_fixed;
   int topk_fixed, prefix;
@@ -76,64 +79,90 @@ struct RouterArgs {
   int32_t* k;
   uint64_t* shr;
   uint64_t* emask;
-  int32_t* q;
-  float* p;
   float* s;
   int32_t* bcnt;
   int32_t* kcnt;
+  int32_t* chunk_cnt;  // [G][n_chunks]: (expert, block) pairs per 32-token chunk
+  int n_chunks;
+  float* y32;          // [T][d] output accumulator, zeroed here
 };
 
-__device__ __forceinline__ float warp_sum_ordered(float v) {
-  // Tree to lane 0, then broadcast: every lane sees the same value.
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
-  return __shfl_sync(0xffffffffu, v, 0);
+__device__ __forceinline__ void load8(const float* src, float (&v)[8]) {
+  const float4 a = *reinterpret_cast<const float4*>(src);
+  const float4 b = *reinterpret_cast<const float4*>(src + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void load8(const __nv_bfloat16* src, float (&v)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(src);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    v[2 * i] = __uint_as_float(w[i] << 16);
+    v[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+  }
 }
 
-__device__ __forceinline__ float warp_max(float v) {
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
+// Blocks of expert e that a token with shared set `shr` and residual expert
+// set `em` runs: the shared blocks for e = 0 (Eq. 28), the complementary
+// blocks for a selected residual expert (Eqs. 23, 29).
+__device__ __forceinline__ uint64_t expert_blocks(int e, uint64_t shr, uint64_t em,
+                                                  uint64_t full) {
+  if (e == 0) return shr;
+  return ((em >> (e - 1)) & 1ull) ? (~shr & full) : 0ull;
 }
 
-template <typename Tin>
+// One CTA: 64 tokens. z = x W on CUDA cores (fp32 accumulate), then one
+// thread per token takes the decisions of Eqs. 18-27, then each of the two
+// deciding warps counts its 32 tokens' (expert, block) pairs per group.
+// NCB = Cp / 32 column blocks (each thread: 4 tokens x 2 NCB columns).
+template <typename Tin, int NCB>
 __global__ void __launch_bounds__(kRouterThreads)
 router_kernel(const Tin* __restrict__ x, RouterArgs a) {
   extern __shared__ float sm[];
-  const int Cp = a.Cpad;
-  float* xs = sm;                           // [kKc][64]
-  float* ws = xs + kKc * kRouterTokens;     // [kKc][Cp]
-  float* zs = ws + kKc * Cp;                // [64][Cp + 1]
-  float* wscr = zs + kRouterTokens * (Cp + 1);  // per warp: s[64], psort[64], qsort[64]
+  constexpr int Cp = 32 * NCB;
+  const int K = a.K, B = a.B;
+  float* xs = sm;                               // [kKc][64]
+  float* ws = xs + kKc * kRouterTokens;         // [kKc][Cp]
+  float* zs = ws + kKc * Cp;                    // [64][Cp + 1] logits
+  float* ss = zs + kRouterTokens * (Cp + 1);    // [64][K + 1] affinities
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int t0 = blockIdx.x * kRouterTokens;
 
-  // ---- z = x W^T for 64 tokens x Cp columns (fp32 accumulate) ----
-  const int ty = tid >> 4, tx = tid & 15;  // 16 x 16 threads: 4 tokens x (Cp/16) cols
-  const int ncol = Cp / 16;
-  float acc[4][9];
+  // ---- z = x W for 64 tokens x Cp columns (Eqs. 17, 21) ----
+  const int ty = tid >> 4, tx = tid & 15;  // tokens 4ty..4ty+3, columns tx + 16 j
+  // The fp32 output accumulator rows of these 64 tokens start at zero (the
+  // down-projection adds into them).
+  {
+    const int rows = min(kRouterTokens, a.T - t0);
+    float4* yz = reinterpret_cast<float4*>(a.y32 + (size_t)t0 * a.d);
+    const int n4 = rows * a.d / 4;
+    for (int i = tid; i < n4; i += kRouterThreads) yz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  float acc[4][2 * NCB];
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
-    for (int j = 0; j < 9; ++j) acc[i][j] = 0.f;
-
+    for (int j = 0; j < 2 * NCB; ++j) acc[i][j] = 0.f;
   for (int k0 = 0; k0 < a.d; k0 += kKc) {
-    // x chunk: 64 tokens x 32 dims, 8 consecutive dims per thread.
     {
       const int tok = tid >> 2, dd = (tid & 3) * 8;
       const int t = t0 + tok;
       float v[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) v[e] = 0.f;
       if (t < a.T && k0 + dd < a.d) {
-        const Tin* src = x + (size_t)t * a.d + k0 + dd;
+        load8(x + (size_t)t * a.d + k0 + dd, v);
+      } else {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) v[e] = to_f32(src[e]);
+        for (int e = 0; e < 8; ++e) v[e] = 0.f;
       }
 #pragma unroll
       for (int e = 0; e < 8; ++e) xs[(dd + e) * kRouterTokens + tok] = v[e];
     }
-    for (int idx = tid; idx < kKc * Cp; idx += kRouterThreads) {
-      const int c = idx / kKc, kk = idx % kKc;
-      ws[kk * Cp + c] = (k0 + kk < a.d) ? a.wr_t[(size_t)c * a.d + k0 + kk] : 0.f;
+    // weight rows k0..k0+31 are contiguous in the [d][Cp] router matrix
+    for (int idx = tid; idx < kKc * Cp / 4; idx += kRouterThreads) {
+      const int kk = (idx * 4) / Cp;
+      float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (k0 + kk < a.d) w4 = reinterpret_cast<const float4*>(a.wr + (size_t)k0 * Cp)[idx];
+      reinterpret_cast<float4*>(ws)[idx] = w4;
     }
     __syncthreads();
 #pragma unroll 4
@@ -141,12 +170,10 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
       const float4 xv = *reinterpret_cast<const float4*>(&xs[kk * kRouterTokens + ty * 4]);
       const float xa[4] = {xv.x, xv.y, xv.z, xv.w};
 #pragma unroll
-      for (int j = 0; j < 9; ++j) {
-        if (j < ncol) {
-          const float w = ws[kk * Cp + tx + 16 * j];
+      for (int j = 0; j < 2 * NCB; ++j) {
+        const float w = ws[kk * Cp + tx + 16 * j];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) acc[i][j] = fmaf(xa[i], w, acc[i][j]);
-        }
+        for (int i = 0; i < 4; ++i) acc[i][j] = fmaf(xa[i], w, acc[i][j]);
       }
     }
     __syncthreads();
@@ -154,32 +181,18 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
-    for (int j = 0; j < 9; ++j)
-      if (j < ncol) zs[(ty * 4 + i) * (Cp + 1) + tx + 16 * j] = acc[i][j];
+    for (int j = 0; j < 2 * NCB; ++j) zs[(ty * 4 + i) * (Cp + 1) + tx + 16 * j] = acc[i][j];
   __syncthreads();
+  if (tid >= kRouterTokens) return;
 
-  // ---- decisions: one warp per token ----
-  float* s_w = wscr + warp * 192;
-  float* ps_w = s_w + 64;
-  int* qs_w = reinterpret_cast<int*>(ps_w + 64);
-  const int K = a.K, B = a.B;
-  for (int lt = warp; lt < kRouterTokens; lt += kRouterThreads / 32) {
-    const int t = t0 + lt;
-    if (t >= a.T) break;
-    const bool valid = (a.mask == nullptr) || a.mask[t] != 0;
-    const float* z = zs + lt * (Cp + 1);
-    if (!valid) {
-      if (lane == 0) {
-        a.alpha[t] = 0.f; a.b[t] = 0; a.k[t] = 0; a.shr[t] = 0ull; a.emask[t] = 0ull;
-        if (a.bcnt) a.bcnt[t] = 0;
-        if (a.kcnt) a.kcnt[t] = 0;
-      }
-      for (int j = lane; j < K; j += 32) {
-        a.q[(size_t)t * K + j] = j; a.p[(size_t)t * K + j] = 0.f; a.s[(size_t)t * K + j] = 0.f;
-      }
-      continue;
-    }
-    // Eq. 18, Eq. 19.
+  // ---- decisions: one thread per token ----
+  const int t = t0 + tid;
+  const bool valid = t < a.T && (a.mask == nullptr || a.mask[t] != 0);
+  float* z = zs + tid * (Cp + 1);
+  float* sv = ss + tid * (K + 1);
+  uint64_t shr = 0ull, em = 0ull;
+  if (valid) {
+    // Eq. 18 (shared demand) and Eq. 19 (shared block count).
     const float z0 = z[0] + (a.bias ? a.bias[0] : 0.f);
     float alpha;
     if (isnan(a.alpha_fixed)) {
@@ -188,126 +201,208 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
     } else {
       alpha = a.alpha_fixed;
     }
-    int bcount = __float2int_rn((float)B * alpha);
-    bcount = min(max(bcount, 0), B);
-    // Eqs. 21-23: rank of each block's priority (ties to the lower index).
-    uint64_t shr = 0ull;
-    for (int base = 0; base < B; base += 32) {
-      const int blk = base + lane;
-      bool in = false;
-      if (blk < B) {
-        if (a.prefix) {
-          in = blk < bcount;
-        } else {
-          const float ub = z[1 + K + blk];
-          int rank = 0;
-          for (int i = 0; i < B; ++i) {
-            const float ui = z[1 + K + i];
-            rank += (ui > ub) || (ui == ub && i < blk);
-          }
-          in = rank < bcount;
-        }
-      }
-      shr |= (uint64_t)__ballot_sync(0xffffffffu, in) << base;
-    }
-    // Eq. 24: softmax over the K residual logits.
-    float zl[2], el[2];
-    float m = -INFINITY;
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int j = lane + 32 * r;
-      zl[r] = (j < K) ? z[1 + j] + (a.bias ? a.bias[1 + j] : 0.f) : -INFINITY;
-      m = fmaxf(m, zl[r]);
-    }
-    m = warp_max(m);
-    float part = 0.f;
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int j = lane + 32 * r;
-      el[r] = (j < K) ? expf(zl[r] - m) : 0.f;
-      part += el[r];
-    }
-    const float den = warp_sum_ordered(part);
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int j = lane + 32 * r;
-      if (j < K) s_w[j] = el[r] / den;
-    }
-    __syncwarp();
-    // Eq. 25: rank by decreasing affinity (ties to the lower index). The
-    // identity fill keeps the sorted lists a permutation even for NaN logits.
-    for (int r = lane; r < K; r += 32) { ps_w[r] = 0.f; qs_w[r] = r; }
-    __syncwarp();
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int j = lane + 32 * r;
-      if (j < K) {
-        const float sj = s_w[j];
-        int rank = 0;
-        for (int i = 0; i < K; ++i) {
-          const float si = s_w[i];
-          rank += (si > sj) || (si == sj && i < j);
-        }
-        ps_w[rank] = sj;
-        qs_w[rank] = j;
-        a.s[(size_t)t * K + j] = sj;
-      }
-    }
-    __syncwarp();
-    // Eqs. 26-27: smallest prefix whose cumulative mass reaches beta.
-    const float beta = isnan(a.beta_fixed) ? 1.0f - alpha : a.beta_fixed;
-    int kcount = K;
-    if (a.topk_fixed > 0) {
-      kcount = a.topk_fixed;
+    const int bcount = min(max(__float2int_rn((float)B * alpha), 0), B);
+    // Eqs. 21-23: the bcount blocks of largest priority (ties: lower index).
+    if (a.prefix) {
+      shr = (bcount >= 64) ? ~0ull : ((1ull << bcount) - 1ull);
     } else {
-      int first = K;
-      for (int base = 0; base < K; base += 32) {
-        const int r = base + lane;
-        bool hit = false;
-        if (r < K) {
-          float P = 0.f;
-          for (int i = 0; i <= r; ++i) P += ps_w[i];
-          hit = P >= beta;
-        }
-        const unsigned bal = __ballot_sync(0xffffffffu, hit);
-        if (bal && first == K) first = base + __ffs(bal) - 1;
+      const float* u = z + 1 + K;
+      for (int r = 0; r < bcount; ++r) {
+        int best = -1;
+        for (int j = 0; j < B; ++j)
+          if (!((shr >> j) & 1ull) && (best < 0 || u[j] > u[best])) best = j;
+        shr |= 1ull << best;
       }
-      kcount = min(first + 1, K);
     }
-    uint64_t em = 0ull;
-    for (int i = 0; i < kcount; ++i) em |= 1ull << qs_w[i];
-    for (int r = lane; r < K; r += 32) {
-      a.q[(size_t)t * K + r] = qs_w[r];
-      a.p[(size_t)t * K + r] = ps_w[r];
+    // Eq. 24: affinities over the K residual experts.
+    float* l = z + 1;  // residual logits (bias added in place)
+    float m = -INFINITY;
+    for (int j = 0; j < K; ++j) {
+      l[j] += a.bias ? a.bias[1 + j] : 0.f;
+      m = fmaxf(m, l[j]);
     }
-    if (lane == 0) {
-      a.alpha[t] = alpha;
-      a.b[t] = bcount;
-      a.k[t] = kcount;
-      a.shr[t] = shr;
-      a.emask[t] = em;
-      if (a.bcnt) a.bcnt[t] = bcount;
-      if (a.kcnt) a.kcnt[t] = kcount;
+    float den = 0.f;
+    for (int j = 0; j < K; ++j) {
+      sv[j] = expf(l[j] - m);
+      den += sv[j];
     }
-    __syncwarp();
+    for (int j = 0; j < K; ++j) {
+      sv[j] = sv[j] / den;
+      a.s[(size_t)t * K + j] = sv[j];
+    }
+    // Eqs. 25-27: experts in decreasing affinity (decreasing logit, ties to
+    // the lower index) until the cumulative mass reaches beta.
+    const float beta = isnan(a.beta_fixed) ? 1.0f - alpha : a.beta_fixed;
+    int kcount = 0;
+    float P = 0.f;
+    for (int n = 0; n < K; ++n) {
+      int best = -1;
+      for (int j = 0; j < K; ++j)
+        if (!((em >> j) & 1ull) && (best < 0 || l[j] > l[best])) best = j;
+      em |= 1ull << best;
+      if (a.topk_fixed > 0) {
+        if (n + 1 == a.topk_fixed) { kcount = n + 1; break; }
+      } else {
+        P += sv[best];
+        if (P >= beta) { kcount = n + 1; break; }
+      }
+    }
+    if (kcount == 0) kcount = K;  // rounding left every prefix below beta
+    a.alpha[t] = alpha;
+    a.b[t] = bcount;
+    a.k[t] = kcount;
+    a.shr[t] = shr;
+    a.emask[t] = em;
+    if (a.bcnt) a.bcnt[t] = bcount;
+    if (a.kcnt) a.kcnt[t] = kcount;
+  } else if (t < a.T) {
+    a.alpha[t] = 0.f; a.b[t] = 0; a.k[t] = 0; a.shr[t] = 0ull; a.emask[t] = 0ull;
+    for (int j = 0; j < K; ++j) a.s[(size_t)t * K + j] = 0.f;
+    if (a.bcnt) a.bcnt[t] = 0;
+    if (a.kcnt) a.kcnt[t] = 0;
+  }
+
+  // ---- (expert, block) pairs per group for this warp's 32 tokens ----
+  const int chunk = blockIdx.x * (kRouterTokens / kWarpChunk) + warp;
+  if (chunk >= a.n_chunks) return;
+  const uint64_t full = (B == 64) ? ~0ull : ((1ull << B) - 1ull);
+  for (int e = 0; e <= K; ++e) {
+    const uint64_t mb = expert_blocks(e, shr, em, full);
+    const bool any = __ballot_sync(0xffffffffu, mb != 0ull) != 0u;
+    for (int blk = 0; blk < B; ++blk) {
+      const int g = e * B + blk;
+      const int c = any ? __popc(__ballot_sync(0xffffffffu, (mb >> blk) & 1ull)) : 0;
+      if (lane == (g & 31)) a.chunk_cnt[(size_t)g * a.n_chunks + chunk] = c;
+    }
+  }
+}
+
+// get_routing helper: experts by decreasing affinity (ties to the lower
+// index) and their affinities, one thread per token.
+__global__ void sort_affinities_kernel(const float* __restrict__ s, int T, int K,
+                                       int32_t* __restrict__ q, float* __restrict__ p) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  const float* st = s + (size_t)t * K;
+  uint64_t used = 0ull;
+  for (int n = 0; n < K; ++n) {
+    int best = -1;
+    for (int j = 0; j < K; ++j)
+      if (!((used >> j) & 1ull) && (best < 0 || st[j] > st[best])) best = j;
+    used |= 1ull << best;
+    if (q) q[(size_t)t * K + n] = best;
+    if (p) p[(size_t)t * K + n] = st[best];
+  }
+}
+
+// Per group: exclusive scan over the 32-token chunks (in place) and the
+// group's row count. One warp per group.
+__global__ void __launch_bounds__(256)
+chunk_scan_kernel(int G, int n_chunks, int32_t* __restrict__ chunk_cnt,
+                  int32_t* __restrict__ grp_cnt) {
+  const int lane = threadIdx.x & 31;
+  const int g = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (g >= G) return;
+  int32_t* col = chunk_cnt + (size_t)g * n_chunks;
+  int carry = 0;
+  for (int c0 = 0; c0 < n_chunks; c0 += 32) {
+    const int c = c0 + lane;
+    const int v = (c < n_chunks) ? col[c] : 0;
+    int inc = v;
+    for (int o = 1; o < 32; o <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += n;
+    }
+    if (c < n_chunks) col[c] = carry + inc - v;
+    carry += __shfl_sync(0xffffffffu, inc, 31);
+  }
+  if (lane == 0) grp_cnt[g] = carry;
+}
+
+// Stable scatter of the (token, weight) rows into their groups, four 32-token
+// chunks per CTA (one per warp). Every CTA first scans the groups' padded
+// sizes into offsets (shared memory); CTA c also writes the tile list and the
+// padding rows of groups g = c, c + gridDim.x, ...
+__global__ void __launch_bounds__(128)
+group_scatter_kernel(const uint64_t* __restrict__ shr_o, const uint64_t* __restrict__ em_o,
+                     const float* __restrict__ alpha_o, const float* __restrict__ s_o, int T,
+                     int K, int B, int n_chunks, const int32_t* __restrict__ chunk_off,
+                     const int32_t* __restrict__ grp_cnt, int32_t* __restrict__ grp_off,
+                     int32_t* __restrict__ n_tiles, int32_t* __restrict__ tile_group,
+                     int32_t* __restrict__ tile_row0, int32_t* __restrict__ row_tok,
+                     float* __restrict__ row_w) {
+  extern __shared__ int goff[];  // [G + 1]
+  __shared__ int wsum[4];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int G = (K + 1) * B;
+  const int per = (G + 127) / 128;
+  const int ga = min(G, tid * per), gb = min(G, ga + per);
+  int mine = 0;
+  for (int g = ga; g < gb; ++g) mine += (grp_cnt[g] + kTileRows - 1) / kTileRows * kTileRows;
+  int inc = mine;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int n = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += n;
+  }
+  if (lane == 31) wsum[warp] = inc;
+  __syncthreads();
+  int base = inc - mine;
+  for (int w = 0; w < warp; ++w) base += wsum[w];
+  for (int g = ga; g < gb; ++g) {
+    goff[g] = base;
+    base += (grp_cnt[g] + kTileRows - 1) / kTileRows * kTileRows;
+  }
+  if (tid == 127) goff[G] = base;
+  __syncthreads();
+  // side outputs: offsets, tile list, padding rows
+  for (int g = blockIdx.x; g < G; g += gridDim.x) {
+    const int cnt = grp_cnt[g], off = goff[g];
+    const int padded = (cnt + kTileRows - 1) / kTileRows * kTileRows;
+    if (tid == 0) grp_off[g] = off;
+    for (int i = tid; i < padded / kTileRows; i += 128) {
+      tile_group[off / kTileRows + i] = g;
+      tile_row0[off / kTileRows + i] = off + i * kTileRows;
+    }
+    for (int r = off + cnt + tid; r < off + padded; r += 128) { row_tok[r] = -1; row_w[r] = 0.f; }
+  }
+  if (blockIdx.x == 0 && tid == 0) {
+    grp_off[G] = goff[G];
+    n_tiles[0] = goff[G] / kTileRows;
+  }
+  // scatter
+  const int chunk = blockIdx.x * 4 + warp;
+  if (chunk >= n_chunks) return;
+  const int t = chunk * kWarpChunk + lane;
+  const uint64_t full = (B == 64) ? ~0ull : ((1ull << B) - 1ull);
+  const uint64_t shr = (t < T) ? shr_o[t] : 0ull;
+  const uint64_t em = (t < T) ? em_o[t] : 0ull;
+  const unsigned lt_mask = (1u << lane) - 1u;
+  for (int e = 0; e <= K; ++e) {
+    const uint64_t mb = expert_blocks(e, shr, em, full);
+    if (__ballot_sync(0xffffffffu, mb != 0ull) == 0u) continue;
+    const float w = (mb == 0ull) ? 0.f : (e == 0 ? alpha_o[t] : s_o[(size_t)t * K + e - 1]);
+    for (int blk = 0; blk < B; ++blk) {
+      const int g = e * B + blk;
+      const bool f = (mb >> blk) & 1ull;
+      const unsigned bal = __ballot_sync(0xffffffffu, f);
+      if (f) {
+        const int pos = goff[g] + chunk_off[(size_t)g * n_chunks + chunk] + __popc(bal & lt_mask);
+        row_tok[pos] = t;
+        row_w[pos] = w;
+      }
+    }
   }
 }
 
 // ---------------------------------------------------------------------------
-// Permute: (expert, block) group table
+// Permute with 256-token chunks and its own counting pass (used by the
+// allocation-free grouping entry point below)
 // ---------------------------------------------------------------------------
 
 constexpr int kPermThreads = kChunkTokens;  // one token per thread
 constexpr int kPermWarps = kPermThreads / 32;
 constexpr int kGroupBatch = 1024;           // groups per shared-memory pass
 
-// Blocks of expert e that token (shr, em) runs: the shared blocks for e = 0,
-// the complementary blocks for a selected residual expert (Eqs. 22-23, 28-29).
-__device__ __forceinline__ uint64_t expert_blocks(int e, uint64_t shr, uint64_t em,
-                                                  uint64_t full) {
-  if (e == 0) return shr;
-  return ((em >> (e - 1)) & 1ull) ? (~shr & full) : 0ull;
-}
 
 __global__ void __launch_bounds__(kPermThreads)
 count_kernel(const uint64_t* __restrict__ shr_o, const uint64_t* __restrict__ em_o, int T,
@@ -496,24 +591,24 @@ __global__ void copy_out_f32(const float4* __restrict__ y, float4* __restrict__ 
 
 cudaError_t launch_prototypes(unif_moe_layer* L, const void* w_router, const float* bias,
                               cudaStream_t s) {
-  cudaError_t e = cudaMemsetAsync(L->wr_t, 0, sizeof(float) * L->router_cols_pad * L->d, s);
+  const int Cp = L->router_cols_pad;
+  cudaError_t e = cudaMemsetAsync(L->wr, 0, sizeof(float) * Cp * L->d, s);
   if (e != cudaSuccess) return e;
   const int C1 = L->K + 1;
   const int n1 = L->d * C1;
   if (L->dtype == UNIF_MOE_BF16)
-    router_transpose_kernel<<<(n1 + 255) / 256, 256, 0, s>>>(
-        static_cast<const __nv_bfloat16*>(w_router), L->d, C1, L->wr_t);
+    router_copy_kernel<<<(n1 + 255) / 256, 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(w_router), L->d, C1, Cp, L->wr);
   else
-    router_transpose_kernel<<<(n1 + 255) / 256, 256, 0, s>>>(static_cast<const float*>(w_router),
-                                                             L->d, C1, L->wr_t);
+    router_copy_kernel<<<(n1 + 255) / 256, 256, 0, s>>>(static_cast<const float*>(w_router),
+                                                        L->d, C1, Cp, L->wr);
   const int n2 = L->B * L->d;
-  float* mu_rows = L->wr_t + (size_t)C1 * L->d;
   if (L->dtype == UNIF_MOE_BF16)
     prototypes_kernel<<<(n2 + 255) / 256, 256, 0, s>>>(
-        static_cast<const __nv_bfloat16*>(L->w_up), L->d, L->H, L->B, 1, mu_rows);
+        static_cast<const __nv_bfloat16*>(L->w_up), L->d, L->H, L->B, 1, Cp, C1, L->wr);
   else
     prototypes_kernel<<<(n2 + 255) / 256, 256, 0, s>>>(static_cast<const float*>(L->w_up), L->d,
-                                                       L->H, L->B, 0, mu_rows);
+                                                       L->H, L->B, 0, Cp, C1, L->wr);
   if (bias)
     e = cudaMemcpyAsync(L->bias, bias, sizeof(float) * C1, cudaMemcpyDeviceToDevice, s);
   else
@@ -525,49 +620,67 @@ cudaError_t launch_prototypes(unif_moe_layer* L, const void* w_router, const flo
 static size_t router_smem(const unif_moe_layer* L) {
   const int Cp = L->router_cols_pad;
   return sizeof(float) * ((size_t)kKc * kRouterTokens + (size_t)kKc * Cp +
-                          (size_t)kRouterTokens * (Cp + 1) + 8 * 192);
+                          (size_t)kRouterTokens * (Cp + 1) + (size_t)kRouterTokens * (L->K + 1));
+}
+
+int forward_chunks(int T) { return (T + kWarpChunk - 1) / kWarpChunk; }
+
+template <typename Tin>
+static void* router_fn(int ncb) {
+  switch (ncb) {
+    case 1: return reinterpret_cast<void*>(router_kernel<Tin, 1>);
+    case 2: return reinterpret_cast<void*>(router_kernel<Tin, 2>);
+    case 3: return reinterpret_cast<void*>(router_kernel<Tin, 3>);
+    case 4: return reinterpret_cast<void*>(router_kernel<Tin, 4>);
+    default: return reinterpret_cast<void*>(router_kernel<Tin, 5>);
+  }
+}
+
+static void* router_entry(const unif_moe_layer* L) {
+  const int ncb = L->router_cols_pad / 32;  // 1 + K + B <= 129 columns: ncb <= 5
+  return L->dtype == UNIF_MOE_BF16 ? router_fn<__nv_bfloat16>(ncb) : router_fn<float>(ncb);
 }
 
 cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
                           int32_t* b_out, int32_t* k_out, cudaStream_t s) {
   RouterArgs a;
   a.mask = mask; a.T = T; a.d = L->d; a.K = L->K; a.B = L->B;
-  a.C = L->router_cols; a.Cpad = L->router_cols_pad;
-  a.wr_t = L->wr_t; a.bias = L->bias;
+  a.wr = L->wr; a.bias = L->bias;
   a.tau = L->tau; a.alpha_fixed = L->th.alpha_fixed; a.beta_fixed = L->th.beta_fixed;
   a.topk_fixed = L->th.topk_fixed; a.prefix = L->th.prefix_blocks;
   a.alpha = L->ws.alpha; a.b = L->ws.b; a.k = L->ws.k; a.shr = L->ws.shr_mask;
-  a.emask = L->ws.exp_mask; a.q = L->ws.q; a.p = L->ws.p; a.s = L->ws.s;
+  a.emask = L->ws.exp_mask; a.s = L->ws.s;
   a.bcnt = b_out; a.kcnt = k_out;
-  const size_t smem = router_smem(L);
+  a.chunk_cnt = L->ws.chunk_cnt; a.n_chunks = forward_chunks(T);
+  a.y32 = L->ws.y32;
+  const void* xp = x;
+  void* args[] = {const_cast<void**>(&xp), &a};
   const int grid = (T + kRouterTokens - 1) / kRouterTokens;
-  if (L->dtype == UNIF_MOE_BF16)
-    router_kernel<__nv_bfloat16><<<grid, kRouterThreads, smem, s>>>(
-        static_cast<const __nv_bfloat16*>(x), a);
-  else
-    router_kernel<float><<<grid, kRouterThreads, smem, s>>>(static_cast<const float*>(x), a);
-  return cudaGetLastError();
+  return cudaLaunchKernel(router_entry(L), dim3(grid), dim3(kRouterThreads), args, router_smem(L),
+                          s);
 }
 
 cudaError_t router_setup(unif_moe_layer* L) {
-  const int smem = (int)router_smem(L);
-  cudaError_t e = cudaFuncSetAttribute(router_kernel<__nv_bfloat16>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = cudaFuncSetAttribute(router_entry(L), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)router_smem(L));
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(router_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              smem);
+  return cudaFuncSetAttribute(group_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)(sizeof(int) * (L->G + 1)));
 }
 
 cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s) {
-  const int n_chunks = (T + kChunkTokens - 1) / kChunkTokens;
+  const int n_chunks = forward_chunks(T);
   Workspace& w = L->ws;
-  count_kernel<<<n_chunks, kPermThreads, 0, s>>>(w.shr_mask, w.exp_mask, T, L->K, L->B, n_chunks,
-                                                 w.chunk_cnt);
-  scan_kernel<<<1, 1024, 0, s>>>(L->G, n_chunks, w.chunk_cnt, w.grp_cnt, w.grp_off, w.n_tiles,
-                                 w.tile_group, w.tile_row0, w.row_tok, w.row_w);
-  scatter_kernel<<<n_chunks, kPermThreads, 0, s>>>(w.shr_mask, w.exp_mask, w.alpha, w.s, T, L->K,
-                                                   L->B, n_chunks, w.chunk_cnt, w.grp_off,
-                                                   w.row_tok, w.row_w);
+  chunk_scan_kernel<<<(L->G + 7) / 8, 256, 0, s>>>(L->G, n_chunks, w.chunk_cnt, w.grp_cnt);
+  group_scatter_kernel<<<(n_chunks + 3) / 4, 128, sizeof(int) * (L->G + 1), s>>>(
+      w.shr_mask, w.exp_mask, w.alpha, w.s, T, L->K, L->B, n_chunks, w.chunk_cnt, w.grp_cnt,
+      w.grp_off, w.n_tiles, w.tile_group, w.tile_row0, w.row_tok, w.row_w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sort_affinities(unif_moe_layer* L, int T, int32_t* q, float* p,
+                                   cudaStream_t s) {
+  sort_affinities_kernel<<<(T + 127) / 128, 128, 0, s>>>(L->ws.s, T, L->K, q, p);
   return cudaGetLastError();
 }
 

@@ -62,8 +62,8 @@ int dalloc(T** p, size_t count) {
 }
 
 void free_all(unif_moe_layer* L) {
-  void* ptrs[] = {L->wr_t, L->bias, L->w_up, L->w_down, L->ws.alpha, L->ws.b, L->ws.k,
-                  L->ws.shr_mask, L->ws.exp_mask, L->ws.q, L->ws.p, L->ws.s, L->ws.chunk_cnt,
+  void* ptrs[] = {L->wr, L->bias, L->w_up, L->w_down, L->ws.alpha, L->ws.b, L->ws.k,
+                  L->ws.shr_mask, L->ws.exp_mask, L->ws.s, L->ws.chunk_cnt,
                   L->ws.grp_cnt, L->ws.grp_off, L->ws.n_tiles, L->ws.tile_group,
                   L->ws.tile_row0, L->ws.row_tok, L->ws.row_w, L->ws.hbuf, L->ws.y32,
                   L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
@@ -146,9 +146,9 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
     return UNIF_MOE_ERR_CAPACITY;
   }
   L->max_tiles = L->max_rows / unif::kTileRows;
-  L->max_chunks = (max_tokens + unif::kChunkTokens - 1) / unif::kChunkTokens;
+  L->max_chunks = unif::forward_chunks(max_tokens);
   L->router_cols = 1 + n_experts + n_blocks;
-  L->router_cols_pad = (L->router_cols + 15) / 16 * 16;
+  L->router_cols_pad = (L->router_cols + 31) / 32 * 32;
   if (cudaGetDevice(&L->device) != cudaSuccess ||
       cudaDeviceGetAttribute(&L->n_sm, cudaDevAttrMultiProcessorCount, L->device) != cudaSuccess) {
     set_error("no CUDA device");
@@ -169,7 +169,7 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   int rc = UNIF_MOE_OK;
 #define ALLOC(ptr, n)                          \
   if (rc == UNIF_MOE_OK) rc = dalloc(&(ptr), (n));
-  ALLOC(L->wr_t, (size_t)L->router_cols_pad * d_model);
+  ALLOC(L->wr, (size_t)L->router_cols_pad * d_model);
   ALLOC(L->bias, E);
   void* wup = nullptr;
   void* wdn = nullptr;
@@ -177,7 +177,7 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&wdn), es * E * d_ff * d_model);
   L->w_up = wup; L->w_down = wdn;
   ALLOC(w.alpha, T); ALLOC(w.b, T); ALLOC(w.k, T); ALLOC(w.shr_mask, T); ALLOC(w.exp_mask, T);
-  ALLOC(w.q, T * K); ALLOC(w.p, T * K); ALLOC(w.s, T * K);
+  ALLOC(w.s, T * K);
   ALLOC(w.chunk_cnt, (size_t)L->G * L->max_chunks);
   ALLOC(w.grp_cnt, (size_t)L->G); ALLOC(w.grp_off, (size_t)L->G + 1); ALLOC(w.n_tiles, 1);
   ALLOC(w.tile_group, (size_t)L->max_tiles); ALLOC(w.tile_row0, (size_t)L->max_tiles);
@@ -188,7 +188,8 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   ALLOC(w.y32, T * d_model);
   ALLOC(w.status, 1);
 #undef ALLOC
-  if (rc == UNIF_MOE_OK && cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess) {
+  if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
+                            cudaMemset(w.y32, 0, sizeof(float) * T * d_model) != cudaSuccess)) {
     set_error("cudaMemset failed");
     rc = UNIF_MOE_ERR_CUDA;
   }
@@ -244,7 +245,6 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = L->stage_ev;
   if (ev[0]) CK(cudaEventRecord(ev[0], s));
-  CK(cudaMemsetAsync(L->ws.y32, 0, sizeof(float) * (size_t)T * L->d, s));
   CK(unif::launch_router(L, x, token_mask, T, shared_counts, residual_counts, s));
   if (ev[1]) CK(cudaEventRecord(ev[1], s));
   CK(unif::launch_permute(L, T, s));
@@ -312,8 +312,7 @@ int unif_moe_get_routing(unif_moe_t L, float* alpha, uint64_t* shared_mask, uint
     if (alpha) CK(cudaMemcpyAsync(alpha, L->ws.alpha, sizeof(float) * T, dd, s));
     if (shared_mask) CK(cudaMemcpyAsync(shared_mask, L->ws.shr_mask, sizeof(uint64_t) * T, dd, s));
     if (expert_mask) CK(cudaMemcpyAsync(expert_mask, L->ws.exp_mask, sizeof(uint64_t) * T, dd, s));
-    if (q) CK(cudaMemcpyAsync(q, L->ws.q, sizeof(int32_t) * T * K, dd, s));
-    if (p) CK(cudaMemcpyAsync(p, L->ws.p, sizeof(float) * T * K, dd, s));
+    if (q || p) CK(unif::launch_sort_affinities(L, (int)T, q, p, s));
   }
   CK(cudaStreamSynchronize(s));
   return UNIF_MOE_OK;
