@@ -31,6 +31,7 @@
 // kStatusTimeout in the handle's status word and the CTA unwinds.
 #include <stdio.h>
 
+#include "decide.cuh"
 #include "internal.cuh"
 
 namespace unif {
@@ -47,6 +48,7 @@ constexpr int kMaxBN = 256;
 constexpr uint32_t kStageA = kBM * kBK * 2;      // 16 KB
 constexpr uint32_t kStageB = kMaxBN * kBK * 2;   // 32 KB
 constexpr int kStageRow = 36;                    // fp32 per staged row (32 + 4 pad, 16 B aligned)
+constexpr uint32_t kHStageRow = 80;              // bytes per staged h row (64 + 16 pad)
 
 // Per-kernel shared memory: the up kernel keeps 4 operand stages; the down
 // kernel keeps 3 and a per-warp 32 x 32 fp32 staging tile that turns its
@@ -54,7 +56,9 @@ constexpr int kStageRow = 36;                    // fp32 per staged row (32 + 4 
 template <int MODE>
 struct Cfg {
   static constexpr int kStages = MODE == 0 ? 4 : 3;
-  static constexpr uint32_t kStaging = MODE == 0 ? 0u : kEpiWarps * 32u * kStageRow * 4u;
+  // up: 32 rows x 32 bf16 per warp (80-byte rows); down: 32 rows x 32 fp32
+  static constexpr uint32_t kStaging =
+      MODE == 0 ? kEpiWarps * 32u * kHStageRow : kEpiWarps * 32u * kStageRow * 4u;
   static constexpr size_t kSmem = 1024 + kStages * (kStageA + kStageB) + kStaging + 256;
 };
 
@@ -342,8 +346,12 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     // chunk j ^ (r mod 8)); lane 0 of warp 0 also brings the weight tile by TMA.
     // A stage is signalled LAG stages after its copies were issued, once
     // cp.async.wait_group shows them complete.
-    constexpr int LAG = 2;
-    const int rbase = (warp == 0 ? 0 : 64) + lane;  // rows rbase and rbase + 32
+    constexpr int LAG = 3;
+    // Each warp covers 64 rows; instruction i of a stage copies rows
+    // r = base + 4 i + lane / 8 (16-byte chunk j = lane % 8 of each), so a
+    // warp instruction reads 4 whole 128-byte rows.
+    const int base = warp == 0 ? 0 : 64;
+    const int j = lane & 7, rsub = lane >> 3;
     int stage = 0;
     uint32_t phase = 0;
     int issued = 0;
@@ -352,11 +360,13 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       const int tile = item / p.n_sub, ns = item % p.n_sub;
       const int g = p.tile_group[tile], row0 = p.tile_row0[tile];
       const int e = g / p.B, blk = g % p.B;
-      int t0 = p.row_tok[row0 + rbase], t1 = p.row_tok[row0 + rbase + 32];
-      t0 = t0 < 0 ? 0 : t0;  // padding rows read token 0; their results are never used
-      t1 = t1 < 0 ? 0 : t1;
-      const __nv_bfloat16* src0 = p.x + (size_t)t0 * p.d;
-      const __nv_bfloat16* src1 = p.x + (size_t)t1 * p.d;
+      // tokens of this lane's 16 rows (padding rows read token 0; never used)
+      const __nv_bfloat16* src[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int t = p.row_tok[row0 + base + 4 * i + rsub];
+        src[i] = p.x + (size_t)(t < 0 ? 0 : t) * p.d + j * 8;
+      }
       const int brow = e * p.H + blk * p.M + ns * p.bn;
       for (int kb = 0; kb < p.num_kb; ++kb) {
         bool w = true;
@@ -369,10 +379,9 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
           tma_load_2d(sB + stage * kStageB, &tmB, full_bar(stage), kb * kBK, brow);
         }
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          cp_async16(a_dst + rbase * 128u + ((j ^ (rbase & 7)) << 4), src0 + kb * kBK + j * 8);
-          cp_async16(a_dst + (rbase + 32) * 128u + ((j ^ (rbase & 7)) << 4),
-                     src1 + kb * kBK + j * 8);
+        for (int i = 0; i < 16; ++i) {
+          const int r = base + 4 * i + rsub;
+          cp_async16(a_dst + r * 128u + ((j ^ (r & 7)) << 4), src[i] + kb * kBK);
         }
         cp_async_commit();
         ++issued;
@@ -468,18 +477,30 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)acc * kAccStride;
       const int c_begin = half * cols;
       if (MODE == 0) {
-        // h = bf16(GeLU(acc)), 32 columns per TMEM load, 64 B stores per row.
-        __nv_bfloat16* dst = p.h + (size_t)row * p.M + ns * p.bn + c_begin;
+        // h = bf16(GeLU(acc)), 32 columns per TMEM load. Each thread stages its
+        // row's 64 bytes; the warp then stores 8 rows x 64 contiguous bytes per
+        // instruction.
+        uint8_t* stg = reinterpret_cast<uint8_t*>(staging) +
+                       (size_t)(warp - kFirstEpiWarp) * 32 * kHStageRow;
+        __nv_bfloat16* hrow0 = p.h + (size_t)(row0 + q * 32) * p.M + ns * p.bn + c_begin;
         for (int c = 0; c < cols; c += 32) {
           float v[32];
           tmem_ld32(t_row + c_begin + c, v);
           uint32_t o[16];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) o[j] = gelu2_bf16x2(v[2 * j], v[2 * j + 1]);
+          for (int jj = 0; jj < 16; ++jj) o[jj] = gelu2_bf16x2(v[2 * jj], v[2 * jj + 1]);
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            *reinterpret_cast<uint4*>(dst + c + 8 * j) =
-                make_uint4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
+          for (int jj = 0; jj < 4; ++jj)
+            *reinterpret_cast<uint4*>(stg + lane * kHStageRow + 16 * jj) =
+                make_uint4(o[4 * jj], o[4 * jj + 1], o[4 * jj + 2], o[4 * jj + 3]);
+          __syncwarp();
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int r = 8 * i + (lane >> 2), seg = lane & 3;
+            *reinterpret_cast<uint4*>(hrow0 + (size_t)r * p.M + c + seg * 8) =
+                *reinterpret_cast<const uint4*>(stg + r * kHStageRow + 16 * seg);
+          }
+          __syncwarp();
         }
       } else {
         // y[tok] += w * acc: each thread scales its row, the warp stages 32 rows x
@@ -534,6 +555,143 @@ __global__ void timeout_probe_kernel(int* status, long long limit) {
     mbar_init(smem_u32(&bar), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     wait_bounded(smem_u32(&bar), 0u, &abort_flag, status, limit);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Router on the tensor cores (bf16 layers)
+// ---------------------------------------------------------------------------
+// One CTA per 128 tokens: z = x [W_shr | W_g | mu] as a 128 x Cp x d MMA
+// (Eqs. 17, 21), TMA-fed, fp32 accumulator in TMEM. Each of the four decision
+// warps then owns 32 tokens = 32 TMEM lanes: a thread reads its token's Cp
+// logits, takes the decisions of Eqs. 18-27 and the warp counts its chunk's
+// (expert, block) pairs.
+constexpr int kRtThreads = 192;   // warp 0 TMA, warp 1 TMEM + MMA, warps 2-5 decisions
+constexpr int kRtStages = 4;
+constexpr uint32_t kRtStageB = 160u * kBK * 2;  // up to 160 router columns
+constexpr size_t kRtSmem = 1024 + kRtStages * (kStageA + kRtStageB) + 256;
+
+struct RouterTcParams {
+  DecideArgs dec;
+  int d, Cp;
+  uint32_t tmem_cols;
+  float* y32;
+  int* status;
+  long long wait_limit;
+};
+
+__global__ void __launch_bounds__(kRtThreads, 1)
+router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
+                 RouterTcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sA = smem_u32(smem);
+  const uint32_t sB = sA + kRtStages * kStageA;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kRtStages * (kStageA + kRtStageB));
+  const uint32_t bar0 = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (kRtStages + s); };
+  const uint32_t accf = bar0 + 8u * (2 * kRtStages);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kRtStages + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t0 = blockIdx.x * kBM;
+  const int Cp = p.Cp, K = p.dec.K;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kRtStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(accf, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), p.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  // the output accumulator rows of these tokens start at zero
+  {
+    const int rows = min(kBM, p.dec.T - t0);
+    float4* yz = reinterpret_cast<float4*>(p.y32 + (size_t)t0 * p.d);
+    const int n4 = rows * p.d / 4;
+    for (int i = threadIdx.x; i < n4; i += kRtThreads) yz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  const int num_kb = p.d / kBK;
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      const uint32_t bytes = kStageA + (uint32_t)Cp * kBK * 2;
+      for (int kb = 0; kb < num_kb; ++kb) {
+        if (!wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit)) break;
+        mbar_expect_tx(full_bar(stage), bytes);
+        tma_load_2d(sA + stage * kStageA, &tm_x, full_bar(stage), kb * kBK, t0);
+        tma_load_2d(sB + stage * kRtStageB, &tm_w, full_bar(stage), kb * kBK, 0);
+        if (++stage == kRtStages) { stage = 0; phase ^= 1u; }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(kBM, Cp);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int kb = 0; kb < num_kb; ++kb) {
+        if (!wait_bounded(full_bar(stage), phase, abort_flag, p.status, p.wait_limit)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_base = sA + stage * kStageA, b_base = sB + stage * kRtStageB;
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k)
+          umma_bf16(tmem_base, sw128_desc(a_base + k * 32), sw128_desc(b_base + k * 32), idesc,
+                    (kb | k) != 0 ? 1u : 0u);
+        umma_commit(empty_bar(stage));
+        if (++stage == kRtStages) { stage = 0; phase ^= 1u; }
+      }
+      if (ok) umma_commit(accf);
+    }
+    __syncwarp();
+  } else {
+    // decision warps: lane quarter q = warp % 4 holds tokens t0 + 32 q + lane
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    bool w = true;
+    if (lane == 0) w = wait_bounded(accf, 0u, abort_flag, p.status, p.wait_limit);
+    if (__shfl_sync(0xffffffffu, w, 0)) {
+      tc_fence_after();
+      // logits and affinities overlay the (now idle) operand ring
+      float* zs = reinterpret_cast<float*>(smem);
+      float* ss = zs + kBM * (Cp + 1);
+      float* z = zs + row * (Cp + 1);
+      for (int c = 0; c < Cp; c += 32) {
+        float v[32];
+        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + c, v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) z[c + i] = v[i];
+      }
+      const int t = t0 + row;
+      const bool valid = t < p.dec.T && (p.dec.mask == nullptr || p.dec.mask[t] != 0);
+      uint64_t shr, em;
+      decide_token(p.dec, t, valid, z, ss + row * (K + 1), shr, em);
+      const int chunk = blockIdx.x * (kBM / 32) + q;
+      if (chunk < p.dec.n_chunks) count_chunk_pairs(p.dec, chunk, lane, shr, em);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, p.tmem_cols);
   }
 }
 
@@ -641,6 +799,41 @@ cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t
   p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
   tc::grouped_gemm_kernel<1><<<L->n_sm, tc::kThreads, tc::Cfg<1>::kSmem, s>>>(L->tm_h, L->tm_wdown,
                                                                              p);
+  return cudaGetLastError();
+}
+
+int router_tc_setup(unif_moe_layer* L) {
+  if (L->router_cols_pad > 160 || L->d % tc::kBK != 0) {
+    set_error("tensor-core router needs 1+K+B <= 160 and d %% 64 == 0");
+    return UNIF_MOE_ERR_SHAPE;
+  }
+  if (!tc::encode_2d(&L->tm_wr, L->wr_bf, L->d, L->router_cols_pad, tc::kBK,
+                     L->router_cols_pad)) {
+    set_error("cuTensorMapEncodeTiled failed for the router matrix");
+    return UNIF_MOE_ERR_CUDA;
+  }
+  if (cudaFuncSetAttribute(tc::router_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)tc::kRtSmem) != cudaSuccess) {
+    set_error("cudaFuncSetAttribute failed for the router kernel");
+    return UNIF_MOE_ERR_CUDA;
+  }
+  return UNIF_MOE_OK;
+}
+
+cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
+                             int32_t* b_out, int32_t* k_out, cudaStream_t s) {
+  CUtensorMap tm_x;
+  if (!tc::encode_2d(&tm_x, x, L->d, (uint64_t)T, tc::kBK, tc::kBM)) return cudaErrorInvalidValue;
+  tc::RouterTcParams p;
+  p.dec = decide_args(L, mask, T, b_out, k_out);
+  p.d = L->d;
+  p.Cp = L->router_cols_pad;
+  p.tmem_cols = p.Cp <= 32 ? 32u : (p.Cp <= 64 ? 64u : (p.Cp <= 128 ? 128u : 256u));
+  p.y32 = L->ws.y32;
+  p.status = L->ws.status;
+  p.wait_limit = tc::g_wait_limit;
+  tc::router_tc_kernel<<<(T + tc::kBM - 1) / tc::kBM, tc::kRtThreads, tc::kRtSmem, s>>>(
+      tm_x, L->tm_wr, p);
   return cudaGetLastError();
 }
 

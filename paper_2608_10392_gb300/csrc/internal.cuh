@@ -70,6 +70,7 @@ struct unif_moe_layer {
   int last_T = -1;
   // Weights (device, owned).
   float* wr = nullptr;      // [d][router_cols_pad]: W_shr, W_g, mu_1..mu_B (fp32)
+  __nv_bfloat16* wr_bf = nullptr;  // [router_cols_pad][d] the same matrix in bf16 (bf16 layers)
   float* bias = nullptr;    // [K+1]
   void* w_up = nullptr;     // [K+1][H][d]
   void* w_down = nullptr;   // [K+1][d][H]
@@ -78,6 +79,7 @@ struct unif_moe_layer {
   CUtensorMap tm_wup;
   CUtensorMap tm_wdown;
   CUtensorMap tm_h;
+  CUtensorMap tm_wr;
   int up_bn = 0, up_nsub = 0, down_bn = 0, down_nsub = 0;
   // Optional caller-owned timing events recorded at the stage boundaries.
   cudaEvent_t stage_ev[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
@@ -106,5 +108,8 @@ int gemm_tc_setup(unif_moe_layer* L);  // tensor maps of weights and h; returns 
 cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
                             cudaStream_t s);
 cudaError_t launch_timeout_probe(unif_moe_layer* L, int timeout_us, cudaStream_t s);
+int router_tc_setup(unif_moe_layer* L);
+cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
+                             int32_t* b_out, int32_t* k_out, cudaStream_t s);
 
 }  // namespace unif

@@ -11,6 +11,7 @@
 //   combine : casts the fp32 accumulator of Eq. 30 to the layer dtype.
 #include <math.h>
 
+#include "decide.cuh"
 #include "internal.cuh"
 
 namespace unif {
@@ -49,6 +50,17 @@ __global__ void prototypes_kernel(const Tin* __restrict__ w_up0, int d, int H, i
   wr[(size_t)i * Cp + col0 + b] = round_bf16 ? round_f64_to_bf16(m) : __double2float_rn(m);
 }
 
+// The router matrix as bf16 [Cp][d] (K-major operand of the tensor-core
+// router). Every entry is a bf16 value already (bf16 weights, prototypes
+// rounded to bf16, zero padding), so the conversion is exact.
+__global__ void router_to_bf16_kernel(const float* __restrict__ wr, int d, int Cp,
+                                      __nv_bfloat16* __restrict__ wr_bf) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= d * Cp) return;
+  const int c = idx / d, i = idx % d;
+  wr_bf[idx] = __float2bfloat16_rn(wr[(size_t)i * Cp + c]);
+}
+
 // Router columns 0..K (Eq. 17) into the [d][Cp] fp32 router matrix.
 template <typename Tin>
 __global__ void router_copy_kernel(const Tin* __restrict__ w_router, int d, int C1, int Cp,
@@ -68,23 +80,10 @@ constexpr int kKc = 32;          // d-chunk of the router GEMM
 constexpr int kWarpChunk = 32;   // tokens per permute chunk on the forward path (one warp)
 
 struct RouterArgs {
-  const uint8_t* mask;
-  int T, d, K, B;
+  DecideArgs dec;
+  int d;
   const float* wr;  // [d][Cp] router matrix
-  const float* bias;
-  float tau, alpha_fixed, beta_fixed;
-  int topk_fixed, prefix;
-  float* alpha;
-  int32_t* b;
-  int32_t* k;
-  uint64_t* shr;
-  uint64_t* emask;
-  float* s;
-  int32_t* bcnt;
-  int32_t* kcnt;
-  int32_t* chunk_cnt;  // [G][n_chunks]: (expert, block) pairs per 32-token chunk
-  int n_chunks;
-  float* y32;          // [T][d] output accumulator, zeroed here
+  float* y32;       // [T][d] output accumulator, zeroed here
 };
 
 __device__ __forceinline__ void load8(const float* src, float (&v)[8]) {
@@ -102,15 +101,6 @@ __device__ __forceinline__ void load8(const __nv_bfloat16* src, float (&v)[8]) {
   }
 }
 
-// Blocks of expert e that a token with shared set `shr` and residual expert
-// set `em` runs: the shared blocks for e = 0 (Eq. 28), the complementary
-// blocks for a selected residual expert (Eqs. 23, 29).
-__device__ __forceinline__ uint64_t expert_blocks(int e, uint64_t shr, uint64_t em,
-                                                  uint64_t full) {
-  if (e == 0) return shr;
-  return ((em >> (e - 1)) & 1ull) ? (~shr & full) : 0ull;
-}
-
 // One CTA: 64 tokens. z = x W on CUDA cores (fp32 accumulate), then one
 // thread per token takes the decisions of Eqs. 18-27, then each of the two
 // deciding warps counts its 32 tokens' (expert, block) pairs per group.
@@ -120,7 +110,7 @@ __global__ void __launch_bounds__(kRouterThreads)
 router_kernel(const Tin* __restrict__ x, RouterArgs a) {
   extern __shared__ float sm[];
   constexpr int Cp = 32 * NCB;
-  const int K = a.K, B = a.B;
+  const int K = a.dec.K;
   float* xs = sm;                               // [kKc][64]
   float* ws = xs + kKc * kRouterTokens;         // [kKc][Cp]
   float* zs = ws + kKc * Cp;                    // [64][Cp + 1] logits
@@ -133,7 +123,7 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
   // The fp32 output accumulator rows of these 64 tokens start at zero (the
   // down-projection adds into them).
   {
-    const int rows = min(kRouterTokens, a.T - t0);
+    const int rows = min(kRouterTokens, a.dec.T - t0);
     float4* yz = reinterpret_cast<float4*>(a.y32 + (size_t)t0 * a.d);
     const int n4 = rows * a.d / 4;
     for (int i = tid; i < n4; i += kRouterThreads) yz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -148,7 +138,7 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
       const int tok = tid >> 2, dd = (tid & 3) * 8;
       const int t = t0 + tok;
       float v[8];
-      if (t < a.T && k0 + dd < a.d) {
+      if (t < a.dec.T && k0 + dd < a.d) {
         load8(x + (size_t)t * a.d + k0 + dd, v);
       } else {
 #pragma unroll
@@ -187,94 +177,13 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
 
   // ---- decisions: one thread per token ----
   const int t = t0 + tid;
-  const bool valid = t < a.T && (a.mask == nullptr || a.mask[t] != 0);
-  float* z = zs + tid * (Cp + 1);
-  float* sv = ss + tid * (K + 1);
-  uint64_t shr = 0ull, em = 0ull;
-  if (valid) {
-    // Eq. 18 (shared demand) and Eq. 19 (shared block count).
-    const float z0 = z[0] + (a.bias ? a.bias[0] : 0.f);
-    float alpha;
-    if (isnan(a.alpha_fixed)) {
-      const float sig = 1.0f / (1.0f + expf(-z0));
-      alpha = a.tau + (1.0f - 2.0f * a.tau) * sig;
-    } else {
-      alpha = a.alpha_fixed;
-    }
-    const int bcount = min(max(__float2int_rn((float)B * alpha), 0), B);
-    // Eqs. 21-23: the bcount blocks of largest priority (ties: lower index).
-    if (a.prefix) {
-      shr = (bcount >= 64) ? ~0ull : ((1ull << bcount) - 1ull);
-    } else {
-      const float* u = z + 1 + K;
-      for (int r = 0; r < bcount; ++r) {
-        int best = -1;
-        for (int j = 0; j < B; ++j)
-          if (!((shr >> j) & 1ull) && (best < 0 || u[j] > u[best])) best = j;
-        shr |= 1ull << best;
-      }
-    }
-    // Eq. 24: affinities over the K residual experts.
-    float* l = z + 1;  // residual logits (bias added in place)
-    float m = -INFINITY;
-    for (int j = 0; j < K; ++j) {
-      l[j] += a.bias ? a.bias[1 + j] : 0.f;
-      m = fmaxf(m, l[j]);
-    }
-    float den = 0.f;
-    for (int j = 0; j < K; ++j) {
-      sv[j] = expf(l[j] - m);
-      den += sv[j];
-    }
-    for (int j = 0; j < K; ++j) {
-      sv[j] = sv[j] / den;
-      a.s[(size_t)t * K + j] = sv[j];
-    }
-    // Eqs. 25-27: experts in decreasing affinity (decreasing logit, ties to
-    // the lower index) until the cumulative mass reaches beta.
-    const float beta = isnan(a.beta_fixed) ? 1.0f - alpha : a.beta_fixed;
-    int kcount = 0;
-    float P = 0.f;
-    for (int n = 0; n < K; ++n) {
-      int best = -1;
-      for (int j = 0; j < K; ++j)
-        if (!((em >> j) & 1ull) && (best < 0 || l[j] > l[best])) best = j;
-      em |= 1ull << best;
-      if (a.topk_fixed > 0) {
-        if (n + 1 == a.topk_fixed) { kcount = n + 1; break; }
-      } else {
-        P += sv[best];
-        if (P >= beta) { kcount = n + 1; break; }
-      }
-    }
-    if (kcount == 0) kcount = K;  // rounding left every prefix below beta
-    a.alpha[t] = alpha;
-    a.b[t] = bcount;
-    a.k[t] = kcount;
-    a.shr[t] = shr;
-    a.emask[t] = em;
-    if (a.bcnt) a.bcnt[t] = bcount;
-    if (a.kcnt) a.kcnt[t] = kcount;
-  } else if (t < a.T) {
-    a.alpha[t] = 0.f; a.b[t] = 0; a.k[t] = 0; a.shr[t] = 0ull; a.emask[t] = 0ull;
-    for (int j = 0; j < K; ++j) a.s[(size_t)t * K + j] = 0.f;
-    if (a.bcnt) a.bcnt[t] = 0;
-    if (a.kcnt) a.kcnt[t] = 0;
-  }
+  const bool valid = t < a.dec.T && (a.dec.mask == nullptr || a.dec.mask[t] != 0);
+  uint64_t shr, em;
+  decide_token(a.dec, t, valid, zs + tid * (Cp + 1), ss + tid * (K + 1), shr, em);
 
   // ---- (expert, block) pairs per group for this warp's 32 tokens ----
   const int chunk = blockIdx.x * (kRouterTokens / kWarpChunk) + warp;
-  if (chunk >= a.n_chunks) return;
-  const uint64_t full = (B == 64) ? ~0ull : ((1ull << B) - 1ull);
-  for (int e = 0; e <= K; ++e) {
-    const uint64_t mb = expert_blocks(e, shr, em, full);
-    const bool any = __ballot_sync(0xffffffffu, mb != 0ull) != 0u;
-    for (int blk = 0; blk < B; ++blk) {
-      const int g = e * B + blk;
-      const int c = any ? __popc(__ballot_sync(0xffffffffu, (mb >> blk) & 1ull)) : 0;
-      if (lane == (g & 31)) a.chunk_cnt[(size_t)g * a.n_chunks + chunk] = c;
-    }
-  }
+  if (chunk < a.dec.n_chunks) count_chunk_pairs(a.dec, chunk, lane, shr, em);
 }
 
 // get_routing helper: experts by decreasing affinity (ties to the lower
@@ -369,24 +278,34 @@ group_scatter_kernel(const uint64_t* __restrict__ shr_o, const uint64_t* __restr
     grp_off[G] = goff[G];
     n_tiles[0] = goff[G] / kTileRows;
   }
-  // scatter
+  // scatter: each warp first stages its chunk's per-group offsets and its
+  // tokens' affinities in shared memory, so the loop below only waits on
+  // shared-memory reads
   const int chunk = blockIdx.x * 4 + warp;
   if (chunk >= n_chunks) return;
+  int* coff = goff + (G + 1) + warp * G;
+  float* sw = reinterpret_cast<float*>(goff + (G + 1) + 4 * G) + warp * 32 * K;
+  for (int g = lane; g < G; g += 32) coff[g] = goff[g] + chunk_off[(size_t)g * n_chunks + chunk];
   const int t = chunk * kWarpChunk + lane;
+  const int tfirst = chunk * kWarpChunk;
+  const int nvalid = min(kWarpChunk, T - tfirst);
+  for (int i = lane; i < nvalid * K; i += 32) sw[i] = s_o[(size_t)tfirst * K + i];
+  __syncwarp();
   const uint64_t full = (B == 64) ? ~0ull : ((1ull << B) - 1ull);
   const uint64_t shr = (t < T) ? shr_o[t] : 0ull;
   const uint64_t em = (t < T) ? em_o[t] : 0ull;
+  const float alpha = (t < T) ? alpha_o[t] : 0.f;
   const unsigned lt_mask = (1u << lane) - 1u;
   for (int e = 0; e <= K; ++e) {
     const uint64_t mb = expert_blocks(e, shr, em, full);
     if (__ballot_sync(0xffffffffu, mb != 0ull) == 0u) continue;
-    const float w = (mb == 0ull) ? 0.f : (e == 0 ? alpha_o[t] : s_o[(size_t)t * K + e - 1]);
+    const float w = (mb == 0ull) ? 0.f : (e == 0 ? alpha : sw[lane * K + e - 1]);
     for (int blk = 0; blk < B; ++blk) {
       const int g = e * B + blk;
       const bool f = (mb >> blk) & 1ull;
       const unsigned bal = __ballot_sync(0xffffffffu, f);
       if (f) {
-        const int pos = goff[g] + chunk_off[(size_t)g * n_chunks + chunk] + __popc(bal & lt_mask);
+        const int pos = coff[g] + __popc(bal & lt_mask);
         row_tok[pos] = t;
         row_w[pos] = w;
       }
@@ -609,6 +528,8 @@ cudaError_t launch_prototypes(unif_moe_layer* L, const void* w_router, const flo
   else
     prototypes_kernel<<<(n2 + 255) / 256, 256, 0, s>>>(static_cast<const float*>(L->w_up), L->d,
                                                        L->H, L->B, 0, Cp, C1, L->wr);
+  if (L->dtype == UNIF_MOE_BF16)
+    router_to_bf16_kernel<<<(L->d * Cp + 255) / 256, 256, 0, s>>>(L->wr, L->d, Cp, L->wr_bf);
   if (bias)
     e = cudaMemcpyAsync(L->bias, bias, sizeof(float) * C1, cudaMemcpyDeviceToDevice, s);
   else
@@ -624,6 +545,20 @@ static size_t router_smem(const unif_moe_layer* L) {
 }
 
 int forward_chunks(int T) { return (T + kWarpChunk - 1) / kWarpChunk; }
+
+DecideArgs decide_args(unif_moe_layer* L, const uint8_t* mask, int T, int32_t* b_out,
+                       int32_t* k_out) {
+  DecideArgs a;
+  a.mask = mask; a.T = T; a.K = L->K; a.B = L->B;
+  a.bias = L->bias;
+  a.tau = L->tau; a.alpha_fixed = L->th.alpha_fixed; a.beta_fixed = L->th.beta_fixed;
+  a.topk_fixed = L->th.topk_fixed; a.prefix = L->th.prefix_blocks;
+  a.alpha = L->ws.alpha; a.b = L->ws.b; a.k = L->ws.k; a.shr = L->ws.shr_mask;
+  a.emask = L->ws.exp_mask; a.s = L->ws.s;
+  a.bcnt = b_out; a.kcnt = k_out;
+  a.chunk_cnt = L->ws.chunk_cnt; a.n_chunks = forward_chunks(T);
+  return a;
+}
 
 template <typename Tin>
 static void* router_fn(int ncb) {
@@ -644,14 +579,9 @@ static void* router_entry(const unif_moe_layer* L) {
 cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
                           int32_t* b_out, int32_t* k_out, cudaStream_t s) {
   RouterArgs a;
-  a.mask = mask; a.T = T; a.d = L->d; a.K = L->K; a.B = L->B;
-  a.wr = L->wr; a.bias = L->bias;
-  a.tau = L->tau; a.alpha_fixed = L->th.alpha_fixed; a.beta_fixed = L->th.beta_fixed;
-  a.topk_fixed = L->th.topk_fixed; a.prefix = L->th.prefix_blocks;
-  a.alpha = L->ws.alpha; a.b = L->ws.b; a.k = L->ws.k; a.shr = L->ws.shr_mask;
-  a.emask = L->ws.exp_mask; a.s = L->ws.s;
-  a.bcnt = b_out; a.kcnt = k_out;
-  a.chunk_cnt = L->ws.chunk_cnt; a.n_chunks = forward_chunks(T);
+  a.dec = decide_args(L, mask, T, b_out, k_out);
+  a.d = L->d;
+  a.wr = L->wr;
   a.y32 = L->ws.y32;
   const void* xp = x;
   void* args[] = {const_cast<void**>(&xp), &a};
@@ -660,19 +590,23 @@ cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask,
                           s);
 }
 
+static size_t scatter_smem(const unif_moe_layer* L) {
+  return sizeof(int) * ((size_t)L->G + 1 + 4 * (size_t)L->G) + sizeof(float) * 4 * 32 * L->K;
+}
+
 cudaError_t router_setup(unif_moe_layer* L) {
   cudaError_t e = cudaFuncSetAttribute(router_entry(L), cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)router_smem(L));
   if (e != cudaSuccess) return e;
   return cudaFuncSetAttribute(group_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)(sizeof(int) * (L->G + 1)));
+                              (int)scatter_smem(L));
 }
 
 cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s) {
   const int n_chunks = forward_chunks(T);
   Workspace& w = L->ws;
   chunk_scan_kernel<<<(L->G + 7) / 8, 256, 0, s>>>(L->G, n_chunks, w.chunk_cnt, w.grp_cnt);
-  group_scatter_kernel<<<(n_chunks + 3) / 4, 128, sizeof(int) * (L->G + 1), s>>>(
+  group_scatter_kernel<<<(n_chunks + 3) / 4, 128, scatter_smem(L), s>>>(
       w.shr_mask, w.exp_mask, w.alpha, w.s, T, L->K, L->B, n_chunks, w.chunk_cnt, w.grp_cnt,
       w.grp_off, w.n_tiles, w.tile_group, w.tile_row0, w.row_tok, w.row_w);
   return cudaGetLastError();

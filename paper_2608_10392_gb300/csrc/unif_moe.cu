@@ -62,7 +62,7 @@ int dalloc(T** p, size_t count) {
 }
 
 void free_all(unif_moe_layer* L) {
-  void* ptrs[] = {L->wr, L->bias, L->w_up, L->w_down, L->ws.alpha, L->ws.b, L->ws.k,
+  void* ptrs[] = {L->wr, L->wr_bf, L->bias, L->w_up, L->w_down, L->ws.alpha, L->ws.b, L->ws.k,
                   L->ws.shr_mask, L->ws.exp_mask, L->ws.s, L->ws.chunk_cnt,
                   L->ws.grp_cnt, L->ws.grp_off, L->ws.n_tiles, L->ws.tile_group,
                   L->ws.tile_row0, L->ws.row_tok, L->ws.row_w, L->ws.hbuf, L->ws.y32,
@@ -170,6 +170,7 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
 #define ALLOC(ptr, n)                          \
   if (rc == UNIF_MOE_OK) rc = dalloc(&(ptr), (n));
   ALLOC(L->wr, (size_t)L->router_cols_pad * d_model);
+  if (dtype == UNIF_MOE_BF16) ALLOC(L->wr_bf, (size_t)L->router_cols_pad * d_model);
   ALLOC(L->bias, E);
   void* wup = nullptr;
   void* wdn = nullptr;
@@ -198,6 +199,7 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
     rc = UNIF_MOE_ERR_CUDA;
   }
   if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::gemm_tc_setup(L);
+  if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::router_tc_setup(L);
   if (rc != UNIF_MOE_OK) {
     free_all(L);
     delete L;
@@ -245,7 +247,11 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = L->stage_ev;
   if (ev[0]) CK(cudaEventRecord(ev[0], s));
-  CK(unif::launch_router(L, x, token_mask, T, shared_counts, residual_counts, s));
+  if (L->dtype == UNIF_MOE_BF16) {
+    CK(unif::launch_router_tc(L, x, token_mask, T, shared_counts, residual_counts, s));
+  } else {
+    CK(unif::launch_router(L, x, token_mask, T, shared_counts, residual_counts, s));
+  }
   if (ev[1]) CK(cudaEventRecord(ev[1], s));
   CK(unif::launch_permute(L, T, s));
   if (ev[2]) CK(cudaEventRecord(ev[2], s));
