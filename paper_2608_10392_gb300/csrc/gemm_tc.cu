@@ -9,14 +9,15 @@
 // (Eq. 16 split at the activation; w = alpha for the shared expert and p_i
 // for residual expert q_i, Eq. 30).
 //
-// Roles inside one CTA (one CTA per SM, 384 threads):
-//   warps 0, 2  up kernel: gather the tile's 128 token rows of x with 16-byte
-//               cp.async into the swizzled operand layout; warp 0 lane 0 also
-//               loads the weight tile with TMA
+// Roles inside one CTA (one CTA per SM, 416 threads):
+//   warps 0-3   up kernel: warp p owns the ring stages s = p (mod 4); it
+//               gathers the stage's 128 token rows of x with 16-byte cp.async
+//               into the swizzled operand layout, brings the weight tile with
+//               TMA, and signals the stage as soon as its own copies landed
 //   warp 0      down kernel: TMA of the h tile and the weight tile
-//   warp 1      TMEM allocator and MMA issuer (one lane): 128 x BN x 16
+//   warp 4      TMEM allocator and MMA issuer (one lane): 128 x BN x 16
 //               kind::f16 MMAs, fp32 accumulators in TMEM
-//   warps 4-11  epilogue: tcgen05.ld of the accumulator, GeLU -> bf16 h
+//   warps 5-12  epilogue: tcgen05.ld of the accumulator, GeLU -> bf16 h
 //               (up), or weight-scale -> fp32 atomic add into y (down)
 // Shared-memory stages are a 4-deep ring (full/empty mbarriers); the TMEM
 // accumulator is double-buffered (2 x 256 columns) so the epilogue of one
@@ -39,9 +40,11 @@ namespace tc {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;
-constexpr int kThreads = 384;
+constexpr int kThreads = 416;     // 13 warps
+constexpr int kProducerWarps = 4;  // warps 0-3
+constexpr int kMmaWarp = 4;        // TMEM allocation and MMA issue
 constexpr int kEpiWarps = 8;
-constexpr int kFirstEpiWarp = 4;
+constexpr int kFirstEpiWarp = 5;   // warps 5-12 (warp % 4 covers every TMEM lane quarter twice)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccStride = 256;  // TMEM columns per accumulator buffer
 constexpr int kMaxBN = 256;
@@ -59,7 +62,8 @@ struct Cfg {
   // up: 32 rows x 32 bf16 per warp (80-byte rows); down: 32 rows x 32 fp32
   static constexpr uint32_t kStaging =
       MODE == 0 ? kEpiWarps * 32u * kHStageRow : kEpiWarps * 32u * kStageRow * 4u;
-  static constexpr size_t kSmem = 1024 + kStages * (kStageA + kStageB) + kStaging + 256;
+  static constexpr uint32_t kTokens = MODE == 0 ? kProducerWarps * kBM * 4u : 0u;
+  static constexpr size_t kSmem = 1024 + kStages * (kStageA + kStageB) + kStaging + kTokens + 256;
 };
 
 struct Params {
@@ -90,6 +94,9 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx_only(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
@@ -304,8 +311,9 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
   const uint32_t sA = smem_u32(smem);
   const uint32_t sB = sA + kStages * kStageA;
   float* staging = reinterpret_cast<float*>(smem + kStages * (kStageA + kStageB));
+  int* tok_smem = reinterpret_cast<int*>(smem + kStages * (kStageA + kStageB) + Cfg<MODE>::kStaging);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * (kStageA + kStageB) +
-                                               Cfg<MODE>::kStaging);
+                                               Cfg<MODE>::kStaging + Cfg<MODE>::kTokens);
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
   auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
@@ -317,7 +325,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(full_bar(s), MODE == 0 ? 3 : 1);
+      mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -327,7 +335,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
   }
@@ -339,77 +347,72 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
   // Bytes the TMA brings per stage (the up kernel gathers A with cp.async).
   const uint32_t stage_bytes = (MODE == 0 ? 0u : kStageA) + (uint32_t)p.bn * kBK * 2;
 
-  if (MODE == 0 && (warp == 0 || warp == 2)) {
-    // ------------------- producer (up): gathered x rows ----------------------
-    // Warps 0 and 2 copy the 128 token rows of a stage with 16-byte cp.async
-    // into the 128-byte-swizzled layout (16-byte chunk j of row r lands at
-    // chunk j ^ (r mod 8)); lane 0 of warp 0 also brings the weight tile by TMA.
-    // A stage is signalled LAG stages after its copies were issued, once
-    // cp.async.wait_group shows them complete.
-    constexpr int LAG = 3;
-    // Each warp covers 64 rows; instruction i of a stage copies rows
-    // r = base + 4 i + lane / 8 (16-byte chunk j = lane % 8 of each), so a
-    // warp instruction reads 4 whole 128-byte rows.
-    const int base = warp == 0 ? 0 : 64;
+  if (MODE == 0 && warp < kProducerWarps) {
+    // ------------------- producers (up): stage owners ----------------------
+    // Warp p handles the stages whose sequence number is p mod 4. For its
+    // stage it copies the 128 token rows (instruction i covers rows
+    // 4 i .. 4 i + 3, one 16-byte chunk per lane, so each instruction reads 4
+    // whole 128-byte rows), waits for its own copies, fences them for the
+    // tensor cores (async proxy) and signals the stage. Lane 0 also brings the
+    // stage's weight tile with TMA.
+    static_assert(Cfg<0>::kStages == kProducerWarps, "one ring stage per producer warp");
     const int j = lane & 7, rsub = lane >> 3;
-    int stage = 0;
-    uint32_t phase = 0;
-    int issued = 0;
+    int seq = 0;  // stage sequence number over all items of this CTA
     bool ok = true;
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
       const int tile = item / p.n_sub, ns = item % p.n_sub;
-      const int g = p.tile_group[tile], row0 = p.tile_row0[tile];
+      // does this warp own any stage of this item?
+      int first = (warp - seq % kProducerWarps + kProducerWarps) % kProducerWarps;
+      if (first >= p.num_kb) { seq += p.num_kb; continue; }
+      const int g = p.tile_group[tile];
       const int e = g / p.B, blk = g % p.B;
-      // tokens of this lane's 16 rows (padding rows read token 0; never used)
-      const __nv_bfloat16* src[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int t = p.row_tok[row0 + base + 4 * i + rsub];
-        src[i] = p.x + (size_t)(t < 0 ? 0 : t) * p.d + j * 8;
-      }
       const int brow = e * p.H + blk * p.M + ns * p.bn;
-      for (int kb = 0; kb < p.num_kb; ++kb) {
+      // this tile's 128 row tokens, in the warp's own shared-memory slot
+      int* tok = tok_smem + warp * kBM;
+      __syncwarp();
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int t = p.row_tok[tile * kBM + 32 * i + lane];  // padding rows: token 0, unused
+        tok[32 * i + lane] = t < 0 ? 0 : t;
+      }
+      __syncwarp();
+      const __nv_bfloat16* xj = p.x + j * 8;
+      for (int kb = first; kb < p.num_kb; kb += kProducerWarps) {
+        const int sq = seq + kb;
+        const int stage = sq % kProducerWarps;  // == warp
+        const uint32_t phase = (uint32_t)(sq / kProducerWarps) & 1u;
         bool w = true;
         if (lane == 0) w = wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
         ok = __shfl_sync(0xffffffffu, w, 0);
         if (!ok) break;
-        const uint32_t a_dst = sA + stage * kStageA;
-        if (warp == 0 && lane == 0) {
-          mbar_expect_tx(full_bar(stage), stage_bytes);
+        if (lane == 0) {
+          mbar_expect_tx_only(full_bar(stage), stage_bytes);
           tma_load_2d(sB + stage * kStageB, &tmB, full_bar(stage), kb * kBK, brow);
         }
+        const uint32_t a_dst = sA + stage * kStageA;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int r = base + 4 * i + rsub;
-          cp_async16(a_dst + r * 128u + ((j ^ (r & 7)) << 4), src[i] + kb * kBK);
+        for (int i = 0; i < 32; ++i) {
+          const int r = 4 * i + rsub;
+          cp_async16(a_dst + r * 128u + ((j ^ (r & 7)) << 4), xj + (size_t)tok[r] * p.d + kb * kBK);
         }
         cp_async_commit();
-        ++issued;
-        if (issued >= LAG) {
-          cp_async_wait<LAG - 1>();
-          fence_proxy_async();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(full_bar((stage + kStages - (LAG - 1)) % kStages));
-        }
-        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        cp_async_wait<0>();
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(full_bar(stage));
       }
-    }
-    // signal the stages still in flight
-    cp_async_wait<0>();
-    fence_proxy_async();
-    __syncwarp();
-    if (ok && lane == 0) {
-      for (int i = (issued < LAG - 1 ? issued : LAG - 1); i >= 1; --i)
-        mbar_arrive(full_bar((stage + kStages - i) % kStages));
+      seq += p.num_kb;
     }
   } else if (MODE == 1 && warp == 0) {
     // ------------------- producer (down): h tile and weight tile ------------
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
+    int g_nxt = (blockIdx.x < n_items) ? p.tile_group[blockIdx.x / p.n_sub] : 0;
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
       const int tile = item / p.n_sub, ns = item % p.n_sub;
-      const int g = p.tile_group[tile], row0 = p.tile_row0[tile];
+      const int g = g_nxt, row0 = tile * kBM;
+      if (item + (int)gridDim.x < n_items) g_nxt = p.tile_group[(item + gridDim.x) / p.n_sub];
       const int e = g / p.B, blk = g % p.B;
       const int brow = e * p.d + ns * p.bn;  // w_down viewed [(K+1)d][H]
       for (int kb = 0; kb < p.num_kb; ++kb) {
@@ -426,7 +429,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
     // ------------------------------ MMA issuer ----------------------------
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(kBM, p.bn);
@@ -466,9 +469,24 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     const int cols = p.bn / 2;
     int acc = 0;
     uint32_t acc_phase = 0;
+    // down: this thread's row token and weight, fetched one tile ahead
+    int t_nxt = 0;
+    float w_nxt = 0.f;
+    if (MODE == 1 && blockIdx.x < n_items) {
+      const int r = (blockIdx.x / p.n_sub) * kBM + q * 32 + lane;
+      t_nxt = p.row_tok[r];
+      w_nxt = p.row_w[r];
+    }
     for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
       const int tile = item / p.n_sub, ns = item % p.n_sub;
-      const int row0 = p.tile_row0[tile];
+      const int row0 = tile * kBM;
+      const int t_cur = t_nxt;
+      const float w_cur = w_nxt;
+      if (MODE == 1 && item + (int)gridDim.x < n_items) {
+        const int r = ((item + gridDim.x) / p.n_sub) * kBM + q * 32 + lane;
+        t_nxt = p.row_tok[r];
+        w_nxt = p.row_w[r];
+      }
       bool w = true;
       if (lane == 0) w = wait_bounded(accf_bar(acc), acc_phase, abort_flag, p.status, p.wait_limit);
       if (!__shfl_sync(0xffffffffu, w, 0)) break;
@@ -484,15 +502,18 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                        (size_t)(warp - kFirstEpiWarp) * 32 * kHStageRow;
         __nv_bfloat16* hrow0 = p.h + (size_t)(row0 + q * 32) * p.M + ns * p.bn + c_begin;
         for (int c = 0; c < cols; c += 32) {
-          float v[32];
-          tmem_ld32(t_row + c_begin + c, v);
-          uint32_t o[16];
 #pragma unroll
-          for (int jj = 0; jj < 16; ++jj) o[jj] = gelu2_bf16x2(v[2 * jj], v[2 * jj + 1]);
+          for (int hh = 0; hh < 2; ++hh) {  // two 16-column TMEM loads keep register use low
+            float v[16];
+            tmem_ld16(t_row + c_begin + c + 16 * hh, v);
+            uint32_t o[8];
 #pragma unroll
-          for (int jj = 0; jj < 4; ++jj)
-            *reinterpret_cast<uint4*>(stg + lane * kHStageRow + 16 * jj) =
-                make_uint4(o[4 * jj], o[4 * jj + 1], o[4 * jj + 2], o[4 * jj + 3]);
+            for (int jj = 0; jj < 8; ++jj) o[jj] = gelu2_bf16x2(v[2 * jj], v[2 * jj + 1]);
+#pragma unroll
+            for (int jj = 0; jj < 2; ++jj)
+              *reinterpret_cast<uint4*>(stg + lane * kHStageRow + 32 * hh + 16 * jj) =
+                  make_uint4(o[4 * jj], o[4 * jj + 1], o[4 * jj + 2], o[4 * jj + 3]);
+          }
           __syncwarp();
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
@@ -507,8 +528,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         // 32 columns in shared memory and adds them back row-contiguously (8 lanes
         // x 16 B per row, 4 rows per instruction).
         float* stg = staging + (size_t)(warp - kFirstEpiWarp) * 32 * kStageRow;
-        const int t = p.row_tok[row];
-        const float wt = p.row_w[row];
+        const int t = t_cur;
+        const float wt = w_cur;
         const int r_sub = lane >> 3, c_sub = (lane & 7) * 4;
         for (int c = 0; c < cols; c += 32) {
           float v[32];
@@ -539,7 +560,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
   }
@@ -567,7 +588,7 @@ __global__ void timeout_probe_kernel(int* status, long long limit) {
 // logits, takes the decisions of Eqs. 18-27 and the warp counts its chunk's
 // (expert, block) pairs.
 constexpr int kRtThreads = 192;   // warp 0 TMA, warp 1 TMEM + MMA, warps 2-5 decisions
-constexpr int kRtStages = 4;
+constexpr int kRtStages = 6;
 constexpr uint32_t kRtStageB = 160u * kBK * 2;  // up to 160 router columns
 constexpr size_t kRtSmem = 1024 + kRtStages * (kStageA + kRtStageB) + 256;
 
@@ -616,13 +637,6 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  // the output accumulator rows of these tokens start at zero
-  {
-    const int rows = min(kBM, p.dec.T - t0);
-    float4* yz = reinterpret_cast<float4*>(p.y32 + (size_t)t0 * p.d);
-    const int n4 = rows * p.d / 4;
-    for (int i = threadIdx.x; i < n4; i += kRtThreads) yz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-  }
   const int num_kb = p.d / kBK;
   if (warp == 0) {
     if (lane == 0) {
@@ -662,7 +676,15 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     }
     __syncwarp();
   } else {
-    // decision warps: lane quarter q = warp % 4 holds tokens t0 + 32 q + lane
+    // decision warps: lane quarter q = warp % 4 holds tokens t0 + 32 q + lane.
+    // While the MMAs run they zero the output accumulator rows of these tokens.
+    {
+      const int rows = min(kBM, p.dec.T - t0);
+      float4* yz = reinterpret_cast<float4*>(p.y32 + (size_t)t0 * p.d);
+      const int n4 = rows * p.d / 4;
+      for (int i = threadIdx.x - 64; i < n4; i += kRtThreads - 64)
+        yz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     const int q = warp & 3;
     const int row = q * 32 + lane;
     bool w = true;
@@ -671,7 +693,8 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
       tc_fence_after();
       // logits and affinities overlay the (now idle) operand ring
       float* zs = reinterpret_cast<float*>(smem);
-      float* ss = zs + kBM * (Cp + 1);
+      float* ss = zs + kBM * (Cp + 1);                                      // [128][2K + 1]
+      uint32_t* cscr = reinterpret_cast<uint32_t*>(ss + kBM * (2 * K + 1));  // [4][128]
       float* z = zs + row * (Cp + 1);
       for (int c = 0; c < Cp; c += 32) {
         float v[32];
@@ -682,9 +705,9 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
       const int t = t0 + row;
       const bool valid = t < p.dec.T && (p.dec.mask == nullptr || p.dec.mask[t] != 0);
       uint64_t shr, em;
-      decide_token(p.dec, t, valid, z, ss + row * (K + 1), shr, em);
+      decide_token(p.dec, t, valid, z, ss + row * (2 * K + 1), shr, em);
       const int chunk = blockIdx.x * (kBM / 32) + q;
-      if (chunk < p.dec.n_chunks) count_chunk_pairs(p.dec, chunk, lane, shr, em);
+      if (chunk < p.dec.n_chunks) count_chunk_pairs(p.dec, chunk, lane, shr, em, cscr + q * 128);
     }
   }
   tc_fence_before();

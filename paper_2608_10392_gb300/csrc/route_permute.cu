@@ -114,7 +114,8 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
   float* xs = sm;                               // [kKc][64]
   float* ws = xs + kKc * kRouterTokens;         // [kKc][Cp]
   float* zs = ws + kKc * Cp;                    // [64][Cp + 1] logits
-  float* ss = zs + kRouterTokens * (Cp + 1);    // [64][K + 1] affinities
+  float* ss = zs + kRouterTokens * (Cp + 1);    // [64][2K + 1] decision scratch
+  uint32_t* cscr = reinterpret_cast<uint32_t*>(ss + kRouterTokens * (2 * K + 1));  // [2][128]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int t0 = blockIdx.x * kRouterTokens;
 
@@ -179,11 +180,11 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
   const int t = t0 + tid;
   const bool valid = t < a.dec.T && (a.dec.mask == nullptr || a.dec.mask[t] != 0);
   uint64_t shr, em;
-  decide_token(a.dec, t, valid, zs + tid * (Cp + 1), ss + tid * (K + 1), shr, em);
+  decide_token(a.dec, t, valid, zs + tid * (Cp + 1), ss + tid * (2 * K + 1), shr, em);
 
   // ---- (expert, block) pairs per group for this warp's 32 tokens ----
   const int chunk = blockIdx.x * (kRouterTokens / kWarpChunk) + warp;
-  if (chunk < a.dec.n_chunks) count_chunk_pairs(a.dec, chunk, lane, shr, em);
+  if (chunk < a.dec.n_chunks) count_chunk_pairs(a.dec, chunk, lane, shr, em, cscr + warp * 128);
 }
 
 // get_routing helper: experts by decreasing affinity (ties to the lower
@@ -541,7 +542,8 @@ cudaError_t launch_prototypes(unif_moe_layer* L, const void* w_router, const flo
 static size_t router_smem(const unif_moe_layer* L) {
   const int Cp = L->router_cols_pad;
   return sizeof(float) * ((size_t)kKc * kRouterTokens + (size_t)kKc * Cp +
-                          (size_t)kRouterTokens * (Cp + 1) + (size_t)kRouterTokens * (L->K + 1));
+                          (size_t)kRouterTokens * (Cp + 1) +
+                          (size_t)kRouterTokens * (2 * L->K + 1) + 2 * 128);
 }
 
 int forward_chunks(int T) { return (T + kWarpChunk - 1) / kWarpChunk; }
