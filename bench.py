@@ -55,6 +55,41 @@ def workload_desc(s, T_valid):
                           "beta fixed %.2f" % s.beta_fixed}
 
 
+# ----------------------------------------------------------------- ranks
+
+def rank_token_seed(s, rank):
+    """Token seed of a rank: rank 0 draws the workload's own batch; every other
+    rank an independent batch of the same shape (weak scaling: each rank owns
+    its tokens, the layer weights are the same everywhere)."""
+    return None if rank == 0 else s.index * 1000 + 1 + 7919 * rank
+
+
+def max_over_ranks(value, dist=None, device="cpu"):
+    """The largest value over all ranks (the slowest rank sets the job time)."""
+    if dist is None:
+        return float(value)
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value, dist=None, device="cpu"):
+    """The sum of a per-rank count over all ranks."""
+    if dist is None:
+        return float(value)
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def job_throughput(total_tokens, ms_per_step):
+    """Whole-job tokens/s: the valid tokens all ranks processed in one step
+    over the slowest rank's step time."""
+    return total_tokens / (ms_per_step / 1e3)
+
+
 # ----------------------------------------------------------------- clocks
 
 class ClockSampler:
@@ -180,7 +215,7 @@ def main():
 
     # every rank draws its own batch of tokens (same layer weights)
     w_router, w_up, w_down, bias = workloads.make_weights(s)
-    x, mask = workloads.make_tokens(s, w_router, seed=None if rank == 0 else s.index * 1000 + 1 + 7919 * rank)
+    x, mask = workloads.make_tokens(s, w_router, seed=rank_token_seed(s, rank))
     T = s.tokens
     T_valid = T if mask is None else int(mask.sum())
     layer = Layer(s.d_model, s.d_ff, s.n_experts, s.n_blocks, dtype=s.dtype, max_tokens=T,
@@ -248,10 +283,8 @@ def main():
     names = ["router", "permute", "up_gemm", "down_gemm", "combine"]
     stage_ms = {n: statistics.fmean(stage_ev[i][j].elapsed_time(stage_ev[i][j + 1]) for i in range(K))
                 for j, n in enumerate(names)}
-    if dist:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dist, dev)
+    total_valid = sum_over_ranks(T_valid, dist, dev)
 
     # e2e through the C ABI with host buffers (copies inside the timed region)
     xh = x.pin_memory()
@@ -280,7 +313,7 @@ def main():
 
     peaks, peak_kind = load_peaks()
     ms = total_ms / K
-    value = world * T_valid / (ms / 1e3)
+    value = job_throughput(total_valid, ms)
     tflops = act_flops / (ms / 1e3) / 1e12
     peak_tf = peaks["bf16_tflops_sustained"]
     hbm = peaks["hbm_gbs"]

@@ -34,12 +34,11 @@
 
 #include "decide.cuh"
 #include "internal.cuh"
+#include "tc_common.cuh"
 
 namespace unif {
 namespace tc {
 
-constexpr int kBM = 128;
-constexpr int kBK = 64;
 constexpr int kThreads = 416;     // 13 warps
 constexpr int kProducerWarps = 4;  // warps 0-3
 constexpr int kMmaWarp = 4;        // TMEM allocation and MMA issue
@@ -48,7 +47,6 @@ constexpr int kFirstEpiWarp = 5;   // warps 5-12 (warp % 4 covers every TMEM lan
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccStride = 256;  // TMEM columns per accumulator buffer
 constexpr int kMaxBN = 256;
-constexpr uint32_t kStageA = kBM * kBK * 2;      // 16 KB
 constexpr uint32_t kStageB = kMaxBN * kBK * 2;   // 32 KB
 constexpr int kStageRow = 36;                    // fp32 per staged row (32 + 4 pad, 16 B aligned)
 constexpr uint32_t kHStageRow = 80;              // bytes per staged h row (64 + 16 pad)
@@ -82,222 +80,6 @@ struct Params {
   int* status;
   long long wait_limit;  // clock cycles before a wait gives up
 };
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-// ---- mbarrier ----
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx_only(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.expect_tx.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0u;
-}
-
-// Bounded wait: gives up after `limit` cycles (or once another role of the
-// CTA has given up), recording the timeout in the status word.
-__device__ __noinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          int* status, long long limit) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  for (;;) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (*abort_flag) return false;
-    if (clock64() - t0 > limit) {
-      *abort_flag = 1;
-      atomicOr(status, kStatusTimeout);
-      return false;
-    }
-  }
-}
-
-// ---- TMA ----
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
-                                            int c0, int c1) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
-      : "memory");
-}
-// ---- cp.async (row gather into the swizzled operand layout) ----
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void fence_proxy_async() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-// ---- tcgen05 ----
-__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
-               "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void tmem_relinquish() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                          uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-__device__ __forceinline__ void umma_commit(uint32_t bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-      : "memory");
-}
-// 32 lanes x 16 consecutive 32-bit TMEM columns; thread i holds lane base+i.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
-  uint32_t r[16];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32"
-      " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// 32 lanes x 32 consecutive 32-bit TMEM columns; thread i holds lane base+i.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32"
-      " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15,"
-      " %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// ---- GeLU on pairs with packed fp32x2 arithmetic ----
-// GeLU(x) = x Phi(x) = max(x, 0) - |x| Q(|x|), Q(a) = Phi(-a) = exp(-a^2/2) R(a),
-// R(a) = erfcx(a / sqrt 2) / 2 (the exact erf form, rewritten through the
-// normal tail). R is a degree-12 polynomial in s = 0.4 min(a, 5) - 1, a
-// least-squares Chebyshev fit on [0, 5] (coefficients from gelu_coeffs.py):
-// GeLU relative error < 5e-6 for |x| <= 5, absolute error < 5e-7 everywhere,
-// far below the bf16 rounding h receives next.
-__device__ __forceinline__ uint64_t pk2(float lo, float hi) {
-  uint64_t r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
-  return r;
-}
-__device__ __forceinline__ void upk2(uint64_t v, float& lo, float& hi) {
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-}
-__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
-  uint64_t d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
-__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ float ex2_approx(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-#define UNIF_K2(bits) ((uint64_t)(bits##u) << 32 | (uint64_t)(bits##u))
-__device__ __forceinline__ uint32_t gelu2_bf16x2(float x0, float x1) {
-  const float a0 = fabsf(x0), a1 = fabsf(x1);
-  const uint64_t s = fma2(pk2(fminf(a0, 5.f), fminf(a1, 5.f)), UNIF_K2(0x3ecccccd),  // 0.4
-                          UNIF_K2(0xbf800000));                                      // -1
-  uint64_t r = UNIF_K2(0x3a5572c6);
-  r = fma2(r, s, UNIF_K2(0xbad23ee0));
-  r = fma2(r, s, UNIF_K2(0x3a403f1b));
-  r = fma2(r, s, UNIF_K2(0xbac3e363));
-  r = fma2(r, s, UNIF_K2(0x3bb29d94));
-  r = fma2(r, s, UNIF_K2(0xbc1d2cf5));
-  r = fma2(r, s, UNIF_K2(0x3c76a00d));
-  r = fma2(r, s, UNIF_K2(0xbccc3410));
-  r = fma2(r, s, UNIF_K2(0x3d22ed53));
-  r = fma2(r, s, UNIF_K2(0xbd754c1d));
-  r = fma2(r, s, UNIF_K2(0x3daeb1a7));
-  r = fma2(r, s, UNIF_K2(0xbde98aa9));
-  r = fma2(r, s, UNIF_K2(0x3e10b92a));
-  const uint64_t aa = pk2(a0, a1);
-  // exp(-a^2/2) = 2^(-a^2 log2(e) / 2)
-  const uint64_t t = mul2(mul2(aa, aa), UNIF_K2(0xbf38aa3b));  // -0.7213475
-  float t0, t1;
-  upk2(t, t0, t1);
-  const uint64_t q = mul2(mul2(pk2(ex2_approx(t0), ex2_approx(t1)), r), aa);
-  float q0, q1;
-  upk2(q, q0, q1);
-  const float g0 = fmaxf(x0, 0.f) - q0, g1 = fmaxf(x1, 0.f) - q1;
-  __nv_bfloat162 h = __floats2bfloat162_rn(g0, g1);
-  return *reinterpret_cast<uint32_t*>(&h);
-}
-#undef UNIF_K2
-
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
-// 1024 bytes apart (stride-dimension offset), leading offset unused (1),
-// descriptor version 1 at bit 46, swizzle mode 2 (128 B) at bits 61-63.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) |
-         ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-
-// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1),
-// A and B bf16 (bits 7-9 = 1, 10-12 = 1), both K-major, N>>3 at bits 17-22,
-// M>>4 at bits 24-28.
-__device__ __forceinline__ uint32_t idesc_bf16(int m, int n) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
-         ((uint32_t)(m >> 4) << 24);
-}
-
 
 // MODE 0 = up-projection (+GeLU), MODE 1 = down-projection (+weighted add).
 template <int MODE>
@@ -381,9 +163,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         const int sq = seq + kb;
         const int stage = sq % kProducerWarps;  // == warp
         const uint32_t phase = (uint32_t)(sq / kProducerWarps) & 1u;
-        bool w = true;
-        if (lane == 0) w = wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
-        ok = __shfl_sync(0xffffffffu, w, 0);
+        ok = wait_warp(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
         if (!ok) break;
         if (lane == 0) {
           mbar_expect_tx_only(full_bar(stage), stage_bytes);
@@ -416,9 +196,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       const int e = g / p.B, blk = g % p.B;
       const int brow = e * p.d + ns * p.bn;  // w_down viewed [(K+1)d][H]
       for (int kb = 0; kb < p.num_kb; ++kb) {
-        bool w = true;
-        if (lane == 0) w = wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
-        ok = __shfl_sync(0xffffffffu, w, 0);
+        ok = wait_warp(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
         if (!ok) break;
         if (lane == 0) {
           mbar_expect_tx(full_bar(stage), stage_bytes);
@@ -487,9 +265,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         t_nxt = p.row_tok[r];
         w_nxt = p.row_w[r];
       }
-      bool w = true;
-      if (lane == 0) w = wait_bounded(accf_bar(acc), acc_phase, abort_flag, p.status, p.wait_limit);
-      if (!__shfl_sync(0xffffffffu, w, 0)) break;
+      if (!wait_warp(accf_bar(acc), acc_phase, abort_flag, p.status, p.wait_limit)) break;
       tc_fence_after();
       const int row = row0 + q * 32 + lane;
       const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)acc * kAccStride;
@@ -687,9 +463,7 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     }
     const int q = warp & 3;
     const int row = q * 32 + lane;
-    bool w = true;
-    if (lane == 0) w = wait_bounded(accf, 0u, abort_flag, p.status, p.wait_limit);
-    if (__shfl_sync(0xffffffffu, w, 0)) {
+    if (wait_warp(accf, 0u, abort_flag, p.status, p.wait_limit)) {
       tc_fence_after();
       // logits and affinities overlay the (now idle) operand ring
       float* zs = reinterpret_cast<float*>(smem);
@@ -741,17 +515,31 @@ EncodeTiledFn encode_fn() {
 // 2-D bf16 tensor map [rows][cols] (cols contiguous), 128-byte swizzle.
 bool encode_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
                uint32_t box_cols, uint32_t box_rows) {
-  EncodeTiledFn fn = encode_fn();
+  return encode_bf16_map(map, base, cols, rows, box_cols, box_rows, 128);
+}
+
+}  // namespace tc
+
+// 2-D bf16 tensor map [rows][cols] (cols contiguous) with a 32-, 64- or
+// 128-byte swizzle.
+bool encode_bf16_map(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
+                     uint32_t box_cols, uint32_t box_rows, int swizzle_bytes) {
+  tc::EncodeTiledFn fn = tc::encode_fn();
   if (!fn) return false;
+  const CUtensorMapSwizzle sw = swizzle_bytes == 32   ? CU_TENSOR_MAP_SWIZZLE_32B
+                                : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                      : CU_TENSOR_MAP_SWIZZLE_128B;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * 2};
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
-                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
+
+namespace tc {
 
 // N split into n_sub sub-tiles of bn columns: bn <= 256 and bn % 64 == 0, so
 // that each of the two epilogue column halves is a whole number of 32-column
@@ -772,6 +560,8 @@ bool pick_split(int n, int* bn, int* nsub) {
 long long g_wait_limit = 4000000000ll;  // ~2 s of SM clock
 
 }  // namespace tc
+
+long long gemm_wait_limit() { return tc::g_wait_limit; }
 
 int gemm_tc_setup(unif_moe_layer* L) {
   if (!tc::pick_split(L->M, &L->up_bn, &L->up_nsub) ||
@@ -796,7 +586,7 @@ int gemm_tc_setup(unif_moe_layer* L) {
     set_error("cudaFuncSetAttribute: %s", cudaGetErrorString(e));
     return UNIF_MOE_ERR_CUDA;
   }
-  return UNIF_MOE_OK;
+  return gemm_ws_setup(L);
 }
 
 cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
@@ -813,12 +603,18 @@ cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t
   p.wait_limit = tc::g_wait_limit;
   // up: N = M (block width), reduction over d
   p.n_sub = L->up_nsub; p.bn = L->up_bn; p.num_kb = L->d / tc::kBK;
-  tc::grouped_gemm_kernel<0><<<L->n_sm, tc::kThreads, tc::Cfg<0>::kSmem, s>>>(L->tm_h, L->tm_wup,
-                                                                             p);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e;
+  if (L->up_ws) {
+    e = launch_up_ws(L, x, s);
+  } else {
+    tc::grouped_gemm_kernel<0><<<L->n_sm, tc::kThreads, tc::Cfg<0>::kSmem, s>>>(L->tm_h,
+                                                                               L->tm_wup, p);
+    e = cudaGetLastError();
+  }
   if (e != cudaSuccess) return e;
   if (mid) cudaEventRecord(mid, s);
   // down: N = d, reduction over the block's M channels
+  if (L->down_ws) return launch_down_ws(L, s);
   p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
   tc::grouped_gemm_kernel<1><<<L->n_sm, tc::kThreads, tc::Cfg<1>::kSmem, s>>>(L->tm_h, L->tm_wdown,
                                                                              p);

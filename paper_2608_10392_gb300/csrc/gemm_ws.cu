@@ -1,0 +1,468 @@
+// Weight-stationary grouped expert GEMMs (tcgen05 + TMEM) for bf16 layers
+// whose per-group weight slice fits in shared memory.
+//
+// The permute step sorts the tile list by group g = (expert e, block b), so
+// consecutive tiles mostly share one weight slice: K_e[:, H_b] (M x d) for the
+// up projection, V_e[H_b, :] (d x M) for the down projection (Eqs. 16, 28-29).
+// Each CTA takes an equal contiguous run of tiles and keeps the current
+// group's slice resident in shared memory, reloading it only when the group
+// changes, slab by slab as the last MMAs of the previous group release each
+// slab. Only the token rows stream: x rows (gathered) for the up projection,
+// h tiles for the down projection, whose A tile then feeds both halves of the
+// d output columns.
+//
+// Roles (one CTA per SM):
+//   up    warps 0-4 own the stages of a 5-deep A ring (16-byte cp.async
+//         gather of 128 token rows per stage), warp 5 loads the weight slabs
+//         (TMA, once per group run), warp 6 allocates TMEM and issues the
+//         MMAs, warps 7-14 run the epilogue (GeLU -> bf16 h);
+//   down  warp 0 brings h tiles (3-deep ring, TMA), warp 4 loads the weight
+//         slabs, warp 5 issues the MMAs, warps 6-13 run the epilogue (weight
+//         scale -> fp32 atomic add into y).
+// Epilogue warp w reads TMEM lane quarter w % 4 and one half of the columns.
+// Every wait is bounded; a wait that runs out records kStatusTimeout in the
+// status word and the CTA unwinds.
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include "internal.cuh"
+#include "tc_common.cuh"
+
+namespace unif {
+namespace tc {
+namespace ws {
+
+constexpr int kEpiWarps = 8;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kAccStride = 256;
+constexpr int kMaxSlabs = 16;
+constexpr uint32_t kBarBytes = 384;
+constexpr uint32_t kMaxSmem = 232448;  // 227 KB opt-in per CTA
+
+// Per-projection layout: warps 0-3 bring A (up: the owners of a 4-deep ring
+// of gathered x stages; down: warp 0 alone, 3-deep ring of h tiles by TMA),
+// warp 4 loads the weight slabs, warp 5 issues the MMAs, warps 6-13 run the
+// epilogue. Each epilogue warp owns a 32-row x 32-column staging tile:
+// bf16 (64-byte rows, 64-byte swizzle) that a TMA store writes to h, or fp32
+// (128-byte rows, 128-byte swizzle) that the warp adds into y.
+template <int MODE>
+struct Cfg {
+  static constexpr int kStagesA = MODE == 0 ? 4 : 3;
+  static constexpr int kProducerWarps = MODE == 0 ? 4 : 1;
+  static constexpr int kLoaderWarp = 4;
+  static constexpr int kMmaWarp = 5;
+  static constexpr int kFirstEpiWarp = 6;
+  static constexpr int kThreads = 32 * (kFirstEpiWarp + kEpiWarps);
+  static constexpr uint32_t kStageRowBytes = MODE == 0 ? 64u : 128u;
+  static constexpr uint32_t kStaging = kEpiWarps * 32u * kStageRowBytes;
+  static constexpr uint32_t kFixed = 1024 + kStagesA * kStageA + kStaging + kBarBytes;
+  static_assert(MODE != 0 || kProducerWarps == kStagesA, "one owner warp per up stage");
+  static_assert(kEpiWarps == 8, "two warps per TMEM lane quarter");
+};
+
+struct Params {
+  const int32_t* n_tiles;
+  const int32_t* tile_group;
+  const int32_t* row_tok;
+  const float* row_w;
+  int n_sub, bn, num_kb;
+  int B, M, H, d;
+  const __nv_bfloat16* x;
+  __nv_bfloat16* h;
+  float* y32;
+  int* status;
+  long long wait_limit;
+};
+
+template <int MODE>
+__global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
+ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  constexpr int kStagesA = Cfg<MODE>::kStagesA;
+  constexpr int kProducerWarps = Cfg<MODE>::kProducerWarps;
+  constexpr int kLoaderWarp = Cfg<MODE>::kLoaderWarp;
+  constexpr int kMmaWarp = Cfg<MODE>::kMmaWarp;
+  constexpr int kFirstEpiWarp = Cfg<MODE>::kFirstEpiWarp;
+  const int n_slabs = p.n_sub * p.num_kb;
+  const uint32_t slab_bytes = (uint32_t)p.bn * kBK * 2;
+  const uint32_t sA = smem_u32(smem);
+  const uint32_t sB = sA + kStagesA * kStageA;
+  uint8_t* tail = smem + kStagesA * kStageA + (size_t)n_slabs * slab_bytes;
+  uint8_t* staging = tail;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(tail + Cfg<MODE>::kStaging);
+  const uint32_t bar0 = smem_u32(bars);
+  auto fullA = [&](int s) { return bar0 + 8u * s; };
+  auto emptyA = [&](int s) { return bar0 + 8u * (5 + s); };
+  auto wfull = [&](int s) { return bar0 + 8u * (10 + s); };
+  auto wempty = [&](int s) { return bar0 + 8u * (10 + kMaxSlabs + s); };
+  auto accf = [&](int a) { return bar0 + 8u * (10 + 2 * kMaxSlabs + a); };
+  auto acce = [&](int a) { return bar0 + 8u * (12 + 2 * kMaxSlabs + a); };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 14 + 2 * kMaxSlabs);
+  static_assert(8 * (14 + 2 * kMaxSlabs) + 8 <= kBarBytes, "barrier region");
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStagesA; ++s) {
+      mbar_init(fullA(s), 1);
+      mbar_init(emptyA(s), 1);
+    }
+    for (int s = 0; s < n_slabs; ++s) {
+      mbar_init(wfull(s), 1);
+      mbar_init(wempty(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(accf(a), 1);
+      mbar_init(acce(a), kEpiWarps);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  // This CTA's contiguous run of tiles (sizes differ by at most one).
+  const int n_tiles = p.n_tiles[0];
+  const int t_begin = (int)(((long long)blockIdx.x * n_tiles) / gridDim.x);
+  const int t_end = (int)(((long long)(blockIdx.x + 1) * n_tiles) / gridDim.x);
+
+  if (MODE == 0 && warp < kProducerWarps) {
+    // ---------------- up: A stage owners (x rows gathered) -----------------
+    // Stage sequence number sq = (tile - t_begin) * num_kb + kb; warp w owns
+    // the stages with sq = w (mod 5). Lane (rsub, j) copies 16-byte chunk j
+    // of rows 4 i + rsub, i = 0..31; the tile's 128 row tokens sit in
+    // registers (lane l holds rows l, l + 32, l + 64, l + 96) and reach the
+    // copying lane by shuffle.
+    const int j = lane & 7, rsub = lane >> 3;
+    bool ok = true;
+    int seq = 0;
+    for (int tile = t_begin; tile < t_end && ok; ++tile, seq += p.num_kb) {
+      const int first = (warp - seq % kProducerWarps + kProducerWarps) % kProducerWarps;
+      if (first >= p.num_kb) continue;
+      int tk[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int t = p.row_tok[tile * kBM + 32 * i + lane];  // padding rows: token 0, unused
+        tk[i] = t < 0 ? 0 : t;
+      }
+      const __nv_bfloat16* xj = p.x + j * 8;
+      for (int kb = first; kb < p.num_kb; kb += kProducerWarps) {
+        const int sq = seq + kb;
+        const int stage = sq % kStagesA;
+        const uint32_t phase = (uint32_t)(sq / kStagesA) & 1u;
+        ok = wait_warp(emptyA(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
+        if (!ok) break;
+        const uint32_t a_dst = sA + stage * kStageA;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int r = 4 * i + rsub;
+          const int t = __shfl_sync(0xffffffffu, tk[i >> 3], r & 31);
+          cp_async16(a_dst + r * 128u + ((j ^ (r & 7)) << 4), xj + (size_t)t * p.d + kb * kBK);
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(fullA(stage));
+      }
+    }
+  } else if (MODE == 1 && warp == 0) {
+    // ---------------- down: h tiles by TMA ---------------------------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int tile = t_begin; tile < t_end && ok; ++tile) {
+        for (int kb = 0; kb < p.num_kb; ++kb) {
+          if (!wait_bounded(emptyA(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(fullA(stage), kStageA);
+          tma_load_2d(sA + stage * kStageA, &tmA, fullA(stage), kb * kBK, tile * kBM);
+          if (++stage == kStagesA) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == kLoaderWarp) {
+    // ---------------- weight slabs, once per group run ---------------------
+    // Slab s = ns * num_kb + kb holds bn rows x 64 reduction elements. Run r
+    // (r >= 1) reuses a slab after the MMAs of run r - 1 released it.
+    if (lane == 0) {
+      int run = 0, g_prev = -1;
+      bool ok = true;
+      for (int tile = t_begin; tile < t_end && ok; ++tile) {
+        const int g = p.tile_group[tile];
+        if (g == g_prev) continue;
+        g_prev = g;
+        const int e = g / p.B, blk = g % p.B;
+        for (int s = 0; s < n_slabs; ++s) {
+          const int ns = s / p.num_kb, kb = s % p.num_kb;
+          if (run > 0 &&
+              !wait_bounded(wempty(s), (uint32_t)(run - 1) & 1u, abort_flag, p.status, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(wfull(s), slab_bytes);
+          if (MODE == 0)  // w_up viewed [(K+1) H][d]
+            tma_load_2d(sB + s * slab_bytes, &tmB, wfull(s), kb * kBK, e * p.H + blk * p.M + ns * p.bn);
+          else            // w_down viewed [(K+1) d][H]
+            tma_load_2d(sB + s * slab_bytes, &tmB, wfull(s), blk * p.M + kb * kBK, e * p.d + ns * p.bn);
+        }
+        ++run;
+      }
+    }
+    __syncwarp();
+  } else if (warp == kMmaWarp) {
+    // ---------------- MMA issuer --------------------------------------------
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(kBM, p.bn);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      int run = -1, g_prev = -1;
+      bool ok = true;
+      for (int tile = t_begin; tile < t_end && ok; ++tile) {
+        const int g = p.tile_group[tile];
+        const bool first_of_run = g != g_prev;
+        if (first_of_run) { ++run; g_prev = g; }
+        // release the slabs after this tile if the next tile of the run
+        // belongs to another group
+        const bool release = tile + 1 < t_end && p.tile_group[tile + 1] != g;
+        const int st0 = stage;
+        const uint32_t ph0 = phase;
+        for (int ns = 0; ns < p.n_sub && ok; ++ns) {
+          if (!wait_bounded(acce(acc), acc_phase ^ 1u, abort_flag, p.status, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + (uint32_t)acc * kAccStride;
+          int st = st0;
+          uint32_t ph = ph0;
+          for (int kb = 0; kb < p.num_kb; ++kb) {
+            const int s = ns * p.num_kb + kb;
+            if (ns == 0 && !wait_bounded(fullA(st), ph, abort_flag, p.status, p.wait_limit)) {
+              ok = false;
+              break;
+            }
+            if (first_of_run &&
+                !wait_bounded(wfull(s), (uint32_t)run & 1u, abort_flag, p.status, p.wait_limit)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t a_base = sA + st * kStageA, b_base = sB + s * slab_bytes;
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k)
+              umma_bf16(d_tmem, sw128_desc(a_base + k * 32), sw128_desc(b_base + k * 32), idesc,
+                        (kb | k) != 0 ? 1u : 0u);
+            if (release) umma_commit(wempty(s));
+            if (MODE == 0) umma_commit(emptyA(st));  // one pass over A: free it now
+            if (++st == kStagesA) { st = 0; ph ^= 1u; }
+          }
+          if (!ok) break;
+          umma_commit(accf(acc));
+          if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+        }
+        if (!ok) break;
+        // advance the A ring past this tile; the down projection frees its
+        // stages only after both column halves read them
+        for (int kb = 0; kb < p.num_kb; ++kb) {
+          if (MODE == 1) umma_commit(emptyA(stage));
+          if (++stage == kStagesA) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp >= kFirstEpiWarp) {
+    // ---------------- epilogue ----------------------------------------------
+    const int q = warp & 3;
+    const int half = (warp - kFirstEpiWarp) >> 2;
+    const int cols = p.bn / 2;
+    const int c_begin = half * cols;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    int t_nxt = 0;
+    float w_nxt = 0.f;
+    if (MODE == 1 && t_begin < t_end) {
+      const int r = t_begin * kBM + q * 32 + lane;
+      t_nxt = p.row_tok[r];
+      w_nxt = p.row_w[r];
+    }
+    uint8_t* stg = staging + (size_t)(warp - kFirstEpiWarp) * 32 * Cfg<MODE>::kStageRowBytes;
+    const uint32_t stg_s = smem_u32(stg);
+    bool ok = true;
+    for (int tile = t_begin; tile < t_end && ok; ++tile) {
+      const int row0 = tile * kBM;
+      const int t_cur = t_nxt;
+      const float w_cur = w_nxt;
+      if (MODE == 1 && tile + 1 < t_end) {
+        const int r = (tile + 1) * kBM + q * 32 + lane;
+        t_nxt = p.row_tok[r];
+        w_nxt = p.row_w[r];
+      }
+      for (int ns = 0; ns < p.n_sub; ++ns) {
+        if (!wait_warp(accf(acc), acc_phase, abort_flag, p.status, p.wait_limit)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)acc * kAccStride;
+        if (MODE == 0) {
+          // h = bf16(GeLU(acc)), 32 columns per pass: each thread writes its
+          // row's 64 bytes into the warp's staging tile (16-byte chunk c of
+          // row r at c ^ ((r >> 1) & 3), the 64-byte swizzle), and lane 0
+          // stores the 32 x 32 tile to h with TMA. The tile is rewritten only
+          // after the previous store has read it.
+          const uint32_t sw = (uint32_t)(lane >> 1) & 3u;
+          for (int c = 0; c < cols; c += 32) {
+            uint32_t o[16];
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+              float v[16];
+              tmem_ld16(t_row + c_begin + c + 16 * hh, v);
+#pragma unroll
+              for (int jj = 0; jj < 8; ++jj) o[8 * hh + jj] = gelu2_bf16x2(v[2 * jj], v[2 * jj + 1]);
+            }
+            if (lane == 0) bulk_wait_read();
+            __syncwarp();
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj)
+              *reinterpret_cast<uint4*>(stg + lane * 64 + ((jj ^ sw) << 4)) =
+                  make_uint4(o[4 * jj], o[4 * jj + 1], o[4 * jj + 2], o[4 * jj + 3]);
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tmA, stg_s, ns * p.bn + c_begin + c, row0 + q * 32);
+              bulk_commit();
+            }
+          }
+        } else {
+          // y[tok] += w * acc, 32 columns per pass: thread = row stages its
+          // 128 scaled bytes (chunk c at c ^ (r & 7)); then 8 lanes per row
+          // add 4 rows x 128 contiguous bytes per instruction.
+          float* stf = reinterpret_cast<float*>(stg);
+          const int r_sub = lane >> 3, c8 = lane & 7;
+          float* ybase = p.y32 + ns * p.bn + c_begin;
+          for (int c = 0; c < cols; c += 32) {
+            float v[32];
+            tmem_ld32(t_row + c_begin + c, v);
+#pragma unroll
+            for (int jj = 0; jj < 8; ++jj)
+              *reinterpret_cast<float4*>(stf + lane * 32 + ((jj ^ (lane & 7)) << 2)) =
+                  make_float4(w_cur * v[4 * jj], w_cur * v[4 * jj + 1], w_cur * v[4 * jj + 2],
+                              w_cur * v[4 * jj + 3]);
+            __syncwarp();
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const int r = 4 * i + r_sub;
+              const int tr = __shfl_sync(0xffffffffu, t_cur, r);
+              const float4 val = *reinterpret_cast<const float4*>(stf + r * 32 + ((c8 ^ (r & 7)) << 2));
+              if (tr >= 0)
+                atomicAdd(reinterpret_cast<float4*>(ybase + (size_t)tr * p.d + c + c8 * 4), val);
+            }
+            __syncwarp();
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acce(acc));
+        if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+      }
+    }
+    if (MODE == 0 && lane == 0) bulk_wait_all();  // h complete before the CTA retires
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+}  // namespace ws
+}  // namespace tc
+
+// Chooses the weight-stationary kernels where their shapes and shared memory
+// allow: the up projection needs the whole block width in one accumulator
+// (M <= 256); the down projection reuses each h tile across all output
+// column sub-tiles, so the tile's M / 64 reduction stages must fit its A ring.
+// UNIF_MOE_GEMM_KERNELS=streaming keeps the streaming kernels.
+int gemm_ws_setup(unif_moe_layer* L) {
+  using namespace tc::ws;
+  L->up_ws = L->down_ws = false;
+  const char* env = getenv("UNIF_MOE_GEMM_KERNELS");
+  if (env && strcmp(env, "streaming") == 0) return UNIF_MOE_OK;
+  const uint64_t up_slabs = (uint64_t)L->up_nsub * (L->d / tc::kBK);
+  const uint64_t up_smem = Cfg<0>::kFixed + up_slabs * (uint64_t)L->up_bn * tc::kBK * 2;
+  if (L->up_nsub == 1 && up_slabs <= (uint64_t)kMaxSlabs && up_smem <= kMaxSmem) {
+    if (cudaFuncSetAttribute(ws_gemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)up_smem) != cudaSuccess) {
+      set_error("cudaFuncSetAttribute failed for the weight-stationary up kernel");
+      return UNIF_MOE_ERR_CUDA;
+    }
+    if (!encode_bf16_map(&L->tm_h_st, L->ws.hbuf, L->M, (uint64_t)L->max_rows, 32, 32, 64)) {
+      set_error("cuTensorMapEncodeTiled failed for the h store map");
+      return UNIF_MOE_ERR_CUDA;
+    }
+    L->up_ws = true;
+    L->up_ws_smem = (uint32_t)up_smem;
+  }
+  const int down_kb = L->M / tc::kBK;
+  const uint64_t down_slabs = (uint64_t)L->down_nsub * down_kb;
+  const uint64_t down_smem = Cfg<1>::kFixed + down_slabs * (uint64_t)L->down_bn * tc::kBK * 2;
+  if (down_kb <= Cfg<1>::kStagesA && down_slabs <= (uint64_t)kMaxSlabs && down_smem <= kMaxSmem) {
+    if (cudaFuncSetAttribute(ws_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)down_smem) != cudaSuccess) {
+      set_error("cudaFuncSetAttribute failed for the weight-stationary down kernel");
+      return UNIF_MOE_ERR_CUDA;
+    }
+    L->down_ws = true;
+    L->down_ws_smem = (uint32_t)down_smem;
+  }
+  return UNIF_MOE_OK;
+}
+
+static tc::ws::Params ws_params(unif_moe_layer* L, const void* x) {
+  tc::ws::Params p;
+  p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group;
+  p.row_tok = L->ws.row_tok; p.row_w = L->ws.row_w;
+  p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;
+  p.x = static_cast<const __nv_bfloat16*>(x);
+  p.h = static_cast<__nv_bfloat16*>(L->ws.hbuf);
+  p.y32 = L->ws.y32;
+  p.status = L->ws.status;
+  p.wait_limit = gemm_wait_limit();
+  return p;
+}
+
+cudaError_t launch_up_ws(unif_moe_layer* L, const void* x, cudaStream_t s) {
+  tc::ws::Params p = ws_params(L, x);
+  p.n_sub = L->up_nsub; p.bn = L->up_bn; p.num_kb = L->d / tc::kBK;
+  tc::ws::ws_gemm_kernel<0><<<L->n_sm, tc::ws::Cfg<0>::kThreads, L->up_ws_smem, s>>>(
+      L->tm_h_st, L->tm_wup, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_down_ws(unif_moe_layer* L, cudaStream_t s) {
+  tc::ws::Params p = ws_params(L, nullptr);
+  p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
+  tc::ws::ws_gemm_kernel<1><<<L->n_sm, tc::ws::Cfg<1>::kThreads, L->down_ws_smem, s>>>(L->tm_h,
+                                                                              L->tm_wdown, p);
+  return cudaGetLastError();
+}
+
+}  // namespace unif

@@ -79,8 +79,13 @@ struct unif_moe_layer {
   CUtensorMap tm_wup;
   CUtensorMap tm_wdown;
   CUtensorMap tm_h;
+  CUtensorMap tm_h_st;  // h as 32 x 32 store boxes (64-byte swizzle), up-projection epilogue
   CUtensorMap tm_wr;
   int up_bn = 0, up_nsub = 0, down_bn = 0, down_nsub = 0;
+  // Weight-stationary kernels (when the group's weight slice fits in shared
+  // memory) and their dynamic shared-memory sizes.
+  bool up_ws = false, down_ws = false;
+  uint32_t up_ws_smem = 0, down_ws_smem = 0;
   // Optional caller-owned timing events recorded at the stage boundaries.
   cudaEvent_t stage_ev[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
 };
@@ -108,6 +113,12 @@ int gemm_tc_setup(unif_moe_layer* L);  // tensor maps of weights and h; returns 
 cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
                             cudaStream_t s);
 cudaError_t launch_timeout_probe(unif_moe_layer* L, int timeout_us, cudaStream_t s);
+int gemm_ws_setup(unif_moe_layer* L);  // picks the weight-stationary kernels where they fit
+cudaError_t launch_up_ws(unif_moe_layer* L, const void* x, cudaStream_t s);
+cudaError_t launch_down_ws(unif_moe_layer* L, cudaStream_t s);
+long long gemm_wait_limit();
+bool encode_bf16_map(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
+                     uint32_t box_cols, uint32_t box_rows, int swizzle_bytes);  // clock cycles before a bounded wait gives up
 int router_tc_setup(unif_moe_layer* L);
 cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
                              int32_t* b_out, int32_t* k_out, cudaStream_t s);

@@ -266,3 +266,25 @@ def test_forward_host_matches_device():
     g.layer.forward_host(xh, out, shared_counts_host=b, residual_counts_host=k)
     np.testing.assert_allclose(out.float().numpy(), g.y, rtol=1e-2, atol=1e-6)  # one bf16 ulp
     assert np.array_equal(b.numpy(), g.b) and np.array_equal(k.numpy(), g.k)
+
+
+# ------------------------------------------- GEMM kernel variants
+
+@pytest.mark.parametrize("kernels", ["weight_stationary", "streaming"])
+def test_gemm_variants_many_group_runs(kernels, monkeypatch):
+    """Enough tiles that every CTA walks several group runs (weight slabs
+    reloaded mid-run), on both GEMM kernel families."""
+    if kernels == "streaming":
+        monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
+    wl = workloads.make_workload(small(tokens=6000, d_model=128, d_ff=512, n_experts=8,
+                                       n_blocks=4))
+    g = run_gpu(wl)
+    assert_parity(wl, g, compare(wl, g, sample=1500))
+
+
+def test_vit_s_streaming_kernels(monkeypatch):
+    """The ViT-S layer through the streaming GEMMs agrees with the oracle too."""
+    monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
+    wl = workloads.make_workload(workloads.spec("vit_s", tokens=4000))
+    g = run_gpu(wl)
+    assert_parity(wl, g, compare(wl, g, sample=800))
