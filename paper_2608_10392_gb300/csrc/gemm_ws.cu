@@ -11,15 +11,15 @@
 // h tiles for the down projection, whose A tile then feeds both halves of the
 // d output columns.
 //
-// Roles (one CTA per SM):
-//   up    warps 0-4 own the stages of a 5-deep A ring (16-byte cp.async
-//         gather of 128 token rows per stage), warp 5 loads the weight slabs
-//         (TMA, once per group run), warp 6 allocates TMEM and issues the
-//         MMAs, warps 7-14 run the epilogue (GeLU -> bf16 h);
-//   down  warp 0 brings h tiles (3-deep ring, TMA), warp 4 loads the weight
-//         slabs, warp 5 issues the MMAs, warps 6-13 run the epilogue (weight
-//         scale -> fp32 atomic add into y).
-// Epilogue warp w reads TMEM lane quarter w % 4 and one half of the columns.
+// Roles (one CTA per SM, 15 warps):
+//   warps 0-3   up: owners of a 4-deep ring of gathered x stages (16-byte
+//               cp.async of 128 token rows per stage); down: warp 0 brings h
+//               tiles (3-deep ring, TMA)
+//   warp 4      weight loader: TMA of the group's slabs, once per group run
+//   warps 5-6   MMA issuers (warp 5 also owns the TMEM allocation)
+//   warps 7-14  epilogue: up, GeLU -> bf16 h staged and stored by TMA; down,
+//               weight scale -> fp32 atomic add into y. Warp w reads TMEM lane
+//               quarter w % 4 and one half of the accumulator's columns.
 // Every wait is bounded; a wait that runs out records kStatusTimeout in the
 // status word and the CTA unwinds.
 #include <stdio.h>
@@ -42,8 +42,8 @@ constexpr uint32_t kMaxSmem = 232448;  // 227 KB opt-in per CTA
 
 // Per-projection layout: warps 0-3 bring A (up: the owners of a 4-deep ring
 // of gathered x stages; down: warp 0 alone, 3-deep ring of h tiles by TMA),
-// warp 4 loads the weight slabs, warp 5 issues the MMAs, warps 6-13 run the
-// epilogue. Each epilogue warp owns a 32-row x 32-column staging tile:
+// warp 4 loads the weight slabs, warps 5-6 issue the MMAs, warps 7-14 run
+// the epilogue. Each epilogue warp owns a 32-row x 32-column staging tile:
 // bf16 (64-byte rows, 64-byte swizzle) that a TMA store writes to h, or fp32
 // (128-byte rows, 128-byte swizzle) that the warp adds into y.
 template <int MODE>
@@ -51,8 +51,9 @@ struct Cfg {
   static constexpr int kStagesA = MODE == 0 ? 4 : 3;
   static constexpr int kProducerWarps = MODE == 0 ? 4 : 1;
   static constexpr int kLoaderWarp = 4;
-  static constexpr int kMmaWarp = 5;
-  static constexpr int kFirstEpiWarp = 6;
+  static constexpr int kMmaWarp = 5;        // warps 5 and 6 issue MMAs
+  static constexpr int kMmaWarps = 2;
+  static constexpr int kFirstEpiWarp = 7;
   static constexpr int kThreads = 32 * (kFirstEpiWarp + kEpiWarps);
   static constexpr uint32_t kStageRowBytes = MODE == 0 ? 64u : 128u;
   static constexpr uint32_t kStaging = kEpiWarps * 32u * kStageRowBytes;
@@ -109,14 +110,14 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStagesA; ++s) {
       mbar_init(fullA(s), 1);
-      mbar_init(emptyA(s), 1);
+      mbar_init(emptyA(s), Cfg<MODE>::kMmaWarps);
     }
     for (int s = 0; s < n_slabs; ++s) {
       mbar_init(wfull(s), 1);
-      mbar_init(wempty(s), 1);
+      mbar_init(wempty(s), Cfg<MODE>::kMmaWarps);
     }
     for (int a = 0; a < 2; ++a) {
-      mbar_init(accf(a), 1);
+      mbar_init(accf(a), Cfg<MODE>::kMmaWarps);
       mbar_init(acce(a), kEpiWarps);
     }
     *abort_flag = 0;
@@ -146,15 +147,18 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int j = lane & 7, rsub = lane >> 3;
     bool ok = true;
     int seq = 0;
+    int tk_nxt[4];  // the next tile's row tokens, loaded one tile ahead
+#pragma unroll
+    for (int i = 0; i < 4; ++i) tk_nxt[i] = t_begin < t_end ? p.row_tok[t_begin * kBM + 32 * i + lane] : 0;
     for (int tile = t_begin; tile < t_end && ok; ++tile, seq += p.num_kb) {
-      const int first = (warp - seq % kProducerWarps + kProducerWarps) % kProducerWarps;
-      if (first >= p.num_kb) continue;
       int tk[4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const int t = p.row_tok[tile * kBM + 32 * i + lane];  // padding rows: token 0, unused
-        tk[i] = t < 0 ? 0 : t;
+        tk[i] = tk_nxt[i] < 0 ? 0 : tk_nxt[i];  // padding rows: token 0, unused
+        if (tile + 1 < t_end) tk_nxt[i] = p.row_tok[(tile + 1) * kBM + 32 * i + lane];
       }
+      const int first = (warp - seq % kProducerWarps + kProducerWarps) % kProducerWarps;
+      if (first >= p.num_kb) continue;
       const __nv_bfloat16* xj = p.x + j * 8;
       for (int kb = first; kb < p.num_kb; kb += kProducerWarps) {
         const int sq = seq + kb;
@@ -224,69 +228,121 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
     __syncwarp();
-  } else if (warp == kMmaWarp) {
-    // ---------------- MMA issuer --------------------------------------------
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(kBM, p.bn);
-      int stage = 0;
-      uint32_t phase = 0;
-      int acc = 0;
-      uint32_t acc_phase = 0;
-      int run = -1, g_prev = -1;
-      bool ok = true;
-      for (int tile = t_begin; tile < t_end && ok; ++tile) {
-        const int g = p.tile_group[tile];
-        const bool first_of_run = g != g_prev;
-        if (first_of_run) { ++run; g_prev = g; }
-        // release the slabs after this tile if the next tile of the run
-        // belongs to another group
-        const bool release = tile + 1 < t_end && p.tile_group[tile + 1] != g;
-        const int st0 = stage;
-        const uint32_t ph0 = phase;
-        for (int ns = 0; ns < p.n_sub && ok; ++ns) {
-          if (!wait_bounded(acce(acc), acc_phase ^ 1u, abort_flag, p.status, p.wait_limit)) {
+  } else if (warp >= kMmaWarp && warp < kMmaWarp + Cfg<MODE>::kMmaWarps) {
+    // ---------------- MMA issuers -------------------------------------------
+    // Two warps issue MMAs side by side: an MMA issue returns only once the
+    // tensor pipe takes it, so one issuer's bookkeeping between MMA groups
+    // would leave the pipe idle; the other issuer's MMAs fill those gaps.
+    // Up (and a single-sub-tile down): warp m computes columns
+    // [m bn/2, (m+1) bn/2) of every accumulator. Down with two sub-tiles:
+    // warp m computes sub-tile m. Both walk every tile, so both wait for the
+    // same stages and weight runs, and each barrier they release counts both.
+    // Within a warp the whole warp runs the loop (warp-uniform values) and an
+    // elected lane issues; the next stage's barrier is tested before the
+    // current stage's MMAs go out and read back after.
+    const int m = warp - kMmaWarp;
+    const bool split_n = !(MODE == 1 && p.n_sub == 2);
+    const int n_mma = split_n ? p.bn / 2 : p.bn;
+    const uint32_t idesc = idesc_bf16(kBM, n_mma);
+    // B rows and accumulator columns this warp covers (split_n), in 16-byte
+    // descriptor units and TMEM columns
+    const uint64_t b_off = split_n ? (uint64_t)(m * n_mma * 128 / 16) : 0ull;
+    const uint32_t d_off = split_n ? (uint32_t)(m * n_mma) : 0u;
+    const uint64_t a_desc0 = sw128_desc(sA), b_desc0 = sw128_desc(sB) + b_off;
+    int stage = 0;
+    uint32_t phase = 0;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    int run = -1, g_prev = -1;
+    bool ok = true;
+    bool ready = false;  // fullA(stage) known complete
+    // groups of this tile and the next, loaded ahead of use
+    int g_cur = t_begin < t_end ? p.tile_group[t_begin] : -1;
+    int g_nxt = t_begin + 1 < t_end ? p.tile_group[t_begin + 1] : -1;
+    for (int tile = t_begin; tile < t_end && ok; ++tile) {
+      const int g = g_cur, gn = g_nxt;
+      g_cur = g_nxt;
+      if (tile + 2 < t_end) g_nxt = p.tile_group[tile + 2];
+      const bool first_of_run = g != g_prev;
+      if (first_of_run) { ++run; g_prev = g; }
+      // release the slabs after this tile if the next tile of the run
+      // belongs to another group
+      const bool release = tile + 1 < t_end && gn != g;
+      const int st0 = stage;
+      const uint32_t ph0 = phase;
+      for (int ns = 0; ns < p.n_sub && ok; ++ns) {
+        const bool mine = split_n || ns == m;
+        if (mine) {
+          if (!wait_warp(acce(acc), acc_phase ^ 1u, abort_flag, p.status, p.wait_limit)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + (uint32_t)acc * kAccStride;
+          const uint32_t d_tmem = tmem_base + (uint32_t)acc * kAccStride + d_off;
           int st = st0;
           uint32_t ph = ph0;
+          // stages are waited for in the first sub-tile this warp computes
+          const bool first_pass = split_n ? ns == 0 : true;
           for (int kb = 0; kb < p.num_kb; ++kb) {
             const int s = ns * p.num_kb + kb;
-            if (ns == 0 && !wait_bounded(fullA(st), ph, abort_flag, p.status, p.wait_limit)) {
+            const int st_n = st + 1 == kStagesA ? 0 : st + 1;
+            const uint32_t ph_n = st + 1 == kStagesA ? ph ^ 1u : ph;
+            if (first_pass && !ready &&
+                !wait_warp(fullA(st), ph, abort_flag, p.status, p.wait_limit)) {
               ok = false;
               break;
             }
             if (first_of_run &&
-                !wait_bounded(wfull(s), (uint32_t)run & 1u, abort_flag, p.status, p.wait_limit)) {
+                !wait_warp(wfull(s), (uint32_t)run & 1u, abort_flag, p.status, p.wait_limit)) {
               ok = false;
               break;
             }
+            // the stage after this one, in ring order (the next tile's first
+            // stage after the last k-block); read back after the MMAs
+            const uint32_t next_done =
+                first_pass && (MODE == 0 || kb + 1 < p.num_kb) ? mbar_test(fullA(st_n), ph_n) : 0u;
             tc_fence_after();
-            const uint32_t a_base = sA + st * kStageA, b_base = sB + s * slab_bytes;
+            // descriptor start addresses advance in 16-byte units: +2 per 32 bytes
+            const uint64_t a_desc = a_desc0 + (uint64_t)(st * (kStageA >> 4));
+            const uint64_t b_desc = b_desc0 + (uint64_t)(s * (slab_bytes >> 4));
+            if (elect_one()) {
 #pragma unroll
-            for (int k = 0; k < kBK / 16; ++k)
-              umma_bf16(d_tmem, sw128_desc(a_base + k * 32), sw128_desc(b_base + k * 32), idesc,
-                        (kb | k) != 0 ? 1u : 0u);
-            if (release) umma_commit(wempty(s));
-            if (MODE == 0) umma_commit(emptyA(st));  // one pass over A: free it now
-            if (++st == kStagesA) { st = 0; ph ^= 1u; }
+              for (int k = 0; k < kBK / 16; ++k)
+                umma_bf16(d_tmem, a_desc + 2 * k, b_desc + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
+              if (release) umma_commit(wempty(s));
+              if (MODE == 0) umma_commit(emptyA(st));  // one pass over A: free it now
+            }
+            ready = __all_sync(0xffffffffu, next_done != 0u);
+            st = st_n;
+            ph = ph_n;
           }
           if (!ok) break;
-          umma_commit(accf(acc));
-          if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+          if (elect_one()) umma_commit(accf(acc));
+          __syncwarp();
+        } else {
+          // the other warp's sub-tile: this warp still owes its arrival on the
+          // accumulator and, at a group change, on the sub-tile's slabs
+          if (elect_one()) {
+            mbar_arrive(accf(acc));
+            if (release)
+              for (int kb = 0; kb < p.num_kb; ++kb) umma_commit(wempty(ns * p.num_kb + kb));
+          }
+          __syncwarp();
         }
-        if (!ok) break;
-        // advance the A ring past this tile; the down projection frees its
-        // stages only after both column halves read them
-        for (int kb = 0; kb < p.num_kb; ++kb) {
-          if (MODE == 1) umma_commit(emptyA(stage));
-          if (++stage == kStagesA) { stage = 0; phase ^= 1u; }
-        }
+        if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
       }
+      if (!ok) break;
+      // advance the A ring past this tile; the down projection frees its
+      // stages only after both sub-tiles read them
+      for (int kb = 0; kb < p.num_kb; ++kb) {
+        if (MODE == 1) {
+          if (elect_one()) umma_commit(emptyA(stage));
+          __syncwarp();
+        }
+        if (++stage == kStagesA) { stage = 0; phase ^= 1u; }
+      }
+      if (MODE == 1) ready = false;
     }
-    __syncwarp();
   } else if (warp >= kFirstEpiWarp) {
     // ---------------- epilogue ----------------------------------------------
     const int q = warp & 3;

@@ -42,9 +42,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0u;
 }
 
+// Non-blocking test of a phase (a plain shared-memory read of the barrier).
+__device__ __forceinline__ uint32_t mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok;
+}
+
 // Bounded wait: gives up after `limit` cycles (or once another role of the
 // CTA has given up), recording the timeout in the status word.
-static __device__ __noinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+static __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                           int* status, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
@@ -67,6 +80,16 @@ static __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity,
                                                  long long limit) {
   const bool ok = wait_bounded(bar, parity, abort_flag, status, limit);
   return __all_sync(0xffffffffu, ok);
+}
+
+// One lane of a converged warp (elect.sync); the warp's uniform values stay
+// on the uniform datapath for the tcgen05 and TMA instructions it guards.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred = 0;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\telect.sync _|p, 0xffffffff;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(pred));
+  return pred != 0u;
 }
 
 // ---- TMA ----
@@ -180,12 +203,11 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 }
 
 // ---- GeLU on pairs with packed fp32x2 arithmetic ----
-// GeLU(x) = x Phi(x) = max(x, 0) - |x| Q(|x|), Q(a) = Phi(-a) = exp(-a^2/2) R(a),
-// R(a) = erfcx(a / sqrt 2) / 2 (the exact erf form, rewritten through the
-// normal tail). R is a degree-12 polynomial in s = 0.4 min(a, 5) - 1, a
-// least-squares Chebyshev fit on [0, 5] (coefficients from gelu_coeffs.py):
-// GeLU relative error < 5e-6 for |x| <= 5, absolute error < 5e-7 everywhere,
-// far below the bf16 rounding h receives next.
+// GeLU(x) = x Phi(x), Phi(x) = (1 + tanh(g(x))) / 2 with g(x) = atanh(2 Phi(x) - 1)
+// approximated by x P(x^2), P of degree 4 (coefficients and their fit in
+// gelu_coeffs.py; |Phi error| < 2e-6 before the hardware tanh, whose own
+// error, about 2^-11, dominates). g increases monotonically, so large |x|
+// saturates cleanly to x or 0. Evaluated as h = x/2 + (x/2) tanh(g).
 __device__ __forceinline__ uint64_t pk2(float lo, float hi) {
   uint64_t r;
   asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
@@ -204,39 +226,26 @@ __device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
   asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
-__device__ __forceinline__ float ex2_approx(float x) {
+__device__ __forceinline__ float tanh_approx(float x) {
   float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
 #define UNIF_K2(bits) ((uint64_t)(bits##u) << 32 | (uint64_t)(bits##u))
 __device__ __forceinline__ uint32_t gelu2_bf16x2(float x0, float x1) {
-  const float a0 = fabsf(x0), a1 = fabsf(x1);
-  const uint64_t s = fma2(pk2(fminf(a0, 5.f), fminf(a1, 5.f)), UNIF_K2(0x3ecccccd),  // 0.4
-                          UNIF_K2(0xbf800000));                                      // -1
-  uint64_t r = UNIF_K2(0x3a5572c6);
-  r = fma2(r, s, UNIF_K2(0xbad23ee0));
-  r = fma2(r, s, UNIF_K2(0x3a403f1b));
-  r = fma2(r, s, UNIF_K2(0xbac3e363));
-  r = fma2(r, s, UNIF_K2(0x3bb29d94));
-  r = fma2(r, s, UNIF_K2(0xbc1d2cf5));
-  r = fma2(r, s, UNIF_K2(0x3c76a00d));
-  r = fma2(r, s, UNIF_K2(0xbccc3410));
-  r = fma2(r, s, UNIF_K2(0x3d22ed53));
-  r = fma2(r, s, UNIF_K2(0xbd754c1d));
-  r = fma2(r, s, UNIF_K2(0x3daeb1a7));
-  r = fma2(r, s, UNIF_K2(0xbde98aa9));
-  r = fma2(r, s, UNIF_K2(0x3e10b92a));
-  const uint64_t aa = pk2(a0, a1);
-  // exp(-a^2/2) = 2^(-a^2 log2(e) / 2)
-  const uint64_t t = mul2(mul2(aa, aa), UNIF_K2(0xbf38aa3b));  // -0.7213475
-  float t0, t1;
-  upk2(t, t0, t1);
-  const uint64_t q = mul2(mul2(pk2(ex2_approx(t0), ex2_approx(t1)), r), aa);
-  float q0, q1;
-  upk2(q, q0, q1);
-  const float g0 = fmaxf(x0, 0.f) - q0, g1 = fmaxf(x1, 0.f) - q1;
-  __nv_bfloat162 h = __floats2bfloat162_rn(g0, g1);
+  const uint64_t x = pk2(x0, x1);
+  const uint64_t u = mul2(x, x);
+  uint64_t r = UNIF_K2(0x35bf442b);         // c4
+  r = fma2(r, u, UNIF_K2(0xb819e7be));      // c3
+  r = fma2(r, u, UNIF_K2(0xb8b82f22));      // c2
+  r = fma2(r, u, UNIF_K2(0x3d151014));      // c1
+  r = fma2(r, u, UNIF_K2(0x3f4c4130));      // c0
+  float g0, g1;
+  upk2(mul2(x, r), g0, g1);
+  const uint64_t hx = mul2(x, UNIF_K2(0x3f000000));  // x / 2
+  float y0, y1;
+  upk2(fma2(hx, pk2(tanh_approx(g0), tanh_approx(g1)), hx), y0, y1);
+  __nv_bfloat162 h = __floats2bfloat162_rn(y0, y1);
   return *reinterpret_cast<uint32_t*>(&h);
 }
 #undef UNIF_K2
