@@ -33,7 +33,8 @@ if ROOT not in sys.path:
 METRIC = "UniF-MoE layer fwd tokens/s & activated TFLOP/s (% of GB300 bf16 peak), 1 GPU"
 UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KERNELS_PER_FORWARD = 7  # router, count, scan, scatter, up GEMM, down GEMM, combine
+# router (+ decisions, pair counts), group scan, group scatter, up GEMM, down GEMM, combine
+KERNELS_PER_FORWARD = 6
 
 
 def load_peaks():
@@ -88,6 +89,24 @@ def job_throughput(total_tokens, ms_per_step):
     """Whole-job tokens/s: the valid tokens all ranks processed in one step
     over the slowest rank's step time."""
     return total_tokens / (ms_per_step / 1e3)
+
+
+def measured_traffic(workload, kernel):
+    """DRAM bytes per launch of `kernel` from the committed ncu capture, or
+    None when there is none or the kernel sources changed since it was taken."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    rec = json.load(open(path)).get(workload, {})
+    csrc = os.path.join(ROOT, "paper_2608_10392_gb300", "csrc")
+    h = hashlib.sha1()
+    for f in ("gemm_ws.cu", "tc_common.cuh"):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
+    if rec.get("kernel_source_sha1") != h.hexdigest():
+        return None
+    return rec.get(kernel)
 
 
 # ----------------------------------------------------------------- clocks
@@ -320,11 +339,7 @@ def main():
     # roofline of the dominant kernel (the larger grouped GEMM), timed live
     dom = "up_gemm" if stage_ms["up_gemm"] >= stage_ms["down_gemm"] else "down_gemm"
     ach = gemm_flops / (stage_ms[dom] / 1e3) / 1e12
-    traffic = None
-    tr_path = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tr_path):
-        tr = json.load(open(tr_path)).get(s.name, {})
-        traffic = tr.get(dom)
+    traffic = measured_traffic(s.name, dom)
     router_bytes = T * d * elt + T * (4 * 3 + 8 * 2 + 12 * s.n_experts)
     combine_bytes = T * d * (4 + elt)
     permute_bytes = sum_cb * 8
