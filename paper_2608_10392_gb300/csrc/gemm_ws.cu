@@ -112,12 +112,16 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       mbar_init(fullA(s), 1);
       mbar_init(emptyA(s), Cfg<MODE>::kMmaWarps);
     }
+    // With the down projection's two sub-tiles split between the issuers,
+    // each accumulator and each weight slab has a single issuer; otherwise
+    // both issuers release every one of them.
+    const int owners = (MODE == 1 && p.n_sub == 2) ? 1 : Cfg<MODE>::kMmaWarps;
     for (int s = 0; s < n_slabs; ++s) {
       mbar_init(wfull(s), 1);
-      mbar_init(wempty(s), Cfg<MODE>::kMmaWarps);
+      mbar_init(wempty(s), owners);
     }
     for (int a = 0; a < 2; ++a) {
-      mbar_init(accf(a), Cfg<MODE>::kMmaWarps);
+      mbar_init(accf(a), owners);
       mbar_init(acce(a), kEpiWarps);
     }
     *abort_flag = 0;
@@ -234,9 +238,10 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // tensor pipe takes it, so one issuer's bookkeeping between MMA groups
     // would leave the pipe idle; the other issuer's MMAs fill those gaps.
     // Up (and a single-sub-tile down): warp m computes columns
-    // [m bn/2, (m+1) bn/2) of every accumulator. Down with two sub-tiles:
-    // warp m computes sub-tile m. Both walk every tile, so both wait for the
-    // same stages and weight runs, and each barrier they release counts both.
+    // [m bn/2, (m+1) bn/2) of every accumulator, and every stage, slab and
+    // accumulator barrier counts both warps' releases. Down with two
+    // sub-tiles: warp m computes sub-tile m; the A stages count both warps,
+    // each sub-tile's slabs and accumulator only their own issuer.
     // Within a warp the whole warp runs the loop (warp-uniform values) and an
     // elected lane issues; the next stage's barrier is tested before the
     // current stage's MMAs go out and read back after.
@@ -319,16 +324,10 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           if (!ok) break;
           if (elect_one()) umma_commit(accf(acc));
           __syncwarp();
-        } else {
-          // the other warp's sub-tile: this warp still owes its arrival on the
-          // accumulator and, at a group change, on the sub-tile's slabs
-          if (elect_one()) {
-            mbar_arrive(accf(acc));
-            if (release)
-              for (int kb = 0; kb < p.num_kb; ++kb) umma_commit(wempty(ns * p.num_kb + kb));
-          }
-          __syncwarp();
         }
+        // (the other warp's sub-tile: its accumulator and slabs have that
+        // warp as their only issuer; an arrival from this warp could run a
+        // whole tile or group ahead of the MMAs it stands for)
         if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
       }
       if (!ok) break;

@@ -288,3 +288,30 @@ def test_vit_s_streaming_kernels(monkeypatch):
     wl = workloads.make_workload(workloads.spec("vit_s", tokens=4000))
     g = run_gpu(wl)
     assert_parity(wl, g, compare(wl, g, sample=800))
+
+
+def test_repeated_forwards_match_streaming_kernels(monkeypatch):
+    """Ten forwards of the ViT-S layer through the weight-stationary kernels
+    agree with the streaming kernels token by token (the two differ only in
+    the order of the fp32 additions into the accumulator): catches
+    synchronisation races that corrupt a tile now and then."""
+    s = workloads.spec("vit_s")
+    wl = workloads.make_workload(s)
+    dev = torch.device("cuda")
+
+    def layer():
+        L = make_layer(s)
+        L.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
+        return L
+
+    x = wl.x.to(dev)
+    monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
+    ref = layer().forward(x).float()
+    monkeypatch.delenv("UNIF_MOE_GEMM_KERNELS")
+    L = layer()
+    for _ in range(10):
+        y = L.forward(x).float()
+        torch.cuda.synchronize()
+        assert L.sync_status() == 0
+        rel = (y - ref).abs().amax(1) / ref.abs().amax(1).clamp_min(1e-6)
+        assert float(rel.max()) < 1e-2, int((rel >= 1e-2).sum())
