@@ -68,6 +68,7 @@ struct Params {
   const int32_t* n_tiles;
   const int32_t* tile_group;
   const int32_t* tile_row0;
+  const int32_t* tile_rows;  // rows of each tile that are not padding
   const int32_t* row_tok;
   const float* row_w;
   int n_sub;       // N sub-tiles per 128-row tile
@@ -151,10 +152,12 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       const int brow = e * p.H + blk * p.M + ns * p.bn;
       // this tile's 128 row tokens, in the warp's own shared-memory slot
       int* tok = tok_smem + warp * kBM;
+      const int r0 = p.tile_row0[tile], nrow = p.tile_rows[tile];
       __syncwarp();
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const int t = p.row_tok[tile * kBM + 32 * i + lane];  // padding rows: token 0, unused
+        // padding rows: token 0, unused
+        const int t = 32 * i + lane < nrow ? p.row_tok[r0 + 32 * i + lane] : 0;
         tok[32 * i + lane] = t < 0 ? 0 : t;
       }
       __syncwarp();
@@ -248,10 +251,11 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     int acc = 0;
     uint32_t acc_phase = 0;
     // down: this thread's row token and weight, fetched one tile ahead
-    int t_nxt = 0;
+    int t_nxt = -1;
     float w_nxt = 0.f;
-    if (MODE == 1 && blockIdx.x < n_items) {
-      const int r = (blockIdx.x / p.n_sub) * kBM + q * 32 + lane;
+    if (MODE == 1 && blockIdx.x < n_items &&
+        q * 32 + lane < p.tile_rows[blockIdx.x / p.n_sub]) {
+      const int r = p.tile_row0[blockIdx.x / p.n_sub] + q * 32 + lane;
       t_nxt = p.row_tok[r];
       w_nxt = p.row_w[r];
     }
@@ -261,9 +265,11 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       const int t_cur = t_nxt;
       const float w_cur = w_nxt;
       if (MODE == 1 && item + (int)gridDim.x < n_items) {
-        const int r = ((item + gridDim.x) / p.n_sub) * kBM + q * 32 + lane;
-        t_nxt = p.row_tok[r];
-        w_nxt = p.row_w[r];
+        const int nt = (item + gridDim.x) / p.n_sub;
+        const int r = p.tile_row0[nt] + q * 32 + lane;
+        const bool real = q * 32 + lane < p.tile_rows[nt];
+        t_nxt = real ? p.row_tok[r] : -1;
+        w_nxt = real ? p.row_w[r] : 0.f;
       }
       if (!wait_warp(accf_bar(acc), acc_phase, abort_flag, p.status, p.wait_limit)) break;
       tc_fence_after();
@@ -370,6 +376,8 @@ constexpr size_t kRtSmem = 1024 + kRtStages * (kStageA + kRtStageB) + 256;
 
 struct RouterTcParams {
   DecideArgs dec;
+  GroupArgs grp;
+  int fused;     // 1: the router also lays out the group rows (group_rows)
   int d, Cp;
   uint32_t tmem_cols;
   float* y32;
@@ -463,12 +471,20 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     }
     const int q = warp & 3;
     const int row = q * 32 + lane;
+    // logits and affinities overlay the (now idle) operand ring
+    float* zs = reinterpret_cast<float*>(smem);
+    float* ss = zs + kBM * (Cp + 1);                                      // [128][2K + 1]
+    uint32_t* cscr = reinterpret_cast<uint32_t*>(ss + kBM * (2 * K + 1));  // [4][128]
+    float* sv = ss + row * (2 * K + 1);
+    const int t = t0 + row;
+    uint64_t shr = 0ull, em = 0ull;
+    float alpha = 0.f;
+    const int G = p.grp.G;
+    int32_t* cnt_s = reinterpret_cast<int32_t*>(cscr + 4 * 128);  // [4][G] (grouping)
+    int32_t* base_s = cnt_s + 4 * G;                              // [4][G]
+    int32_t* misc_s = base_s + 4 * G;                             // [8]
     if (wait_warp(accf, 0u, abort_flag, p.status, p.wait_limit)) {
       tc_fence_after();
-      // logits and affinities overlay the (now idle) operand ring
-      float* zs = reinterpret_cast<float*>(smem);
-      float* ss = zs + kBM * (Cp + 1);                                      // [128][2K + 1]
-      uint32_t* cscr = reinterpret_cast<uint32_t*>(ss + kBM * (2 * K + 1));  // [4][128]
       float* z = zs + row * (Cp + 1);
       for (int c = 0; c < Cp; c += 32) {
         float v[32];
@@ -476,12 +492,28 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
 #pragma unroll
         for (int i = 0; i < 32; ++i) z[c + i] = v[i];
       }
-      const int t = t0 + row;
       const bool valid = t < p.dec.T && (p.dec.mask == nullptr || p.dec.mask[t] != 0);
-      uint64_t shr, em;
-      decide_token(p.dec, t, valid, z, ss + row * (2 * K + 1), shr, em);
+      decide_token(p.dec, t, valid, z, sv, shr, em, alpha);
       const int chunk = blockIdx.x * (kBM / 32) + q;
-      if (chunk < p.dec.n_chunks) count_chunk_pairs(p.dec, chunk, lane, shr, em, cscr + q * 128);
+      if (!p.fused) {
+        if (chunk < p.dec.n_chunks)
+          count_chunk_pairs(p.dec, lane, shr, em, cscr + q * 128,
+                            p.dec.chunk_cnt + chunk, p.dec.n_chunks);
+      } else {
+        // per-chunk counts stay in shared memory (chunk q = tokens
+        // 32 q .. 32 q + 31 of this CTA)
+        count_chunk_pairs(p.dec, lane, shr, em, cscr + q * 128, cnt_s + q * G, 1);
+      }
+    }
+    if (p.fused) {
+      // all four decision warps meet here, also when a wait gave up (which
+      // sets the abort flag for all of them), then place this CTA's rows
+      named_bar(1, 128);
+      if (row == 0) misc_s[7] = *abort_flag;  // one reading for all four warps
+      named_bar(1, 128);
+      if (!misc_s[7])
+        group_rows<4>(p.grp, blockIdx.x, row, q, lane, t, shr, em, alpha, sv, cscr + q * 128,
+                      cnt_s, base_s, misc_s, 1);
     }
   }
   tc_fence_before();
@@ -594,6 +626,7 @@ cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t
   (void)T;
   tc::Params p;
   p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group; p.tile_row0 = L->ws.tile_row0;
+  p.tile_rows = L->ws.tile_rows;
   p.row_tok = L->ws.row_tok; p.row_w = L->ws.row_w;
   p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;
   p.x = static_cast<const __nv_bfloat16*>(x);
@@ -645,6 +678,23 @@ cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* ma
   if (!tc::encode_2d(&tm_x, x, L->d, (uint64_t)T, tc::kBK, tc::kBM)) return cudaErrorInvalidValue;
   tc::RouterTcParams p;
   p.dec = decide_args(L, mask, T, b_out, k_out);
+  p.fused = L->fused_group ? 1 : 0;
+  if (L->fused_group) {
+    Workspace& w = L->ws;
+    GroupArgs& g = p.grp;
+    g.G = L->G; g.K = L->K; g.B = L->B;
+    g.n_ctas = (T + tc::kBM - 1) / tc::kBM;
+    g.region = L->region_rows;
+    L->epoch = (L->epoch + 1) & 0x3FFFFFFFu;
+    if (L->epoch == 0) L->epoch = 1;
+    g.epoch = L->epoch;
+    g.lb_agg = w.lb_agg; g.lb_incl = w.lb_incl; g.lb_flag = w.lb_flag; g.ticket = w.ticket;
+    g.row_tok = w.row_tok; g.row_w = w.row_w;
+    g.grp_cnt = w.grp_cnt; g.grp_off = w.grp_off; g.n_tiles = w.n_tiles;
+    g.tile_group = w.tile_group; g.tile_row0 = w.tile_row0; g.tile_rows = w.tile_rows;
+    g.status = w.status;
+    g.wait_limit = tc::g_wait_limit;
+  }
   p.d = L->d;
   p.Cp = L->router_cols_pad;
   p.tmem_cols = p.Cp <= 32 ? 32u : (p.Cp <= 64 ? 64u : (p.Cp <= 128 ? 128u : 256u));

@@ -65,6 +65,8 @@ struct Cfg {
 struct Params {
   const int32_t* n_tiles;
   const int32_t* tile_group;
+  const int32_t* tile_row0;  // first row of each tile in row_tok / row_w
+  const int32_t* tile_rows;  // rows of each tile that are not padding
   const int32_t* row_tok;
   const float* row_w;
   int n_sub, bn, num_kb;
@@ -151,15 +153,29 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int j = lane & 7, rsub = lane >> 3;
     bool ok = true;
     int seq = 0;
-    int tk_nxt[4];  // the next tile's row tokens, loaded one tile ahead
+    // the next tile's row tokens, loaded one tile ahead (and its first row
+    // index two tiles ahead)
+    // (padding rows gather token 0; their h rows are never used)
+    int tk_nxt[4];
+    int r0_nxt = t_begin + 1 < t_end ? p.tile_row0[t_begin + 1] : 0;
+    int n_nxt = t_begin + 1 < t_end ? p.tile_rows[t_begin + 1] : 0;
+    {
+      const int r0 = t_begin < t_end ? p.tile_row0[t_begin] : 0;
+      const int n = t_begin < t_end ? p.tile_rows[t_begin] : 0;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) tk_nxt[i] = t_begin < t_end ? p.row_tok[t_begin * kBM + 32 * i + lane] : 0;
+      for (int i = 0; i < 4; ++i) tk_nxt[i] = 32 * i + lane < n ? p.row_tok[r0 + 32 * i + lane] : 0;
+    }
     for (int tile = t_begin; tile < t_end && ok; ++tile, seq += p.num_kb) {
       int tk[4];
+      const int r0n = r0_nxt, nn = n_nxt;
+      if (tile + 2 < t_end) {
+        r0_nxt = p.tile_row0[tile + 2];
+        n_nxt = p.tile_rows[tile + 2];
+      }
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        tk[i] = tk_nxt[i] < 0 ? 0 : tk_nxt[i];  // padding rows: token 0, unused
-        if (tile + 1 < t_end) tk_nxt[i] = p.row_tok[(tile + 1) * kBM + 32 * i + lane];
+        tk[i] = tk_nxt[i] < 0 ? 0 : tk_nxt[i];
+        if (tile + 1 < t_end) tk_nxt[i] = 32 * i + lane < nn ? p.row_tok[r0n + 32 * i + lane] : 0;
       }
       const int first = (warp - seq % kProducerWarps + kProducerWarps) % kProducerWarps;
       if (first >= p.num_kb) continue;
@@ -350,10 +366,14 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int c_begin = half * cols;
     int acc = 0;
     uint32_t acc_phase = 0;
-    int t_nxt = 0;
+    // down: this thread's row token (-1 for a padding row) and weight, one
+    // tile ahead
+    int t_nxt = -1;
     float w_nxt = 0.f;
-    if (MODE == 1 && t_begin < t_end) {
-      const int r = t_begin * kBM + q * 32 + lane;
+    int r0_nxt = (MODE == 1 && t_begin + 1 < t_end) ? p.tile_row0[t_begin + 1] : 0;
+    int n_nxt = (MODE == 1 && t_begin + 1 < t_end) ? p.tile_rows[t_begin + 1] : 0;
+    if (MODE == 1 && t_begin < t_end && q * 32 + lane < p.tile_rows[t_begin]) {
+      const int r = p.tile_row0[t_begin] + q * 32 + lane;
       t_nxt = p.row_tok[r];
       w_nxt = p.row_w[r];
     }
@@ -365,9 +385,13 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       const int t_cur = t_nxt;
       const float w_cur = w_nxt;
       if (MODE == 1 && tile + 1 < t_end) {
-        const int r = (tile + 1) * kBM + q * 32 + lane;
-        t_nxt = p.row_tok[r];
-        w_nxt = p.row_w[r];
+        const int r = r0_nxt + q * 32 + lane;
+        t_nxt = q * 32 + lane < n_nxt ? p.row_tok[r] : -1;
+        w_nxt = q * 32 + lane < n_nxt ? p.row_w[r] : 0.f;
+        if (tile + 2 < t_end) {
+          r0_nxt = p.tile_row0[tile + 2];
+          n_nxt = p.tile_rows[tile + 2];
+        }
       }
       for (int ns = 0; ns < p.n_sub; ++ns) {
         if (!wait_warp(accf(acc), acc_phase, abort_flag, p.status, p.wait_limit)) {
@@ -493,8 +517,8 @@ int gemm_ws_setup(unif_moe_layer* L) {
 
 static tc::ws::Params ws_params(unif_moe_layer* L, const void* x) {
   tc::ws::Params p;
-  p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group;
-  p.row_tok = L->ws.row_tok; p.row_w = L->ws.row_w;
+  p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group; p.tile_row0 = L->ws.tile_row0;
+  p.tile_rows = L->ws.tile_rows; p.row_tok = L->ws.row_tok; p.row_w = L->ws.row_w;
   p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;
   p.x = static_cast<const __nv_bfloat16*>(x);
   p.h = static_cast<__nv_bfloat16*>(L->ws.hbuf);

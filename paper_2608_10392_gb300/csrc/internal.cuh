@@ -35,8 +35,14 @@ struct Workspace {
   int32_t* n_tiles = nullptr;    // [1]
   int32_t* tile_group = nullptr; // [max_tiles]
   int32_t* tile_row0 = nullptr;  // [max_tiles]
-  int32_t* row_tok = nullptr;    // [max_rows] (-1 = padding row)
-  float* row_w = nullptr;        // [max_rows]
+  int32_t* tile_rows = nullptr;  // [max_tiles] rows of the tile that are not padding
+  int32_t* row_tok = nullptr;    // [max_rows], or [G][region] when the router groups (-1 = padding)
+  float* row_w = nullptr;        // same layout
+  // Look-back state of the grouping inside the router (bf16 layers).
+  int32_t* lb_agg = nullptr;     // [router CTAs][G]
+  int32_t* lb_incl = nullptr;    // [router CTAs][G]
+  uint32_t* lb_flag = nullptr;   // [router CTAs]
+  int32_t* ticket = nullptr;     // [1]
   // Intermediate activations h = GeLU(x K_e[:, H_b]) per row, and the fp32
   // output accumulator.
   void* hbuf = nullptr;          // [max_rows][M] (layer dtype)
@@ -65,6 +71,11 @@ struct unif_moe_layer {
   int router_cols = 0;      // 1 + K + B
   int router_cols_pad = 0;  // padded to a multiple of 32
   int n_sm = 0;
+  // bf16 layers: the tensor-core router also lays out the rows of each group
+  // in its own region of region_rows rows (no separate grouping kernels).
+  bool fused_group = false;
+  int region_rows = 0;
+  uint32_t epoch = 0;
   int device = 0;
   bool loaded = false;
   int last_T = -1;

@@ -180,11 +180,14 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
   const int t = t0 + tid;
   const bool valid = t < a.dec.T && (a.dec.mask == nullptr || a.dec.mask[t] != 0);
   uint64_t shr, em;
-  decide_token(a.dec, t, valid, zs + tid * (Cp + 1), ss + tid * (2 * K + 1), shr, em);
+  float alpha;
+  decide_token(a.dec, t, valid, zs + tid * (Cp + 1), ss + tid * (2 * K + 1), shr, em, alpha);
 
   // ---- (expert, block) pairs per group for this warp's 32 tokens ----
   const int chunk = blockIdx.x * (kRouterTokens / kWarpChunk) + warp;
-  if (chunk < a.dec.n_chunks) count_chunk_pairs(a.dec, chunk, lane, shr, em, cscr + warp * 128);
+  if (chunk < a.dec.n_chunks)
+    count_chunk_pairs(a.dec, lane, shr, em, cscr + warp * 128, a.dec.chunk_cnt + chunk,
+                      a.dec.n_chunks);
 }
 
 // get_routing helper: experts by decreasing affinity (ties to the lower
@@ -239,8 +242,8 @@ group_scatter_kernel(const uint64_t* __restrict__ shr_o, const uint64_t* __restr
                      int K, int B, int n_chunks, const int32_t* __restrict__ chunk_off,
                      const int32_t* __restrict__ grp_cnt, int32_t* __restrict__ grp_off,
                      int32_t* __restrict__ n_tiles, int32_t* __restrict__ tile_group,
-                     int32_t* __restrict__ tile_row0, int32_t* __restrict__ row_tok,
-                     float* __restrict__ row_w) {
+                     int32_t* __restrict__ tile_row0, int32_t* __restrict__ tile_rows,
+                     int32_t* __restrict__ row_tok, float* __restrict__ row_w) {
   extern __shared__ int goff[];  // [G + 1]
   __shared__ int wsum[4];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -272,6 +275,7 @@ group_scatter_kernel(const uint64_t* __restrict__ shr_o, const uint64_t* __restr
     for (int i = tid; i < padded / kTileRows; i += 128) {
       tile_group[off / kTileRows + i] = g;
       tile_row0[off / kTileRows + i] = off + i * kTileRows;
+      tile_rows[off / kTileRows + i] = min(kTileRows, cnt - i * kTileRows);
     }
     for (int r = off + cnt + tid; r < off + padded; r += 128) { row_tok[r] = -1; row_w[r] = 0.f; }
   }
@@ -610,7 +614,7 @@ cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s) {
   chunk_scan_kernel<<<(L->G + 7) / 8, 256, 0, s>>>(L->G, n_chunks, w.chunk_cnt, w.grp_cnt);
   group_scatter_kernel<<<(n_chunks + 3) / 4, 128, scatter_smem(L), s>>>(
       w.shr_mask, w.exp_mask, w.alpha, w.s, T, L->K, L->B, n_chunks, w.chunk_cnt, w.grp_cnt,
-      w.grp_off, w.n_tiles, w.tile_group, w.tile_row0, w.row_tok, w.row_w);
+      w.grp_off, w.n_tiles, w.tile_group, w.tile_row0, w.tile_rows, w.row_tok, w.row_w);
   return cudaGetLastError();
 }
 

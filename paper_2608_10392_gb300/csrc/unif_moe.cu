@@ -7,6 +7,7 @@
 #include <stdarg.h>
 #include <stdio.h>
 #include <string.h>
+#include <vector>
 
 #include <new>
 
@@ -67,7 +68,8 @@ void free_all(unif_moe_layer* L) {
                   L->ws.grp_cnt, L->ws.grp_off, L->ws.n_tiles, L->ws.tile_group,
                   L->ws.tile_row0, L->ws.row_tok, L->ws.row_w, L->ws.hbuf, L->ws.y32,
                   L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
-                  L->ws.k_stage, L->ws.status};
+                  L->ws.k_stage, L->ws.status, L->ws.lb_agg, L->ws.lb_incl, L->ws.lb_flag,
+                  L->ws.ticket, L->ws.tile_rows};
   for (void* q : ptrs)
     if (q) cudaFree(q);
 }
@@ -182,7 +184,18 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   ALLOC(w.chunk_cnt, (size_t)L->G * L->max_chunks);
   ALLOC(w.grp_cnt, (size_t)L->G); ALLOC(w.grp_off, (size_t)L->G + 1); ALLOC(w.n_tiles, 1);
   ALLOC(w.tile_group, (size_t)L->max_tiles); ALLOC(w.tile_row0, (size_t)L->max_tiles);
-  ALLOC(w.row_tok, (size_t)L->max_rows); ALLOC(w.row_w, (size_t)L->max_rows);
+  ALLOC(w.tile_rows, (size_t)L->max_tiles);
+  // bf16 layers group inside the router: each group owns a region of
+  // max_tokens rows (rounded up to whole tiles) in the row arrays
+  L->fused_group = dtype == UNIF_MOE_BF16 && L->G <= 1024;
+  L->region_rows = (max_tokens + 127) / 128 * 128;
+  const size_t row_cap = L->fused_group ? (size_t)L->G * L->region_rows : (size_t)L->max_rows;
+  ALLOC(w.row_tok, row_cap); ALLOC(w.row_w, row_cap);
+  const size_t lb_ctas = ((size_t)max_tokens + 127) / 128;
+  if (L->fused_group) {
+    ALLOC(w.lb_agg, lb_ctas * L->G); ALLOC(w.lb_incl, lb_ctas * L->G);
+    ALLOC(w.lb_flag, lb_ctas); ALLOC(w.ticket, 1);
+  }
   void* hb = nullptr;
   if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&hb), es * (size_t)L->max_rows * M);
   w.hbuf = hb;
@@ -190,7 +203,10 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   ALLOC(w.status, 1);
 #undef ALLOC
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
-                            cudaMemset(w.y32, 0, sizeof(float) * T * d_model) != cudaSuccess)) {
+                            cudaMemset(w.y32, 0, sizeof(float) * T * d_model) != cudaSuccess ||
+                            (L->fused_group &&
+                             (cudaMemset(w.lb_flag, 0, sizeof(uint32_t) * lb_ctas) != cudaSuccess ||
+                              cudaMemset(w.ticket, 0, sizeof(int32_t)) != cudaSuccess)))) {
     set_error("cudaMemset failed");
     rc = UNIF_MOE_ERR_CUDA;
   }
@@ -253,7 +269,7 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
     CK(unif::launch_router(L, x, token_mask, T, shared_counts, residual_counts, s));
   }
   if (ev[1]) CK(cudaEventRecord(ev[1], s));
-  CK(unif::launch_permute(L, T, s));
+  if (!L->fused_group) CK(unif::launch_permute(L, T, s));
   if (ev[2]) CK(cudaEventRecord(ev[2], s));
   if (L->dtype == UNIF_MOE_BF16) {
     CK(unif::launch_gemms_tc(L, x, T, ev[3], s));
@@ -335,7 +351,30 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
   int32_t total = 0;
   if (L->last_T > 0) CK(cudaMemcpyAsync(&total, L->ws.grp_off + L->G, sizeof(int32_t), dh, s));
   CK(cudaStreamSynchronize(s));
-  if (L->last_T > 0) {
+  if (L->last_T > 0 && L->fused_group) {
+    // rows live in per-group regions on the device: gather them group by
+    // group into the contiguous padded layout
+    std::vector<int32_t> cnt(L->G), off(L->G + 1);
+    CK(cudaMemcpyAsync(cnt.data(), L->ws.grp_cnt, sizeof(int32_t) * L->G, dh, s));
+    CK(cudaMemcpyAsync(off.data(), L->ws.grp_off, sizeof(int32_t) * (L->G + 1), dh, s));
+    CK(cudaStreamSynchronize(s));
+    if (counts) memcpy(counts, cnt.data(), sizeof(int32_t) * L->G);
+    if (offsets) memcpy(offsets, off.data(), sizeof(int32_t) * (L->G + 1));
+    for (int g = 0; g < L->G; ++g) {
+      const size_t n = (size_t)cnt[g];
+      const size_t src = (size_t)g * L->region_rows;
+      // padding rows (the device leaves them untouched): token -1, weight 0
+      for (int r = off[g] + cnt[g]; r < off[g + 1]; ++r) {
+        if (row_token) row_token[r] = -1;
+        if (row_weight) row_weight[r] = 0.f;
+      }
+      if (n == 0) continue;
+      if (row_token)
+        CK(cudaMemcpyAsync(row_token + off[g], L->ws.row_tok + src, sizeof(int32_t) * n, dh, s));
+      if (row_weight)
+        CK(cudaMemcpyAsync(row_weight + off[g], L->ws.row_w + src, sizeof(float) * n, dh, s));
+    }
+  } else if (L->last_T > 0) {
     if (counts) CK(cudaMemcpyAsync(counts, L->ws.grp_cnt, sizeof(int32_t) * L->G, dh, s));
     if (offsets) CK(cudaMemcpyAsync(offsets, L->ws.grp_off, sizeof(int32_t) * (L->G + 1), dh, s));
     if (row_token && total > 0) CK(cudaMemcpyAsync(row_token, L->ws.row_tok, sizeof(int32_t) * total, dh, s));
