@@ -266,21 +266,21 @@ __device__ __forceinline__ void count_chunk_pairs(const DecideArgs& a, int lane,
 // Grouping inside the router (Eq. 35's pairs laid out per group)
 // ---------------------------------------------------------------------------
 // Each group g owns a region of `region` rows (at most one row per token) in
-// row_tok / row_w, so a router CTA can place its tokens' rows as soon as it
-// knows, per group, how many rows the CTAs before it produced: a single-pass
-// scan with decoupled look-back over per-CTA aggregates. The last CTA to
-// finish numbers the tiles (128 rows) of every group into the tile list,
-// with each tile's count of real rows (the rest of a group's last tile is
-// padding, which the GEMM kernels skip).
+// row_tok / row_w. A router CTA reserves its rows of every group with one
+// atomic add on the group's fill counter, so rows of different CTAs land in
+// arrival order (within a CTA, in token order); nothing downstream depends
+// on the order of a group's rows. The CTA that finishes last (a ticket
+// counter) reads the final fills, the group sizes, and numbers the tiles
+// (128 rows) of every group into the tile list, with each tile's count of
+// real rows (the rest of a group's last tile is padding, which the GEMM
+// kernels skip). The combine kernel zeroes the fill and ticket counters for
+// the next forward, also after a forward whose router gave up a wait.
 struct GroupArgs {
   int G, K, B;
   int n_ctas;
   int region;
-  uint32_t epoch;          // this forward's tag in the look-back flags
-  int32_t* lb_agg;         // [n_ctas][G] rows per CTA and group
-  int32_t* lb_incl;        // [n_ctas][G] rows of CTAs 0..c per group
-  uint32_t* lb_flag;       // [n_ctas] (epoch << 2) | 1 aggregate, | 2 inclusive
-  int32_t* ticket;         // CTAs done; the last resets it
+  int32_t* fill;           // [G] rows reserved so far (0 at the start of a forward)
+  int32_t* ticket;         // [1] CTAs done (0 at the start of a forward)
   int32_t* row_tok;
   float* row_w;
   int32_t* grp_cnt;
@@ -290,177 +290,119 @@ struct GroupArgs {
   int32_t* tile_row0;
   int32_t* tile_rows;
   int* status;
-  long long wait_limit;
 };
-constexpr int kMaxGroupsPerThread = 8;
 
 __device__ __forceinline__ void named_bar(uint32_t id, uint32_t n) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
-__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-__device__ __forceinline__ void st_release_u32(uint32_t* p, uint32_t v) {
-  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+
+// Shared-memory ints group_rows needs.
+__host__ __device__ constexpr int group_rows_smem_ints(int NW, int G) {
+  return NW * G + 8;
 }
 
-// Runs in the NW decision warps of router CTA `cta` (threads tid = 0 ..
-// NW*32-1, named barrier `bar`), after warp w's count_chunk_pairs wrote its
-// 32-token chunk's per-group pair counts to cnt_s[w][g] and its lane masks
-// to `masks`. Lane `lane` of warp w holds token t
-// (valid or not) with its shared block set, residual expert set, alpha and
-// affinities s_tok[0..K-1]. base_s is [NW][G] ints of shared memory, misc_s
-// NW + 3 ints.
+// Exclusive scan of v over the NT threads of the decision warps (thread
+// order); returns the scan and sets total. warp_s holds NW ints.
 template <int NW>
-__device__ void group_rows(const GroupArgs& a, int cta, int tid, int w, int lane, int t,
-                           uint64_t shr, uint64_t em, float alpha, const float* s_tok,
-                           const uint32_t* masks, const int32_t* cnt_s, int32_t* base_s,
-                           int32_t* misc_s, uint32_t bar) {
-  constexpr int NT = NW * 32;
-  const int G = a.G;
-  const uint32_t tag = a.epoch << 2;
-  // 1. this CTA's rows per group, published
-  int gl[kMaxGroupsPerThread], agg[kMaxGroupsPerThread], excl[kMaxGroupsPerThread];
-  int ng = 0;
-  for (int g = tid; g < G && ng < kMaxGroupsPerThread; g += NT) {
-    int sum = 0;
-    for (int v = 0; v < NW; ++v) sum += cnt_s[v * G + g];
-    gl[ng] = g;
-    agg[ng] = sum;
-    excl[ng] = 0;
-    a.lb_agg[(size_t)cta * G + g] = sum;
-    ++ng;
-  }
-  __threadfence();
-  named_bar(bar, NT);
-  if (tid == 0) st_release_u32(a.lb_flag + cta, tag | 1u);
-  // 2. rows of all CTAs before this one: walk back 32 CTAs at a time (warp
-  // 0 reads their flags together), summing aggregates up to the nearest CTA
-  // whose inclusive count is published
-  for (int top = cta - 1; top >= 0;) {
-    if (w == 0) {
-      const int j = top - lane;
-      uint32_t st = 0u;
-      if (j >= 0) {
-        const long long t0 = clock64();
-        for (;;) {
-          const uint32_t f = ld_acquire_u32(a.lb_flag + j);
-          if ((f & ~3u) == tag && (f & 3u) != 0u) { st = f & 3u; break; }
-          if (clock64() - t0 > a.wait_limit) {
-            atomicOr(a.status, kStatusTimeout);
-            st = 2u;  // give up: treat as published (the result is invalid anyway)
-            break;
-          }
-        }
-      }
-      const unsigned incl_lanes = __ballot_sync(0xffffffffu, st == 2u);
-      // nearest inclusive CTA in this window, or none (-1)
-      const int k = incl_lanes ? __ffs(incl_lanes) - 1 : -1;
-      if (lane == 0) {
-        misc_s[NW + 1] = k;
-        misc_s[NW + 2] = min(32, top + 1);  // CTAs in this window
-      }
-    }
-    named_bar(bar, NT);
-    const int k = misc_s[NW + 1], n = misc_s[NW + 2];
-    named_bar(bar, NT);  // misc_s is rewritten by the next window
-    const int n_agg = k >= 0 ? k : n;
-    for (int i = 0; i < ng; ++i) {
-      int sum = 0;
-      for (int v = 0; v < n_agg; ++v) sum += __ldcg(a.lb_agg + (size_t)(top - v) * G + gl[i]);
-      if (k >= 0) sum += __ldcg(a.lb_incl + (size_t)(top - k) * G + gl[i]);
-      excl[i] += sum;
-    }
-    if (k >= 0) break;
-    top -= n;
-  }
-  // 3. inclusive counts published; each warp's first row per group
-  for (int i = 0; i < ng; ++i) {
-    const int g = gl[i];
-    a.lb_incl[(size_t)cta * G + g] = excl[i] + agg[i];
-    int b = excl[i];
-    for (int v = 0; v < NW; ++v) {
-      base_s[v * G + g] = b;
-      b += cnt_s[v * G + g];
-    }
-  }
-  __threadfence();
-  named_bar(bar, NT);
-  if (tid == 0) st_release_u32(a.lb_flag + cta, tag | 2u);
-  // 4. this lane's rows, one per (expert, block) pair of its token: the
-  // row's rank among the chunk's tokens in the group (tokens stay in index
-  // order) comes from the lane masks count_chunk_pairs left in `masks`
-  // (masks[blk]: lanes sharing block blk, masks[64 + j]: lanes selecting
-  // residual expert j)
-  {
-    const uint64_t full = (a.B == 64) ? ~0ull : ((1ull << a.B) - 1ull);
-    const unsigned lt_mask = (1u << lane) - 1u;
-    const int32_t* base = base_s + w * G;
-    for (uint64_t m = shr; m != 0ull; m &= m - 1ull) {
-      const int blk = __ffsll((long long)m) - 1;
-      const size_t pos = (size_t)blk * a.region + base[blk] + __popc(masks[blk] & lt_mask);
-      a.row_tok[pos] = t;
-      a.row_w[pos] = alpha;
-    }
-    const uint64_t comp = ~shr & full;
-    for (uint64_t ee = em; ee != 0ull; ee &= ee - 1ull) {
-      const int j = __ffsll((long long)ee) - 1;
-      const float wt = s_tok[j];
-      const uint32_t ej = masks[64 + j];
-      for (uint64_t m = comp; m != 0ull; m &= m - 1ull) {
-        const int blk = __ffsll((long long)m) - 1;
-        const int g = (j + 1) * a.B + blk;
-        const size_t pos = (size_t)g * a.region + base[g] + __popc(ej & ~masks[blk] & lt_mask);
-        a.row_tok[pos] = t;
-        a.row_w[pos] = wt;
-      }
-    }
-  }
-  // 5. the last CTA to finish builds the tile list
-  if (tid == 0) {
-    int old;
-    asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], 1;" : "=r"(old) : "l"(a.ticket) : "memory");
-    misc_s[NW] = old;
-  }
-  named_bar(bar, NT);
-  if (misc_s[NW] != a.n_ctas - 1) return;
-  if (tid == 0) *a.ticket = 0;  // every CTA has taken its ticket
-  // group totals into shared memory first (one round of loads), then the
-  // groups in contiguous runs per thread, so that a block scan numbers the
-  // tiles in group order
-  int32_t* tot = base_s;  // no longer needed for row offsets
-  for (int g = tid; g < G; g += NT) tot[g] = __ldcg(a.lb_incl + (size_t)(a.n_ctas - 1) * G + g);
-  named_bar(bar, NT);
-  const int per = (G + NT - 1) / NT;
-  const int g0 = min(G, tid * per), g1 = min(G, g0 + per);
-  int my_tiles = 0;
-  for (int g = g0; g < g1; ++g) my_tiles += (tot[g] + 127) / 128;
-  int inc = my_tiles;
+__device__ __forceinline__ int block_excl_scan1(int v, int tid, int lane, int w, int32_t* warp_s,
+                                                uint32_t bar, int& total) {
+  int inc = v;
   for (int o = 1; o < 32; o <<= 1) {
     const int n = __shfl_up_sync(0xffffffffu, inc, o);
     if (lane >= o) inc += n;
   }
-  if (lane == 31) misc_s[w] = inc;
-  named_bar(bar, NT);
-  int first_tile = inc - my_tiles;
-  for (int v = 0; v < w; ++v) first_tile += misc_s[v];
-  for (int g = g0; g < g1; ++g) {
-    const int cnt = tot[g];
-    const int tiles = (cnt + 127) / 128;
-    a.grp_cnt[g] = cnt;
-    a.grp_off[g] = first_tile * 128;
-    for (int i = 0; i < tiles; ++i) {
-      a.tile_group[first_tile + i] = g;
-      a.tile_row0[first_tile + i] = g * a.region + 128 * i;
-      a.tile_rows[first_tile + i] = min(128, cnt - 128 * i);
-    }
-    first_tile += tiles;
+  if (lane == 31) warp_s[w] = inc;
+  named_bar(bar, NW * 32);
+  int before = 0;
+  total = 0;
+#pragma unroll
+  for (int u = 0; u < NW; ++u) {
+    const int s = warp_s[u];
+    before += u < w ? s : 0;
+    total += s;
   }
-  if (tid == NT - 1) {
-    a.n_tiles[0] = first_tile;
-    a.grp_off[G] = first_tile * 128;
+  named_bar(bar, NW * 32);
+  return before + inc - v;
+}
+
+// Runs in the NW decision warps of a router CTA (threads tid = 0 .. NW*32-1,
+// named barrier `bar`; thread tid holds token t0 + tid), after warp w's
+// count_chunk_pairs wrote its 32-token chunk's per-group pair counts to
+// sm[w * G + g] and its lane masks to masks[w * 128 ...] (masks[blk] = lanes
+// sharing block blk, masks[64 + j] = lanes selecting residual expert j).
+// Token i of the CTA has alpha at dec_s[i * dec_stride + 2K] and its
+// affinities s_1..s_K at dec_s[i * dec_stride + j]. `sm` has
+// group_rows_smem_ints(NW, G) ints.
+//
+// Threads take whole groups: with one warp per scheduler, per-row work must
+// be short and free of shared-memory round trips, so a thread walks its
+// group's member bits (token order) and writes the rows one after another.
+template <int NW>
+__device__ void group_rows(const GroupArgs& a, int tid, int w, int lane, int t0,
+                           const uint32_t* masks, const float* dec_s, int dec_stride, int32_t* sm,
+                           uint32_t bar) {
+  constexpr int NT = NW * 32;
+  const int G = a.G, B = a.B;
+  int32_t* cnt_s = sm;                    // [NW][G] chunk counts
+  int32_t* misc_s = cnt_s + NW * G;       // [8]: ticket flag, scan scratch (1..NW)
+  for (int g = tid; g < G; g += NT) {
+    // 1. this CTA's rows of group g, reserved in the group's region
+    int n = 0;
+#pragma unroll
+    for (int v = 0; v < NW; ++v) n += cnt_s[v * G + g];
+    if (n == 0) continue;
+    int base = atomicAdd(a.fill + g, n);
+    if (base + n > a.region) {  // stale counters: keep the writes inside the region
+      atomicOr(a.status, kStatusBadIndex);
+      continue;
+    }
+    // 2. the rows, in token order
+    const int e = g / B, blk = g - e * B;
+    const int wcol = e == 0 ? 2 * a.K : e - 1;
+    int32_t* tok = a.row_tok + (size_t)g * a.region + base;
+    float* wt = a.row_w + (size_t)g * a.region + base;
+    int r = 0;
+#pragma unroll
+    for (int c = 0; c < NW; ++c) {
+      const uint32_t sh = masks[c * 128 + blk];
+      uint32_t m = e == 0 ? sh : (masks[c * 128 + 64 + e - 1] & ~sh);
+      while (m != 0u && r < n) {
+        const int i = c * 32 + __ffs(m) - 1;
+        m &= m - 1u;
+        tok[r] = t0 + i;
+        wt[r] = dec_s[i * dec_stride + wcol];
+        ++r;
+      }
+    }
+  }
+  // 3. the CTA that finishes last numbers the tiles
+  __threadfence();
+  named_bar(bar, NT);
+  if (tid == 0) misc_s[0] = atomicAdd(a.ticket, 1) == a.n_ctas - 1;
+  named_bar(bar, NT);
+  if (!misc_s[0]) return;
+  __threadfence();
+  int carry = 0;
+  for (int g0 = 0; g0 < G; g0 += NT) {
+    const int g = g0 + tid;
+    const int tot = g < G ? min(__ldcg(a.fill + g), a.region) : 0;
+    const int nt = (tot + 127) / 128;
+    int total;
+    const int k0 = carry + block_excl_scan1<NW>(nt, tid, lane, w, misc_s + 1, bar, total);
+    carry += total;
+    if (g < G) {
+      a.grp_cnt[g] = tot;
+      a.grp_off[g] = k0 * 128;
+      for (int i = 0; i < nt; ++i) {
+        a.tile_group[k0 + i] = g;
+        a.tile_row0[k0 + i] = g * a.region + 128 * i;
+        a.tile_rows[k0 + i] = min(128, tot - 128 * i);
+      }
+    }
+  }
+  if (tid == 0) {
+    a.n_tiles[0] = carry;
+    a.grp_off[G] = carry * 128;
   }
 }
 

@@ -88,8 +88,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     Params p) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
+  // 1024-byte aligned base, derived from smem_raw by an offset so that the
+  // compiler keeps every access through it in the shared state space
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   constexpr int kStages = Cfg<MODE>::kStages;
   const uint32_t sA = smem_u32(smem);
   const uint32_t sB = sA + kStages * kStageA;
@@ -373,6 +374,15 @@ constexpr int kRtThreads = 192;   // warp 0 TMA, warp 1 TMEM + MMA, warps 2-5 de
 constexpr int kRtStages = 6;
 constexpr uint32_t kRtStageB = 160u * kBK * 2;  // up to 160 router columns
 constexpr size_t kRtSmem = 1024 + kRtStages * (kStageA + kRtStageB) + 256;
+constexpr int kRtRingBytes = kRtStages * (kStageA + kRtStageB);
+
+// Bytes of the operand ring that the decision warps reuse once the MMAs are
+// done: logits [128][Cp + 1] and decision scratch [128][2K + 1] (fp32), lane
+// masks [4][128], and (grouping) group_rows' counters.
+__host__ __device__ constexpr int router_overlay_bytes(int Cp, int K, int G, bool fused) {
+  return 4 * (kBM * (Cp + 1) + kBM * (2 * K + 1) + 4 * 128) +
+         (fused ? 4 * group_rows_smem_ints(4, G) : 0);
+}
 
 struct RouterTcParams {
   DecideArgs dec;
@@ -389,8 +399,9 @@ __global__ void __launch_bounds__(kRtThreads, 1)
 router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
                  RouterTcParams p) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
+  // 1024-byte aligned base, derived from smem_raw by an offset so that the
+  // compiler keeps every access through it in the shared state space
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const uint32_t sA = smem_u32(smem);
   const uint32_t sB = sA + kRtStages * kStageA;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kRtStages * (kStageA + kRtStageB));
@@ -480,9 +491,8 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     uint64_t shr = 0ull, em = 0ull;
     float alpha = 0.f;
     const int G = p.grp.G;
-    int32_t* cnt_s = reinterpret_cast<int32_t*>(cscr + 4 * 128);  // [4][G] (grouping)
-    int32_t* base_s = cnt_s + 4 * G;                              // [4][G]
-    int32_t* misc_s = base_s + 4 * G;                             // [8]
+    int32_t* gsm = reinterpret_cast<int32_t*>(cscr + 4 * 128);  // group_rows' counters
+    int32_t* misc_s = gsm + group_rows_smem_ints(4, G) - 8;
     if (wait_warp(accf, 0u, abort_flag, p.status, p.wait_limit)) {
       tc_fence_after();
       float* z = zs + row * (Cp + 1);
@@ -501,8 +511,9 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
                             p.dec.chunk_cnt + chunk, p.dec.n_chunks);
       } else {
         // per-chunk counts stay in shared memory (chunk q = tokens
-        // 32 q .. 32 q + 31 of this CTA)
-        count_chunk_pairs(p.dec, lane, shr, em, cscr + q * 128, cnt_s + q * G, 1);
+        // 32 q .. 32 q + 31 of this CTA); alpha joins the affinities
+        count_chunk_pairs(p.dec, lane, shr, em, cscr + q * 128, gsm + q * G, 1);
+        sv[2 * K] = alpha;
       }
     }
     if (p.fused) {
@@ -511,9 +522,7 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
       named_bar(1, 128);
       if (row == 0) misc_s[7] = *abort_flag;  // one reading for all four warps
       named_bar(1, 128);
-      if (!misc_s[7])
-        group_rows<4>(p.grp, blockIdx.x, row, q, lane, t, shr, em, alpha, sv, cscr + q * 128,
-                      cnt_s, base_s, misc_s, 1);
+      if (!misc_s[7]) group_rows<4>(p.grp, row, q, lane, t0, cscr, ss, 2 * K + 1, gsm, 1);
     }
   }
   tc_fence_before();
@@ -654,6 +663,10 @@ cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t
   return cudaGetLastError();
 }
 
+bool router_can_group(int Cp, int K, int G) {
+  return tc::router_overlay_bytes(Cp, K, G, true) <= tc::kRtRingBytes;
+}
+
 int router_tc_setup(unif_moe_layer* L) {
   if (L->router_cols_pad > 160 || L->d % tc::kBK != 0) {
     set_error("tensor-core router needs 1+K+B <= 160 and d %% 64 == 0");
@@ -685,15 +698,11 @@ cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* ma
     g.G = L->G; g.K = L->K; g.B = L->B;
     g.n_ctas = (T + tc::kBM - 1) / tc::kBM;
     g.region = L->region_rows;
-    L->epoch = (L->epoch + 1) & 0x3FFFFFFFu;
-    if (L->epoch == 0) L->epoch = 1;
-    g.epoch = L->epoch;
-    g.lb_agg = w.lb_agg; g.lb_incl = w.lb_incl; g.lb_flag = w.lb_flag; g.ticket = w.ticket;
+    g.fill = w.grp_fill; g.ticket = w.grp_fill + L->G;
     g.row_tok = w.row_tok; g.row_w = w.row_w;
     g.grp_cnt = w.grp_cnt; g.grp_off = w.grp_off; g.n_tiles = w.n_tiles;
     g.tile_group = w.tile_group; g.tile_row0 = w.tile_row0; g.tile_rows = w.tile_rows;
     g.status = w.status;
-    g.wait_limit = tc::g_wait_limit;
   }
   p.d = L->d;
   p.Cp = L->router_cols_pad;

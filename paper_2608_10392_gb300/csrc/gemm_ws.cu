@@ -83,8 +83,9 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
 ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                Params p) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
+  // 1024-byte aligned base, derived from smem_raw by an offset so that the
+  // compiler keeps every access through it in the shared state space
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   constexpr int kStagesA = Cfg<MODE>::kStagesA;
   constexpr int kProducerWarps = Cfg<MODE>::kProducerWarps;
   constexpr int kLoaderWarp = Cfg<MODE>::kLoaderWarp;

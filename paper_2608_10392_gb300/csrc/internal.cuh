@@ -39,10 +39,7 @@ struct Workspace {
   int32_t* row_tok = nullptr;    // [max_rows], or [G][region] when the router groups (-1 = padding)
   float* row_w = nullptr;        // same layout
   // Look-back state of the grouping inside the router (bf16 layers).
-  int32_t* lb_agg = nullptr;     // [router CTAs][G]
-  int32_t* lb_incl = nullptr;    // [router CTAs][G]
-  uint32_t* lb_flag = nullptr;   // [router CTAs]
-  int32_t* ticket = nullptr;     // [1]
+  int32_t* grp_fill = nullptr;   // [G + 1] rows reserved per group, then the ticket
   // Intermediate activations h = GeLU(x K_e[:, H_b]) per row, and the fp32
   // output accumulator.
   void* hbuf = nullptr;          // [max_rows][M] (layer dtype)
@@ -75,7 +72,6 @@ struct unif_moe_layer {
   // in its own region of region_rows rows (no separate grouping kernels).
   bool fused_group = false;
   int region_rows = 0;
-  uint32_t epoch = 0;
   int device = 0;
   bool loaded = false;
   int last_T = -1;
@@ -131,6 +127,9 @@ long long gemm_wait_limit();
 bool encode_bf16_map(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
                      uint32_t box_cols, uint32_t box_rows, int swizzle_bytes);  // clock cycles before a bounded wait gives up
 int router_tc_setup(unif_moe_layer* L);
+// Whether the tensor-core router's shared memory holds the grouping's
+// counters (and at least one tile of staged rows) for these sizes.
+bool router_can_group(int Cp, int K, int G);
 cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
                              int32_t* b_out, int32_t* k_out, cudaStream_t s);
 

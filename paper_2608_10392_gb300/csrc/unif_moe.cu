@@ -3,6 +3,7 @@
 // forward pass
 //   router (Eqs. 17-27) -> permute (groups of Eqs. 28-29) ->
 //   grouped up/down GEMMs (Eq. 16) -> combine (Eq. 30).
+#include <algorithm>
 #include <math.h>
 #include <stdarg.h>
 #include <stdio.h>
@@ -68,8 +69,8 @@ void free_all(unif_moe_layer* L) {
                   L->ws.grp_cnt, L->ws.grp_off, L->ws.n_tiles, L->ws.tile_group,
                   L->ws.tile_row0, L->ws.row_tok, L->ws.row_w, L->ws.hbuf, L->ws.y32,
                   L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
-                  L->ws.k_stage, L->ws.status, L->ws.lb_agg, L->ws.lb_incl, L->ws.lb_flag,
-                  L->ws.ticket, L->ws.tile_rows};
+                  L->ws.k_stage, L->ws.status, L->ws.grp_fill,
+                  L->ws.tile_rows};
   for (void* q : ptrs)
     if (q) cudaFree(q);
 }
@@ -187,15 +188,12 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   ALLOC(w.tile_rows, (size_t)L->max_tiles);
   // bf16 layers group inside the router: each group owns a region of
   // max_tokens rows (rounded up to whole tiles) in the row arrays
-  L->fused_group = dtype == UNIF_MOE_BF16 && L->G <= 1024;
+  L->fused_group = dtype == UNIF_MOE_BF16 && L->router_cols_pad <= 160 &&
+                   unif::router_can_group(L->router_cols_pad, L->K, L->G);
   L->region_rows = (max_tokens + 127) / 128 * 128;
   const size_t row_cap = L->fused_group ? (size_t)L->G * L->region_rows : (size_t)L->max_rows;
   ALLOC(w.row_tok, row_cap); ALLOC(w.row_w, row_cap);
-  const size_t lb_ctas = ((size_t)max_tokens + 127) / 128;
-  if (L->fused_group) {
-    ALLOC(w.lb_agg, lb_ctas * L->G); ALLOC(w.lb_incl, lb_ctas * L->G);
-    ALLOC(w.lb_flag, lb_ctas); ALLOC(w.ticket, 1);
-  }
+  if (L->fused_group) ALLOC(w.grp_fill, (size_t)L->G + 1);
   void* hb = nullptr;
   if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&hb), es * (size_t)L->max_rows * M);
   w.hbuf = hb;
@@ -205,8 +203,7 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
                             cudaMemset(w.y32, 0, sizeof(float) * T * d_model) != cudaSuccess ||
                             (L->fused_group &&
-                             (cudaMemset(w.lb_flag, 0, sizeof(uint32_t) * lb_ctas) != cudaSuccess ||
-                              cudaMemset(w.ticket, 0, sizeof(int32_t)) != cudaSuccess)))) {
+                             cudaMemset(w.grp_fill, 0, sizeof(int32_t) * (L->G + 1)) != cudaSuccess))) {
     set_error("cudaMemset failed");
     rc = UNIF_MOE_ERR_CUDA;
   }
@@ -352,8 +349,9 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
   if (L->last_T > 0) CK(cudaMemcpyAsync(&total, L->ws.grp_off + L->G, sizeof(int32_t), dh, s));
   CK(cudaStreamSynchronize(s));
   if (L->last_T > 0 && L->fused_group) {
-    // rows live in per-group regions on the device: gather them group by
-    // group into the contiguous padded layout
+    // rows live in per-group regions on the device, each group's rows in the
+    // order the router CTAs reserved them: gather them group by group into
+    // the contiguous padded layout, in token order
     std::vector<int32_t> cnt(L->G), off(L->G + 1);
     CK(cudaMemcpyAsync(cnt.data(), L->ws.grp_cnt, sizeof(int32_t) * L->G, dh, s));
     CK(cudaMemcpyAsync(off.data(), L->ws.grp_off, sizeof(int32_t) * (L->G + 1), dh, s));
@@ -368,11 +366,19 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
         if (row_token) row_token[r] = -1;
         if (row_weight) row_weight[r] = 0.f;
       }
-      if (n == 0) continue;
-      if (row_token)
-        CK(cudaMemcpyAsync(row_token + off[g], L->ws.row_tok + src, sizeof(int32_t) * n, dh, s));
-      if (row_weight)
-        CK(cudaMemcpyAsync(row_weight + off[g], L->ws.row_w + src, sizeof(float) * n, dh, s));
+      if (n == 0 || (!row_token && !row_weight)) continue;
+      std::vector<int32_t> tok(n);
+      std::vector<float> wt(n);
+      std::vector<size_t> ord(n);
+      CK(cudaMemcpyAsync(tok.data(), L->ws.row_tok + src, sizeof(int32_t) * n, dh, s));
+      CK(cudaMemcpyAsync(wt.data(), L->ws.row_w + src, sizeof(float) * n, dh, s));
+      CK(cudaStreamSynchronize(s));
+      for (size_t i = 0; i < n; ++i) ord[i] = i;
+      std::sort(ord.begin(), ord.end(), [&](size_t a, size_t b) { return tok[a] < tok[b]; });
+      for (size_t i = 0; i < n; ++i) {
+        if (row_token) row_token[off[g] + i] = tok[ord[i]];
+        if (row_weight) row_weight[off[g] + i] = wt[ord[i]];
+      }
     }
   } else if (L->last_T > 0) {
     if (counts) CK(cudaMemcpyAsync(counts, L->ws.grp_cnt, sizeof(int32_t) * L->G, dh, s));
