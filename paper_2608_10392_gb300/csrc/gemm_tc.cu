@@ -414,6 +414,8 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t0 = blockIdx.x * kBM;
   const int Cp = p.Cp, K = p.dec.K;
+  // the up projection may start its prologue on SMs this grid leaves free
+  grid_dep_launch();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kRtStages; ++s) {

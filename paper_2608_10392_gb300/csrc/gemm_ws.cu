@@ -138,6 +138,13 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // The up projection reads the router's tile list and rows: it waits for
+  // the router here. The down projection needs only the up projection's h
+  // (its tile list and rows come from the router, which completed before
+  // the up projection started), so only its h loader waits, below, and the
+  // weight slabs of its first run load meanwhile.
+  if (MODE == 0) grid_dep_wait();
+  grid_dep_launch();
 
   // This CTA's contiguous run of tiles (sizes differ by at most one).
   const int n_tiles = p.n_tiles[0];
@@ -203,6 +210,7 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
   } else if (MODE == 1 && warp == 0) {
     // ---------------- down: h tiles by TMA ---------------------------------
+    grid_dep_wait();
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
@@ -532,17 +540,15 @@ static tc::ws::Params ws_params(unif_moe_layer* L, const void* x) {
 cudaError_t launch_up_ws(unif_moe_layer* L, const void* x, cudaStream_t s) {
   tc::ws::Params p = ws_params(L, x);
   p.n_sub = L->up_nsub; p.bn = L->up_bn; p.num_kb = L->d / tc::kBK;
-  tc::ws::ws_gemm_kernel<0><<<L->n_sm, tc::ws::Cfg<0>::kThreads, L->up_ws_smem, s>>>(
-      L->tm_h_st, L->tm_wup, p);
-  return cudaGetLastError();
+  return launch_dependent(tc::ws::ws_gemm_kernel<0>, dim3(L->n_sm), dim3(tc::ws::Cfg<0>::kThreads),
+                          L->up_ws_smem, s, L->tm_h_st, L->tm_wup, p);
 }
 
 cudaError_t launch_down_ws(unif_moe_layer* L, cudaStream_t s) {
   tc::ws::Params p = ws_params(L, nullptr);
   p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
-  tc::ws::ws_gemm_kernel<1><<<L->n_sm, tc::ws::Cfg<1>::kThreads, L->down_ws_smem, s>>>(L->tm_h,
-                                                                              L->tm_wdown, p);
-  return cudaGetLastError();
+  return launch_dependent(tc::ws::ws_gemm_kernel<1>, dim3(L->n_sm), dim3(tc::ws::Cfg<1>::kThreads),
+                          L->down_ws_smem, s, L->tm_h, L->tm_wdown, p);
 }
 
 }  // namespace unif

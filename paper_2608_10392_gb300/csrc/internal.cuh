@@ -20,6 +20,35 @@ constexpr int kChunkTokens = 256;
 constexpr int kStatusTimeout = 1;
 constexpr int kStatusBadIndex = 2;
 
+// Programmatic dependent launch. The kernels of a forward after the router
+// are launched with launch_dependent: each may start (prologue: barriers,
+// tensor memory, loads that need no result of the kernel before it) while
+// the kernel before it still runs, and waits in grid_dep_wait, which
+// returns once that kernel has completed and its writes are visible. A
+// kernel lets its dependent start with grid_dep_launch. In a kernel launched
+// without the attribute grid_dep_wait returns at once.
+__device__ __forceinline__ void grid_dep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 struct Workspace {
   // Routing records of the last forward (one entry per token slot).
   float* alpha = nullptr;        // [T]

@@ -496,6 +496,7 @@ scatter_kernel(const uint64_t* __restrict__ shr_o, const uint64_t* __restrict__ 
 // the next forward: every kernel that reads them has finished.
 __global__ void cast_out_bf16(const float4* __restrict__ y, uint2* __restrict__ out, size_t n4,
                               int32_t* zero, int n_zero) {
+  grid_dep_wait();  // the down projection's sums are complete
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4;
@@ -633,9 +634,9 @@ cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s) 
   const size_t n4 = (size_t)T * L->d / 4;
   const int grid = L->n_sm * 8;
   if (L->dtype == UNIF_MOE_BF16)
-    cast_out_bf16<<<grid, 256, 0, s>>>(reinterpret_cast<const float4*>(L->ws.y32),
-                                       static_cast<uint2*>(out), n4, L->ws.grp_fill,
-                                       L->fused_group ? L->G + 1 : 0);
+    return launch_dependent(cast_out_bf16, dim3(grid), dim3(256), 0, s,
+                            reinterpret_cast<const float4*>(L->ws.y32), static_cast<uint2*>(out),
+                            n4, L->ws.grp_fill, L->fused_group ? L->G + 1 : 0);
   else
     copy_out_f32<<<grid, 256, 0, s>>>(reinterpret_cast<const float4*>(L->ws.y32),
                                       static_cast<float4*>(out), n4);
