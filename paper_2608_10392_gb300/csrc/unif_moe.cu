@@ -203,7 +203,10 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
                             cudaMemset(w.y32, 0, sizeof(float) * T * d_model) != cudaSuccess ||
                             (L->fused_group &&
-                             cudaMemset(w.grp_fill, 0, sizeof(int32_t) * (L->G + 1)) != cudaSuccess))) {
+                             (cudaMemset(w.grp_fill, 0, sizeof(int32_t) * (L->G + 1)) != cudaSuccess ||
+                              // rows hold token indices from the start, also any row a
+                              // forward that gave up a wait left unwritten
+                              cudaMemset(w.row_tok, 0, sizeof(int32_t) * row_cap) != cudaSuccess)))) {
     set_error("cudaMemset failed");
     rc = UNIF_MOE_ERR_CUDA;
   }
