@@ -33,8 +33,6 @@ if ROOT not in sys.path:
 METRIC = "UniF-MoE layer fwd tokens/s & activated TFLOP/s (% of GB300 bf16 peak), 1 GPU"
 UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# router (+ decisions, pair counts), group scan, group scatter, up GEMM, down GEMM, combine
-KERNELS_PER_FORWARD = 6
 
 
 def load_peaks():
@@ -382,7 +380,7 @@ def main():
             "value": T_valid / (statistics.fmean(e2e_ms) / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": statistics.fmean(e2e_ms)},
-        "gpu_launches": KERNELS_PER_FORWARD * K,
+        "gpu_launches": layer.kernels_per_forward() * K,
         "clocks": clocks,
     }
     if not args.no_cpu_baseline and world >= 1:

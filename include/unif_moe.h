@@ -160,6 +160,12 @@ UNIF_MOE_API int unif_moe_set_stage_events(unif_moe_t h, void* const* events);
 /* Upper bound on group-table rows (padded) of a forward at max_tokens. */
 UNIF_MOE_API int64_t unif_moe_max_rows(unif_moe_t h);
 
+/* Number of kernels one unif_moe_forward launches with T > 0 (the same for
+ * every T): 4 for bf16 layers whose router also groups the pairs (router,
+ * up projection, down projection, combine), else 6 (router, group scan,
+ * group scatter, up, down, combine). -1 for a NULL handle. */
+UNIF_MOE_API int unif_moe_kernels_per_forward(unif_moe_t h);
+
 /* Waits for `stream`, then reads and clears the handle's device status word.
  * Returns UNIF_MOE_OK, UNIF_MOE_ERR_TIMEOUT if a kernel abandoned a bounded
  * wait since the last call, or UNIF_MOE_ERR_CUDA. */

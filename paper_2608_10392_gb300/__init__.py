@@ -30,7 +30,8 @@ ERR = {0: "OK", -1: "ERR_ARG", -2: "ERR_SHAPE", -3: "ERR_CAPACITY", -4: "ERR_CUD
 # Every symbol include/unif_moe.h declares.
 EXPORTS = ["unif_moe_default_thresholds", "unif_moe_create", "unif_moe_load_weights",
            "unif_moe_forward", "unif_moe_forward_host", "unif_moe_get_routing",
-           "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_set_stage_events",
+           "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_kernels_per_forward",
+           "unif_moe_set_stage_events",
            "unif_moe_sync_status", "unif_moe_selftest_timeout", "unif_moe_group_noalloc",
            "unif_moe_destroy", "unif_moe_last_error"]
 
@@ -67,6 +68,7 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_get_groups.argtypes = [P, P, P, P, P, C.POINTER(C.c_int64), P]
         L.unif_moe_max_rows.argtypes = [P]
         L.unif_moe_max_rows.restype = C.c_int64
+        L.unif_moe_kernels_per_forward.argtypes = [P]
         L.unif_moe_set_stage_events.argtypes = [P, P]
         L.unif_moe_sync_status.argtypes = [P, P]
         L.unif_moe_selftest_timeout.argtypes = [P, I, P]
@@ -177,6 +179,9 @@ class Layer:
 
     def max_rows(self) -> int:
         return int(lib().unif_moe_max_rows(self._h))
+
+    def kernels_per_forward(self) -> int:
+        return int(lib().unif_moe_kernels_per_forward(self._h))
 
     def groups(self, stream=None):
         """Group table of the last forward (host tensors): counts [G],

@@ -399,6 +399,11 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
 
 int64_t unif_moe_max_rows(unif_moe_t L) { return L ? L->max_rows : -1; }
 
+int unif_moe_kernels_per_forward(unif_moe_t L) {
+  if (!L) return -1;
+  return L->fused_group ? 4 : 6;
+}
+
 int unif_moe_set_stage_events(unif_moe_t L, void* const* events) {
   unif::g_err[0] = 0;
   if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }

@@ -67,6 +67,7 @@ def test_argument_errors_without_gpu(lib):
     assert lib.unif_moe_load_weights(None, None, None, None, None, None) == -1
     assert lib.unif_moe_sync_status(None, None) == -1
     assert lib.unif_moe_max_rows(None) == -1
+    assert lib.unif_moe_kernels_per_forward(None) == -1
     lib.unif_moe_destroy(None)
 
 
