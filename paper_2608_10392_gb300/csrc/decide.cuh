@@ -298,7 +298,7 @@ __device__ __forceinline__ void named_bar(uint32_t id, uint32_t n) {
 
 // Shared-memory ints group_rows needs.
 __host__ __device__ constexpr int group_rows_smem_ints(int NW, int G) {
-  return NW * G + 8;
+  return NW * G + G + 8;
 }
 
 // Exclusive scan of v over the NT threads of the decision warps (thread
@@ -334,9 +334,10 @@ __device__ __forceinline__ int block_excl_scan1(int v, int tid, int lane, int w,
 // affinities s_1..s_K at dec_s[i * dec_stride + j]. `sm` has
 // group_rows_smem_ints(NW, G) ints.
 //
-// Threads take whole groups: with one warp per scheduler, per-row work must
-// be short and free of shared-memory round trips, so a thread walks its
-// group's member bits (token order) and writes the rows one after another.
+// With one warp per scheduler, per-row work must be short and free of
+// shared-memory round trips: a thread takes one (group, chunk) pair, walks
+// the chunk's member bits of the group (token order) and writes those rows
+// one after another.
 template <int NW>
 __device__ void group_rows(const GroupArgs& a, int tid, int w, int lane, int t0,
                            const uint32_t* masks, const float* dec_s, int dec_stride, int32_t* sm,
@@ -344,35 +345,45 @@ __device__ void group_rows(const GroupArgs& a, int tid, int w, int lane, int t0,
   constexpr int NT = NW * 32;
   const int G = a.G, B = a.B;
   int32_t* cnt_s = sm;                    // [NW][G] chunk counts
-  int32_t* misc_s = cnt_s + NW * G;       // [8]: ticket flag, scan scratch (1..NW)
+  int32_t* base_s = cnt_s + NW * G;       // [G] first reserved row, or -1
+  int32_t* misc_s = base_s + G;           // [8]: ticket flag, scan scratch (1..NW)
+  // 1. this CTA's rows of each group, reserved in the group's region
   for (int g = tid; g < G; g += NT) {
-    // 1. this CTA's rows of group g, reserved in the group's region
     int n = 0;
 #pragma unroll
     for (int v = 0; v < NW; ++v) n += cnt_s[v * G + g];
-    if (n == 0) continue;
-    int base = atomicAdd(a.fill + g, n);
-    if (base + n > a.region) {  // stale counters: keep the writes inside the region
-      atomicOr(a.status, kStatusBadIndex);
-      continue;
+    int base = -1;
+    if (n > 0) {
+      base = atomicAdd(a.fill + g, n);
+      if (base + n > a.region) {  // stale counters: keep the writes inside the region
+        atomicOr(a.status, kStatusBadIndex);
+        base = -1;
+      }
     }
-    // 2. the rows, in token order
+    base_s[g] = base;
+  }
+  named_bar(bar, NT);
+  // 2. the rows, in token order: a thread takes the rows of one group from
+  // one 32-token chunk (after the rows of the group's earlier chunks)
+  for (int idx = tid; idx < G * NW; idx += NT) {
+    const int g = idx / NW, c = idx - g * NW;
+    const int base = base_s[g];
+    if (base < 0) continue;
+    int off = 0;
+#pragma unroll
+    for (int v = 0; v < NW; ++v) off += v < c ? cnt_s[v * G + g] : 0;
     const int e = g / B, blk = g - e * B;
     const int wcol = e == 0 ? 2 * a.K : e - 1;
-    int32_t* tok = a.row_tok + (size_t)g * a.region + base;
-    float* wt = a.row_w + (size_t)g * a.region + base;
-    int r = 0;
-#pragma unroll
-    for (int c = 0; c < NW; ++c) {
-      const uint32_t sh = masks[c * 128 + blk];
-      uint32_t m = e == 0 ? sh : (masks[c * 128 + 64 + e - 1] & ~sh);
-      while (m != 0u && r < n) {
-        const int i = c * 32 + __ffs(m) - 1;
-        m &= m - 1u;
-        tok[r] = t0 + i;
-        wt[r] = dec_s[i * dec_stride + wcol];
-        ++r;
-      }
+    const size_t r0 = (size_t)g * a.region + base + off;
+    int32_t* tok = a.row_tok + r0;
+    float* wt = a.row_w + r0;
+    const uint32_t sh = masks[c * 128 + blk];
+    uint32_t m = e == 0 ? sh : (masks[c * 128 + 64 + e - 1] & ~sh);
+    for (int r = 0; m != 0u; ++r) {
+      const int i = c * 32 + __ffs(m) - 1;
+      m &= m - 1u;
+      tok[r] = t0 + i;
+      wt[r] = dec_s[i * dec_stride + wcol];
     }
   }
   // 3. the CTA that finishes last numbers the tiles

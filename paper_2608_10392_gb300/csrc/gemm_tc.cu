@@ -390,7 +390,6 @@ struct RouterTcParams {
   int fused;     // 1: the router also lays out the group rows (group_rows)
   int d, Cp;
   uint32_t tmem_cols;
-  float* y32;
   int* status;
   long long wait_limit;
 };
@@ -474,14 +473,6 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     __syncwarp();
   } else {
     // decision warps: lane quarter q = warp % 4 holds tokens t0 + 32 q + lane.
-    // While the MMAs run they zero the output accumulator rows of these tokens.
-    {
-      const int rows = min(kBM, p.dec.T - t0);
-      float4* yz = reinterpret_cast<float4*>(p.y32 + (size_t)t0 * p.d);
-      const int n4 = rows * p.d / 4;
-      for (int i = threadIdx.x - 64; i < n4; i += kRtThreads - 64)
-        yz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
     const int q = warp & 3;
     const int row = q * 32 + lane;
     // logits and affinities overlay the (now idle) operand ring
@@ -709,7 +700,6 @@ cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* ma
   p.d = L->d;
   p.Cp = L->router_cols_pad;
   p.tmem_cols = p.Cp <= 32 ? 32u : (p.Cp <= 64 ? 64u : (p.Cp <= 128 ? 128u : 256u));
-  p.y32 = L->ws.y32;
   p.status = L->ws.status;
   p.wait_limit = tc::g_wait_limit;
   tc::router_tc_kernel<<<(T + tc::kBM - 1) / tc::kBM, tc::kRtThreads, tc::kRtSmem, s>>>(

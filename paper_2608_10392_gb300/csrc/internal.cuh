@@ -103,6 +103,7 @@ struct unif_moe_layer {
   int region_rows = 0;
   int device = 0;
   bool loaded = false;
+  bool y_dirty = false;  // the output accumulator may hold sums of a forward cut short
   int last_T = -1;
   // Weights (device, owned).
   float* wr = nullptr;      // [d][router_cols_pad]: W_shr, W_g, mu_1..mu_B (fp32)

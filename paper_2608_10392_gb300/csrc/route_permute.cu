@@ -83,7 +83,6 @@ struct RouterArgs {
   DecideArgs dec;
   int d;
   const float* wr;  // [d][Cp] router matrix
-  float* y32;       // [T][d] output accumulator, zeroed here
 };
 
 __device__ __forceinline__ void load8(const float* src, float (&v)[8]) {
@@ -121,14 +120,6 @@ router_kernel(const Tin* __restrict__ x, RouterArgs a) {
 
   // ---- z = x W for 64 tokens x Cp columns (Eqs. 17, 21) ----
   const int ty = tid >> 4, tx = tid & 15;  // tokens 4ty..4ty+3, columns tx + 16 j
-  // The fp32 output accumulator rows of these 64 tokens start at zero (the
-  // down-projection adds into them).
-  {
-    const int rows = min(kRouterTokens, a.dec.T - t0);
-    float4* yz = reinterpret_cast<float4*>(a.y32 + (size_t)t0 * a.d);
-    const int n4 = rows * a.d / 4;
-    for (int i = tid; i < n4; i += kRouterThreads) yz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-  }
   float acc[4][2 * NCB];
 #pragma unroll
   for (int i = 0; i < 4; ++i)
@@ -492,29 +483,46 @@ scatter_kernel(const uint64_t* __restrict__ shr_o, const uint64_t* __restrict__ 
 // Combine: y (fp32 accumulator) -> output dtype
 // ---------------------------------------------------------------------------
 
-// Also zeroes the router's group fill and ticket counters (n_zero ints) for
-// the next forward: every kernel that reads them has finished.
-__global__ void cast_out_bf16(const float4* __restrict__ y, uint2* __restrict__ out, size_t n4,
+// The fp32 accumulator is all zero between forwards: each combine zeroes
+// the rows it reads (the down projection of the next forward adds into
+// them). Also zeroes the router's group fill and ticket counters (n_zero
+// ints) for the next forward: every kernel that reads them has finished.
+__global__ void cast_out_bf16(float4* __restrict__ y, uint2* __restrict__ out, size_t n4,
                               int32_t* zero, int n_zero) {
   grid_dep_wait();  // the down projection's sums are complete
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
-  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4;
-       i += (size_t)gridDim.x * blockDim.x) {
-    const float4 v = y[i];
-    __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y);
-    __nv_bfloat162 hi = __floats2bfloat162_rn(v.z, v.w);
-    uint2 o;
-    o.x = *reinterpret_cast<unsigned*>(&lo);
-    o.y = *reinterpret_cast<unsigned*>(&hi);
-    out[i] = o;
+  // four elements per thread and round: all loads first, then the stores
+  constexpr int kU = 4;
+  const size_t stride = (size_t)gridDim.x * blockDim.x;
+  for (size_t i0 = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i0 < n4; i0 += kU * stride) {
+    float4 v[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const size_t i = i0 + u * stride;
+      v[u] = i < n4 ? y[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const size_t i = i0 + u * stride;
+      if (i >= n4) break;
+      __nv_bfloat162 lo = __floats2bfloat162_rn(v[u].x, v[u].y);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(v[u].z, v[u].w);
+      uint2 o;
+      o.x = *reinterpret_cast<unsigned*>(&lo);
+      o.y = *reinterpret_cast<unsigned*>(&hi);
+      out[i] = o;
+      y[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
   }
 }
 
-__global__ void copy_out_f32(const float4* __restrict__ y, float4* __restrict__ out, size_t n4) {
+__global__ void copy_out_f32(float4* __restrict__ y, float4* __restrict__ out, size_t n4) {
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4;
-       i += (size_t)gridDim.x * blockDim.x)
+       i += (size_t)gridDim.x * blockDim.x) {
     out[i] = y[i];
+    y[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
 }
 
 }  // namespace
@@ -594,7 +602,6 @@ cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask,
   a.dec = decide_args(L, mask, T, b_out, k_out);
   a.d = L->d;
   a.wr = L->wr;
-  a.y32 = L->ws.y32;
   const void* xp = x;
   void* args[] = {const_cast<void**>(&xp), &a};
   const int grid = (T + kRouterTokens - 1) / kRouterTokens;
@@ -635,10 +642,10 @@ cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s) 
   const int grid = L->n_sm * 8;
   if (L->dtype == UNIF_MOE_BF16)
     return launch_dependent(cast_out_bf16, dim3(grid), dim3(256), 0, s,
-                            reinterpret_cast<const float4*>(L->ws.y32), static_cast<uint2*>(out),
+                            reinterpret_cast<float4*>(L->ws.y32), static_cast<uint2*>(out),
                             n4, L->ws.grp_fill, L->fused_group ? L->G + 1 : 0);
   else
-    copy_out_f32<<<grid, 256, 0, s>>>(reinterpret_cast<const float4*>(L->ws.y32),
+    copy_out_f32<<<grid, 256, 0, s>>>(reinterpret_cast<float4*>(L->ws.y32),
                                       static_cast<float4*>(out), n4);
   return cudaGetLastError();
 }

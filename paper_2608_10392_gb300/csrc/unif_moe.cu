@@ -262,6 +262,12 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
   DeviceGuard dg(L->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = L->stage_ev;
+  // The output accumulator is all zero between forwards (each combine zeroes
+  // the rows it reads). A forward that returned before launching its
+  // combine leaves it dirty: clear it all first.
+  if (L->y_dirty)
+    CK(cudaMemsetAsync(L->ws.y32, 0, sizeof(float) * (size_t)L->max_tokens * L->d, s));
+  L->y_dirty = true;
   if (ev[0]) CK(cudaEventRecord(ev[0], s));
   if (L->dtype == UNIF_MOE_BF16) {
     CK(unif::launch_router_tc(L, x, token_mask, T, shared_counts, residual_counts, s));
@@ -278,6 +284,7 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
   }
   if (ev[4]) CK(cudaEventRecord(ev[4], s));
   CK(unif::launch_combine(L, out, T, s));
+  L->y_dirty = false;
   if (ev[5]) CK(cudaEventRecord(ev[5], s));
   L->last_T = T;
   return UNIF_MOE_OK;
