@@ -269,26 +269,19 @@ __device__ __forceinline__ void count_chunk_pairs(const DecideArgs& a, int lane,
 // row_tok / row_w. A router CTA reserves its rows of every group with one
 // atomic add on the group's fill counter, so rows of different CTAs land in
 // arrival order (within a CTA, in token order); nothing downstream depends
-// on the order of a group's rows. The CTA that finishes last (a ticket
-// counter) reads the final fills, the group sizes, and numbers the tiles
-// (128 rows) of every group into the tile list, with each tile's count of
-// real rows (the rest of a group's last tile is padding, which the GEMM
-// kernels skip). The combine kernel zeroes the fill and ticket counters for
-// the next forward, also after a forward whose router gave up a wait.
+// on the order of a group's rows. Once the router grid has completed, the
+// fill counters are the group sizes: the GEMM kernels number the 128-row
+// tiles of every group from them (tile_table below), each tile with its
+// count of real rows (the rest of a group's last tile is padding, which
+// they skip). The combine kernel copies the sizes out for the group table
+// and zeroes the counters for the next forward, also after a forward whose
+// router gave up a wait.
 struct GroupArgs {
   int G, K, B;
-  int n_ctas;
   int region;
   int32_t* fill;           // [G] rows reserved so far (0 at the start of a forward)
-  int32_t* ticket;         // [1] CTAs done (0 at the start of a forward)
   int32_t* row_tok;
   float* row_w;
-  int32_t* grp_cnt;
-  int32_t* grp_off;        // padded offsets as if the groups were contiguous
-  int32_t* n_tiles;
-  int32_t* tile_group;
-  int32_t* tile_row0;
-  int32_t* tile_rows;
   int* status;
 };
 
@@ -298,31 +291,7 @@ __device__ __forceinline__ void named_bar(uint32_t id, uint32_t n) {
 
 // Shared-memory ints group_rows needs.
 __host__ __device__ constexpr int group_rows_smem_ints(int NW, int G) {
-  return NW * G + G + 8;
-}
-
-// Exclusive scan of v over the NT threads of the decision warps (thread
-// order); returns the scan and sets total. warp_s holds NW ints.
-template <int NW>
-__device__ __forceinline__ int block_excl_scan1(int v, int tid, int lane, int w, int32_t* warp_s,
-                                                uint32_t bar, int& total) {
-  int inc = v;
-  for (int o = 1; o < 32; o <<= 1) {
-    const int n = __shfl_up_sync(0xffffffffu, inc, o);
-    if (lane >= o) inc += n;
-  }
-  if (lane == 31) warp_s[w] = inc;
-  named_bar(bar, NW * 32);
-  int before = 0;
-  total = 0;
-#pragma unroll
-  for (int u = 0; u < NW; ++u) {
-    const int s = warp_s[u];
-    before += u < w ? s : 0;
-    total += s;
-  }
-  named_bar(bar, NW * 32);
-  return before + inc - v;
+  return NW * G + G + 8;  // chunk counts, bases, misc
 }
 
 // Runs in the NW decision warps of a router CTA (threads tid = 0 .. NW*32-1,
@@ -346,7 +315,6 @@ __device__ void group_rows(const GroupArgs& a, int tid, int w, int lane, int t0,
   const int G = a.G, B = a.B;
   int32_t* cnt_s = sm;                    // [NW][G] chunk counts
   int32_t* base_s = cnt_s + NW * G;       // [G] first reserved row, or -1
-  int32_t* misc_s = base_s + G;           // [8]: ticket flag, scan scratch (1..NW)
   // 1. this CTA's rows of each group, reserved in the group's region
   for (int g = tid; g < G; g += NT) {
     int n = 0;
@@ -386,35 +354,44 @@ __device__ void group_rows(const GroupArgs& a, int tid, int w, int lane, int t0,
       wt[r] = dec_s[i * dec_stride + wcol];
     }
   }
-  // 3. the CTA that finishes last numbers the tiles
-  __threadfence();
-  named_bar(bar, NT);
-  if (tid == 0) misc_s[0] = atomicAdd(a.ticket, 1) == a.n_ctas - 1;
-  named_bar(bar, NT);
-  if (!misc_s[0]) return;
-  __threadfence();
+}
+
+// The tiles of the groups whose sizes are fill[0..G) (each clamped to the
+// region): first_s[g] = first tile of group g (first_s[G] = all tiles),
+// cnt_s[g] = its size. Run by one warp; shared arrays of G + 1 and G ints.
+__device__ __forceinline__ void tile_table(const int32_t* fill, int G, int region, int lane,
+                                           int32_t* first_s, int32_t* cnt_s) {
   int carry = 0;
-  for (int g0 = 0; g0 < G; g0 += NT) {
-    const int g = g0 + tid;
-    const int tot = g < G ? min(__ldcg(a.fill + g), a.region) : 0;
-    const int nt = (tot + 127) / 128;
-    int total;
-    const int k0 = carry + block_excl_scan1<NW>(nt, tid, lane, w, misc_s + 1, bar, total);
-    carry += total;
-    if (g < G) {
-      a.grp_cnt[g] = tot;
-      a.grp_off[g] = k0 * 128;
-      for (int i = 0; i < nt; ++i) {
-        a.tile_group[k0 + i] = g;
-        a.tile_row0[k0 + i] = g * a.region + 128 * i;
-        a.tile_rows[k0 + i] = min(128, tot - 128 * i);
-      }
+  for (int g0 = 0; g0 < G; g0 += 32) {
+    const int g = g0 + lane;
+    const int c = g < G ? min(__ldcg(fill + g), region) : 0;
+    const int nt = (c + 127) / 128;
+    int inc = nt;
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += v;
     }
+    if (g < G) {
+      first_s[g] = carry + inc - nt;
+      cnt_s[g] = c;
+    }
+    carry += __shfl_sync(0xffffffffu, inc, 31);
   }
-  if (tid == 0) {
-    a.n_tiles[0] = carry;
-    a.grp_off[G] = carry * 128;
+  if (lane == 0) first_s[G] = carry;
+}
+
+// Group, first row and real rows of tile k, from tile_table's arrays.
+__device__ __forceinline__ void tile_lookup(int k, const int32_t* first_s, const int32_t* cnt_s,
+                                            int G, int region, int& g, int& row0, int& rows) {
+  int lo = 0, hi = G - 1;  // the last group whose first tile is <= k
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (first_s[mid] <= k) lo = mid; else hi = mid - 1;
   }
+  const int i = k - first_s[lo];
+  g = lo;
+  row0 = lo * region + 128 * i;
+  rows = min(128, cnt_s[lo] - 128 * i);
 }
 
 DecideArgs decide_args(unif_moe_layer* L, const uint8_t* mask, int T, int32_t* b_out,

@@ -620,7 +620,9 @@ int gemm_tc_setup(unif_moe_layer* L) {
     set_error("cudaFuncSetAttribute: %s", cudaGetErrorString(e));
     return UNIF_MOE_ERR_CUDA;
   }
-  return gemm_ws_setup(L);
+  const int rc = gemm_ws_setup(L);
+  L->tile_list = L->fused_group && !(L->up_ws && L->down_ws);
+  return rc;
 }
 
 cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
@@ -689,12 +691,9 @@ cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* ma
     Workspace& w = L->ws;
     GroupArgs& g = p.grp;
     g.G = L->G; g.K = L->K; g.B = L->B;
-    g.n_ctas = (T + tc::kBM - 1) / tc::kBM;
     g.region = L->region_rows;
-    g.fill = w.grp_fill; g.ticket = w.grp_fill + L->G;
+    g.fill = w.grp_fill;
     g.row_tok = w.row_tok; g.row_w = w.row_w;
-    g.grp_cnt = w.grp_cnt; g.grp_off = w.grp_off; g.n_tiles = w.n_tiles;
-    g.tile_group = w.tile_group; g.tile_row0 = w.tile_row0; g.tile_rows = w.tile_rows;
     g.status = w.status;
   }
   p.d = L->d;

@@ -26,6 +26,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include "decide.cuh"
 #include "internal.cuh"
 #include "tc_common.cuh"
 
@@ -63,6 +64,12 @@ struct Cfg {
 };
 
 struct Params {
+  // Tiles: numbered here from the group sizes (fill != nullptr: per-group
+  // regions of `region` rows, the router's grouping), or the tile list of
+  // the grouping kernels.
+  const int32_t* fill;
+  int G, region;
+  int per_cta;  // room for this many tiles of a CTA's run in the shared tile table
   const int32_t* n_tiles;
   const int32_t* tile_group;
   const int32_t* tile_row0;  // first row of each tile in row_tok / row_w
@@ -107,6 +114,11 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   auto acce = [&](int a) { return bar0 + 8u * (12 + 2 * kMaxSlabs + a); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 14 + 2 * kMaxSlabs);
   static_assert(8 * (14 + 2 * kMaxSlabs) + 8 <= kBarBytes, "barrier region");
+  // tile table (fill != nullptr): first tile and size of every group, then
+  // the group, first row and real rows of each tile of this CTA's run
+  int32_t* first_s = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(bars) + kBarBytes);
+  int32_t* gcnt_s = first_s + p.G + 1;
+  int32_t* run_s = gcnt_s + p.G;  // [3][per_cta]
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -134,6 +146,23 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
   }
+  if (p.fill && warp == Cfg<MODE>::kThreads / 32 - 1) {
+    // the group sizes are final once the router completed: the up
+    // projection waits for it here (the down projection starts after it)
+    if (MODE == 0) grid_dep_wait();
+    tile_table(p.fill, p.G, p.region, lane, first_s, gcnt_s);
+    __syncwarp();
+    const int nt = first_s[p.G];
+    const int tb = (int)(((long long)blockIdx.x * nt) / gridDim.x);
+    const int te = (int)(((long long)(blockIdx.x + 1) * nt) / gridDim.x);
+    for (int k = tb + lane; k < te; k += 32) {
+      int g, r0, rows;
+      tile_lookup(k, first_s, gcnt_s, p.G, p.region, g, r0, rows);
+      run_s[k - tb] = g;
+      run_s[p.per_cta + k - tb] = r0;
+      run_s[2 * p.per_cta + k - tb] = rows;
+    }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -147,9 +176,22 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   grid_dep_launch();
 
   // This CTA's contiguous run of tiles (sizes differ by at most one).
-  const int n_tiles = p.n_tiles[0];
+  const int n_tiles = p.fill ? first_s[p.G] : p.n_tiles[0];
   const int t_begin = (int)(((long long)blockIdx.x * n_tiles) / gridDim.x);
   const int t_end = (int)(((long long)(blockIdx.x + 1) * n_tiles) / gridDim.x);
+  // group, first row and real rows of tile k (t_begin <= k < t_end)
+  auto tile_of = [&](int k, int& g, int& r0, int& rows) {
+    if (p.fill) {
+      const int j = k - t_begin;
+      g = run_s[j];
+      r0 = run_s[p.per_cta + j];
+      rows = run_s[2 * p.per_cta + j];
+    } else {
+      g = p.tile_group[k];
+      r0 = p.tile_row0[k];
+      rows = p.tile_rows[k];
+    }
+  };
 
   if (MODE == 0 && warp < kProducerWarps) {
     // ---------------- up: A stage owners (x rows gathered) -----------------
@@ -165,21 +207,18 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // index two tiles ahead)
     // (padding rows gather token 0; their h rows are never used)
     int tk_nxt[4];
-    int r0_nxt = t_begin + 1 < t_end ? p.tile_row0[t_begin + 1] : 0;
-    int n_nxt = t_begin + 1 < t_end ? p.tile_rows[t_begin + 1] : 0;
+    int gq, r0_nxt = 0, n_nxt = 0;
+    if (t_begin + 1 < t_end) tile_of(t_begin + 1, gq, r0_nxt, n_nxt);
     {
-      const int r0 = t_begin < t_end ? p.tile_row0[t_begin] : 0;
-      const int n = t_begin < t_end ? p.tile_rows[t_begin] : 0;
+      int r0 = 0, n = 0;
+      if (t_begin < t_end) tile_of(t_begin, gq, r0, n);
 #pragma unroll
       for (int i = 0; i < 4; ++i) tk_nxt[i] = 32 * i + lane < n ? p.row_tok[r0 + 32 * i + lane] : 0;
     }
     for (int tile = t_begin; tile < t_end && ok; ++tile, seq += p.num_kb) {
       int tk[4];
       const int r0n = r0_nxt, nn = n_nxt;
-      if (tile + 2 < t_end) {
-        r0_nxt = p.tile_row0[tile + 2];
-        n_nxt = p.tile_rows[tile + 2];
-      }
+      if (tile + 2 < t_end) tile_of(tile + 2, gq, r0_nxt, n_nxt);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         tk[i] = tk_nxt[i] < 0 ? 0 : tk_nxt[i];
@@ -236,7 +275,8 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       int run = 0, g_prev = -1;
       bool ok = true;
       for (int tile = t_begin; tile < t_end && ok; ++tile) {
-        const int g = p.tile_group[tile];
+        int g, r0_unused, rows_unused;
+        tile_of(tile, g, r0_unused, rows_unused);
         if (g == g_prev) continue;
         g_prev = g;
         const int e = g / p.B, blk = g % p.B;
@@ -287,12 +327,13 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     bool ok = true;
     bool ready = false;  // fullA(stage) known complete
     // groups of this tile and the next, loaded ahead of use
-    int g_cur = t_begin < t_end ? p.tile_group[t_begin] : -1;
-    int g_nxt = t_begin + 1 < t_end ? p.tile_group[t_begin + 1] : -1;
+    int g_cur = -1, g_nxt = -1, r0_unused, rows_unused;
+    if (t_begin < t_end) tile_of(t_begin, g_cur, r0_unused, rows_unused);
+    if (t_begin + 1 < t_end) tile_of(t_begin + 1, g_nxt, r0_unused, rows_unused);
     for (int tile = t_begin; tile < t_end && ok; ++tile) {
       const int g = g_cur, gn = g_nxt;
       g_cur = g_nxt;
-      if (tile + 2 < t_end) g_nxt = p.tile_group[tile + 2];
+      if (tile + 2 < t_end) tile_of(tile + 2, g_nxt, r0_unused, rows_unused);
       const bool first_of_run = g != g_prev;
       if (first_of_run) { ++run; g_prev = g; }
       // release the slabs after this tile if the next tile of the run
@@ -379,12 +420,15 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // tile ahead
     int t_nxt = -1;
     float w_nxt = 0.f;
-    int r0_nxt = (MODE == 1 && t_begin + 1 < t_end) ? p.tile_row0[t_begin + 1] : 0;
-    int n_nxt = (MODE == 1 && t_begin + 1 < t_end) ? p.tile_rows[t_begin + 1] : 0;
-    if (MODE == 1 && t_begin < t_end && q * 32 + lane < p.tile_rows[t_begin]) {
-      const int r = p.tile_row0[t_begin] + q * 32 + lane;
-      t_nxt = p.row_tok[r];
-      w_nxt = p.row_w[r];
+    int gq, r0_nxt = 0, n_nxt = 0;
+    if (MODE == 1 && t_begin + 1 < t_end) tile_of(t_begin + 1, gq, r0_nxt, n_nxt);
+    if (MODE == 1 && t_begin < t_end) {
+      int r0, n;
+      tile_of(t_begin, gq, r0, n);
+      if (q * 32 + lane < n) {
+        t_nxt = p.row_tok[r0 + q * 32 + lane];
+        w_nxt = p.row_w[r0 + q * 32 + lane];
+      }
     }
     uint8_t* stg = staging + (size_t)(warp - kFirstEpiWarp) * 32 * Cfg<MODE>::kStageRowBytes;
     const uint32_t stg_s = smem_u32(stg);
@@ -397,10 +441,7 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const int r = r0_nxt + q * 32 + lane;
         t_nxt = q * 32 + lane < n_nxt ? p.row_tok[r] : -1;
         w_nxt = q * 32 + lane < n_nxt ? p.row_w[r] : 0.f;
-        if (tile + 2 < t_end) {
-          r0_nxt = p.tile_row0[tile + 2];
-          n_nxt = p.tile_rows[tile + 2];
-        }
+        if (tile + 2 < t_end) tile_of(tile + 2, gq, r0_nxt, n_nxt);
       }
       for (int ns = 0; ns < p.n_sub; ++ns) {
         if (!wait_warp(accf(acc), acc_phase, abort_flag, p.status, p.wait_limit)) {
@@ -494,8 +535,14 @@ int gemm_ws_setup(unif_moe_layer* L) {
   L->up_ws = L->down_ws = false;
   const char* env = getenv("UNIF_MOE_GEMM_KERNELS");
   if (env && strcmp(env, "streaming") == 0) return UNIF_MOE_OK;
+  // the tile table (first tile and size of every group, the tiles of one
+  // CTA's run) follows the barriers
+  const uint64_t per_cta = (uint64_t)((L->max_tiles + L->n_sm - 1) / L->n_sm);
+  const uint64_t table =
+      L->fused_group ? ((uint64_t)(2 * L->G + 1 + 3 * per_cta) * 4 + 15) / 16 * 16 : 0;
   const uint64_t up_slabs = (uint64_t)L->up_nsub * (L->d / tc::kBK);
-  const uint64_t up_smem = Cfg<0>::kFixed + up_slabs * (uint64_t)L->up_bn * tc::kBK * 2;
+  const uint64_t up_smem =
+      Cfg<0>::kFixed + up_slabs * (uint64_t)L->up_bn * tc::kBK * 2 + table;
   if (L->up_nsub == 1 && up_slabs <= (uint64_t)kMaxSlabs && up_smem <= kMaxSmem) {
     if (cudaFuncSetAttribute(ws_gemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)up_smem) != cudaSuccess) {
@@ -511,7 +558,8 @@ int gemm_ws_setup(unif_moe_layer* L) {
   }
   const int down_kb = L->M / tc::kBK;
   const uint64_t down_slabs = (uint64_t)L->down_nsub * down_kb;
-  const uint64_t down_smem = Cfg<1>::kFixed + down_slabs * (uint64_t)L->down_bn * tc::kBK * 2;
+  const uint64_t down_smem =
+      Cfg<1>::kFixed + down_slabs * (uint64_t)L->down_bn * tc::kBK * 2 + table;
   if (down_kb <= Cfg<1>::kStagesA && down_slabs <= (uint64_t)kMaxSlabs && down_smem <= kMaxSmem) {
     if (cudaFuncSetAttribute(ws_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)down_smem) != cudaSuccess) {
@@ -526,6 +574,10 @@ int gemm_ws_setup(unif_moe_layer* L) {
 
 static tc::ws::Params ws_params(unif_moe_layer* L, const void* x) {
   tc::ws::Params p;
+  p.fill = L->fused_group ? L->ws.grp_fill : nullptr;
+  p.G = L->G;
+  p.region = L->region_rows;
+  p.per_cta = (int)((L->max_tiles + L->n_sm - 1) / L->n_sm);
   p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group; p.tile_row0 = L->ws.tile_row0;
   p.tile_rows = L->ws.tile_rows; p.row_tok = L->ws.row_tok; p.row_w = L->ws.row_w;
   p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;

@@ -68,7 +68,7 @@ struct Workspace {
   int32_t* row_tok = nullptr;    // [max_rows], or [G][region] when the router groups (-1 = padding)
   float* row_w = nullptr;        // same layout
   // Look-back state of the grouping inside the router (bf16 layers).
-  int32_t* grp_fill = nullptr;   // [G + 1] rows reserved per group, then the ticket
+  int32_t* grp_fill = nullptr;   // [G] rows reserved per group (the group sizes once the router completed)
   // Intermediate activations h = GeLU(x K_e[:, H_b]) per row, and the fp32
   // output accumulator.
   void* hbuf = nullptr;          // [max_rows][M] (layer dtype)
@@ -101,6 +101,7 @@ struct unif_moe_layer {
   // in its own region of region_rows rows (no separate grouping kernels).
   bool fused_group = false;
   int region_rows = 0;
+  bool tile_list = false;  // a streaming GEMM reads the tile list: build it after the router
   int device = 0;
   bool loaded = false;
   bool y_dirty = false;  // the output accumulator may hold sums of a forward cut short
@@ -139,6 +140,8 @@ cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask,
                           int32_t* b_out, int32_t* k_out, cudaStream_t s);
 cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s);
 cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s);
+// Tile list from the router's group sizes, for streaming grouped GEMMs.
+cudaError_t launch_tile_list(unif_moe_layer* L, cudaStream_t s);
 cudaError_t launch_sort_affinities(unif_moe_layer* L, int T, int32_t* q, float* p,
                                    cudaStream_t s);
 int forward_chunks(int T);

@@ -480,18 +480,44 @@ scatter_kernel(const uint64_t* __restrict__ shr_o, const uint64_t* __restrict__ 
 }
 
 // ---------------------------------------------------------------------------
+// Tile list from the router's group sizes (bf16 layers that group inside the
+// router, when a streaming grouped GEMM reads the list; the weight-stationary
+// kernels number their tiles themselves)
+// ---------------------------------------------------------------------------
+__global__ void tile_list_kernel(const int32_t* __restrict__ fill, int G, int region,
+                                 int32_t* __restrict__ n_tiles, int32_t* __restrict__ tile_group,
+                                 int32_t* __restrict__ tile_row0, int32_t* __restrict__ tile_rows) {
+  extern __shared__ int32_t tl_s[];  // [G + 1] first tiles, [G] sizes
+  if (threadIdx.x < 32) tile_table(fill, G, region, threadIdx.x, tl_s, tl_s + G + 1);
+  __syncthreads();
+  const int nt = tl_s[G];
+  if (threadIdx.x == 0) n_tiles[0] = nt;
+  for (int k = threadIdx.x; k < nt; k += blockDim.x) {
+    int g, r0, rows;
+    tile_lookup(k, tl_s, tl_s + G + 1, G, region, g, r0, rows);
+    tile_group[k] = g;
+    tile_row0[k] = r0;
+    tile_rows[k] = rows;
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Combine: y (fp32 accumulator) -> output dtype
 // ---------------------------------------------------------------------------
 
 // The fp32 accumulator is all zero between forwards: each combine zeroes
 // the rows it reads (the down projection of the next forward adds into
-// them). Also zeroes the router's group fill and ticket counters (n_zero
-// ints) for the next forward: every kernel that reads them has finished.
+// them). Also copies the router's group fill counters (n_fill ints, the
+// group sizes) to the group table's counts and zeroes them for the next
+// forward: every kernel that reads them has finished.
 __global__ void cast_out_bf16(float4* __restrict__ y, uint2* __restrict__ out, size_t n4,
-                              int32_t* zero, int n_zero) {
+                              int32_t* fill, int32_t* counts, int n_fill, int region) {
   grid_dep_wait();  // the down projection's sums are complete
   if (blockIdx.x == 0)
-    for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
+    for (int i = threadIdx.x; i < n_fill; i += blockDim.x) {
+      counts[i] = min(fill[i], region);
+      fill[i] = 0;
+    }
   // four elements per thread and round: all loads first, then the stores
   constexpr int kU = 4;
   const size_t stride = (size_t)gridDim.x * blockDim.x;
@@ -637,13 +663,21 @@ cudaError_t launch_sort_affinities(unif_moe_layer* L, int T, int32_t* q, float* 
   return cudaGetLastError();
 }
 
+cudaError_t launch_tile_list(unif_moe_layer* L, cudaStream_t s) {
+  Workspace& w = L->ws;
+  tile_list_kernel<<<1, 256, sizeof(int32_t) * (2 * (size_t)L->G + 1), s>>>(
+      w.grp_fill, L->G, L->region_rows, w.n_tiles, w.tile_group, w.tile_row0, w.tile_rows);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s) {
   const size_t n4 = (size_t)T * L->d / 4;
   const int grid = L->n_sm * 8;
   if (L->dtype == UNIF_MOE_BF16)
     return launch_dependent(cast_out_bf16, dim3(grid), dim3(256), 0, s,
                             reinterpret_cast<float4*>(L->ws.y32), static_cast<uint2*>(out),
-                            n4, L->ws.grp_fill, L->fused_group ? L->G + 1 : 0);
+                            n4, L->ws.grp_fill, L->ws.grp_cnt, L->fused_group ? L->G : 0,
+                            L->region_rows);
   else
     copy_out_f32<<<grid, 256, 0, s>>>(reinterpret_cast<float4*>(L->ws.y32),
                                       static_cast<float4*>(out), n4);

@@ -193,7 +193,7 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   L->region_rows = (max_tokens + 127) / 128 * 128;
   const size_t row_cap = L->fused_group ? (size_t)L->G * L->region_rows : (size_t)L->max_rows;
   ALLOC(w.row_tok, row_cap); ALLOC(w.row_w, row_cap);
-  if (L->fused_group) ALLOC(w.grp_fill, (size_t)L->G + 1);
+  if (L->fused_group) ALLOC(w.grp_fill, (size_t)L->G);
   void* hb = nullptr;
   if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&hb), es * (size_t)L->max_rows * M);
   w.hbuf = hb;
@@ -203,7 +203,7 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
                             cudaMemset(w.y32, 0, sizeof(float) * T * d_model) != cudaSuccess ||
                             (L->fused_group &&
-                             (cudaMemset(w.grp_fill, 0, sizeof(int32_t) * (L->G + 1)) != cudaSuccess ||
+                             (cudaMemset(w.grp_fill, 0, sizeof(int32_t) * L->G) != cudaSuccess ||
                               // rows hold token indices from the start, also any row a
                               // forward that gave up a wait left unwritten
                               cudaMemset(w.row_tok, 0, sizeof(int32_t) * row_cap) != cudaSuccess)))) {
@@ -276,6 +276,7 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
   }
   if (ev[1]) CK(cudaEventRecord(ev[1], s));
   if (!L->fused_group) CK(unif::launch_permute(L, T, s));
+  else if (L->tile_list) CK(unif::launch_tile_list(L, s));
   if (ev[2]) CK(cudaEventRecord(ev[2], s));
   if (L->dtype == UNIF_MOE_BF16) {
     CK(unif::launch_gemms_tc(L, x, T, ev[3], s));
@@ -356,16 +357,21 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const cudaMemcpyKind dh = cudaMemcpyDeviceToHost;
   int32_t total = 0;
-  if (L->last_T > 0) CK(cudaMemcpyAsync(&total, L->ws.grp_off + L->G, sizeof(int32_t), dh, s));
+  if (L->last_T > 0 && !L->fused_group)
+    CK(cudaMemcpyAsync(&total, L->ws.grp_off + L->G, sizeof(int32_t), dh, s));
   CK(cudaStreamSynchronize(s));
   if (L->last_T > 0 && L->fused_group) {
     // rows live in per-group regions on the device, each group's rows in the
     // order the router CTAs reserved them: gather them group by group into
     // the contiguous padded layout, in token order
+    // (the combine copied the group sizes to grp_cnt; offsets pad each group
+    // to whole 128-row tiles)
     std::vector<int32_t> cnt(L->G), off(L->G + 1);
     CK(cudaMemcpyAsync(cnt.data(), L->ws.grp_cnt, sizeof(int32_t) * L->G, dh, s));
-    CK(cudaMemcpyAsync(off.data(), L->ws.grp_off, sizeof(int32_t) * (L->G + 1), dh, s));
     CK(cudaStreamSynchronize(s));
+    off[0] = 0;
+    for (int g = 0; g < L->G; ++g) off[g + 1] = off[g] + (cnt[g] + 127) / 128 * 128;
+    total = off[L->G];
     if (counts) memcpy(counts, cnt.data(), sizeof(int32_t) * L->G);
     if (offsets) memcpy(offsets, off.data(), sizeof(int32_t) * (L->G + 1));
     for (int g = 0; g < L->G; ++g) {
@@ -408,7 +414,7 @@ int64_t unif_moe_max_rows(unif_moe_t L) { return L ? L->max_rows : -1; }
 
 int unif_moe_kernels_per_forward(unif_moe_t L) {
   if (!L) return -1;
-  return L->fused_group ? 4 : 6;
+  return L->fused_group ? (L->tile_list ? 5 : 4) : 6;
 }
 
 int unif_moe_set_stage_events(unif_moe_t L, void* const* events) {
