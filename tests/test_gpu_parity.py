@@ -110,6 +110,26 @@ def test_max_tokens_and_reuse():
     np.testing.assert_allclose(g2.y, g.y[:333], rtol=1e-2, atol=1e-6)  # one bf16 ulp
 
 
+def test_smaller_then_larger_forward_on_one_handle():
+    """A small forward, then the full one: the accumulator rows and the
+    group counters the first forward used are clean for the second."""
+    wl = workloads.make_workload(small(tokens=1000))
+    g1 = run_gpu(wl, x=wl.x[:200].clone(), mask=None)
+    g = run_gpu(wl, layer=g1.layer)
+    assert_parity(wl, g, compare(wl, g))
+
+
+def test_kernels_per_forward():
+    s = small(tokens=500)
+    assert make_layer(s).kernels_per_forward() == 4   # grouping inside the router
+    assert make_layer(small("f32", tokens=64)).kernels_per_forward() == 6
+
+
+def test_kernels_per_forward_streaming(monkeypatch):
+    monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
+    assert make_layer(small(tokens=500)).kernels_per_forward() == 5   # + tile list
+
+
 @pytest.mark.parametrize("shape", [
     dict(d_model=64, d_ff=256, n_experts=2, n_blocks=2),     # B = 2: b = 1 always
     dict(d_model=192, d_ff=768, n_experts=6, n_blocks=4),
