@@ -44,14 +44,39 @@ def load_peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
+# Routing variants (the ablations of Table IV and the fixed cumulative-mass
+# thresholds): overrides of the layer's thresholds.
+ROUTINGS = {
+    "adaptive": {},
+    "alpha0.4": {"alpha_fixed": 0.4},
+    "top2": {"topk_fixed": 2},
+    "prefix": {"prefix_blocks": 1},
+    "theta0.5": {"beta_fixed": 0.5},
+    "theta0.7": {"beta_fixed": 0.7},
+    "theta0.9": {"beta_fixed": 0.9},
+}
+
+
+def routing_desc(s):
+    parts = []
+    if not math.isnan(s.alpha_fixed):
+        parts.append("alpha fixed %.2f" % s.alpha_fixed)
+    if not math.isnan(s.beta_fixed):
+        parts.append("beta fixed %.2f" % s.beta_fixed)
+    if s.topk_fixed:
+        parts.append("top-%d residual experts" % s.topk_fixed)
+    if s.prefix_blocks:
+        parts.append("prefix block selection")
+    return ", ".join(parts) if parts else "adaptive (Eqs. 18-27)"
+
+
 def workload_desc(s, T_valid):
     return {"workload": "%s: %d tokens (%d valid), d=%d, H=%d in B=%d blocks of %d, K=%d residual "
                         "experts + 1 shared, %s" % (s.name, s.tokens, T_valid, s.d_model, s.d_ff,
                                                     s.n_blocks, s.block_width, s.n_experts, s.dtype),
             "tokens": s.tokens, "valid_tokens": T_valid, "d_model": s.d_model, "d_ff": s.d_ff,
             "n_blocks": s.n_blocks, "n_experts": s.n_experts,
-            "thresholds": "adaptive (Eqs. 18-27)" if math.isnan(s.beta_fixed) else
-                          "beta fixed %.2f" % s.beta_fixed}
+            "thresholds": routing_desc(s)}
 
 
 # ----------------------------------------------------------------- ranks
@@ -200,6 +225,8 @@ def main():
     ap.add_argument("--workload", default="vit_s")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--routing", default="adaptive", choices=sorted(ROUTINGS),
+                    help="routing variant (Table IV ablations, fixed thresholds)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -210,7 +237,7 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    s = workloads.spec(args.workload)
+    s = workloads.spec(args.workload, **ROUTINGS[args.routing])
 
     if args.impl == "reference":
         if rank != 0:
