@@ -117,7 +117,9 @@ UNIF_MOE_API int unif_moe_forward(unif_moe_t h, const void* x_dev, void* out_dev
  * not NULL) to the handle's device staging buffers, runs the forward, copies
  * the output to out_host and the counts to shared_counts_host /
  * residual_counts_host (each may be NULL), and synchronises `stream` before
- * returning. Host buffers should be pinned for asynchronous copies. */
+ * returning. Host buffers should be pinned for asynchronous copies; output
+ * buffers (out_host and the counts) in pinned host memory the device can
+ * address are written by the kernels directly, with no copy back. */
 UNIF_MOE_API int unif_moe_forward_host(unif_moe_t h, const void* x_host, void* out_host, int T,
                           const uint8_t* token_mask_host, int32_t* shared_counts_host,
                           int32_t* residual_counts_host, void* stream);

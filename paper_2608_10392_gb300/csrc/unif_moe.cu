@@ -291,6 +291,20 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
   return UNIF_MOE_OK;
 }
 
+// The device address of pinned, mapped host memory (nullptr for any other
+// pointer, including NULL): the kernels can store into it directly.
+static void* mapped_host(void* p) {
+  if (!p) return nullptr;
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();  // an unregistered pointer is not an error here
+    return nullptr;
+  }
+  if (at.type != cudaMemoryTypeHost || !at.devicePointer) return nullptr;
+  if ((reinterpret_cast<uintptr_t>(at.devicePointer) & 15u) != 0) return nullptr;
+  return at.devicePointer;
+}
+
 int unif_moe_forward_host(unif_moe_t L, const void* x_host, void* out_host, int T,
                           const uint8_t* mask_host, int32_t* b_host, int32_t* k_host,
                           void* stream) {
@@ -319,12 +333,22 @@ int unif_moe_forward_host(unif_moe_t L, const void* x_host, void* out_host, int 
   const size_t xb = es * (size_t)T * L->d;
   CK(cudaMemcpyAsync(w.x_stage, x_host, xb, cudaMemcpyHostToDevice, s));
   if (mask_host) CK(cudaMemcpyAsync(w.mask_stage, mask_host, (size_t)T, cudaMemcpyHostToDevice, s));
-  int rc = unif_moe_forward(L, w.x_stage, w.out_stage, T, mask_host ? w.mask_stage : nullptr,
-                            b_host ? w.b_stage : nullptr, k_host ? w.k_stage : nullptr, stream);
+  // Outputs in pinned host memory that the device can address are written
+  // there by the kernels themselves (the combine, the router), without a
+  // staging buffer and a copy back.
+  void* out_dev = mapped_host(out_host);
+  int32_t* b_dev = static_cast<int32_t*>(mapped_host(b_host));
+  int32_t* k_dev = static_cast<int32_t*>(mapped_host(k_host));
+  int rc = unif_moe_forward(L, w.x_stage, out_dev ? out_dev : w.out_stage, T,
+                            mask_host ? w.mask_stage : nullptr,
+                            b_host ? (b_dev ? b_dev : w.b_stage) : nullptr,
+                            k_host ? (k_dev ? k_dev : w.k_stage) : nullptr, stream);
   if (rc != UNIF_MOE_OK) return rc;
-  CK(cudaMemcpyAsync(out_host, w.out_stage, xb, cudaMemcpyDeviceToHost, s));
-  if (b_host) CK(cudaMemcpyAsync(b_host, w.b_stage, sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
-  if (k_host) CK(cudaMemcpyAsync(k_host, w.k_stage, sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
+  if (!out_dev) CK(cudaMemcpyAsync(out_host, w.out_stage, xb, cudaMemcpyDeviceToHost, s));
+  if (b_host && !b_dev)
+    CK(cudaMemcpyAsync(b_host, w.b_stage, sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
+  if (k_host && !k_dev)
+    CK(cudaMemcpyAsync(k_host, w.k_stage, sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
   CK(cudaStreamSynchronize(s));
   return UNIF_MOE_OK;
 }

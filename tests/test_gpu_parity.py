@@ -288,6 +288,19 @@ def test_forward_host_matches_device():
     assert np.array_equal(b.numpy(), g.b) and np.array_equal(k.numpy(), g.k)
 
 
+def test_forward_host_pageable_buffers():
+    """Pageable host buffers go through the staging buffers and copies."""
+    wl = workloads.make_workload(small(tokens=500))
+    g = run_gpu(wl)
+    xh = wl.x.clone()
+    out = torch.empty_like(xh)
+    b = torch.empty(500, dtype=torch.int32)
+    k = torch.empty(500, dtype=torch.int32)
+    g.layer.forward_host(xh, out, shared_counts_host=b, residual_counts_host=k)
+    np.testing.assert_allclose(out.float().numpy(), g.y, rtol=1e-2, atol=1e-6)  # one bf16 ulp
+    assert np.array_equal(b.numpy(), g.b) and np.array_equal(k.numpy(), g.k)
+
+
 # ------------------------------------------- GEMM kernel variants
 
 @pytest.mark.parametrize("kernels", ["weight_stationary", "streaming"])
