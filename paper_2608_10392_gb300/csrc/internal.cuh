@@ -104,7 +104,7 @@ struct unif_moe_layer {
   bool tile_list = false;  // a streaming GEMM reads the tile list: build it after the router
   int device = 0;
   bool loaded = false;
-  bool y_dirty = false;  // the output accumulator may hold sums of a forward cut short
+  bool y_dirty = false;  // accumulator / grouping counters may hold state of a forward cut short
   int last_T = -1;
   // Weights (device, owned).
   float* wr = nullptr;      // [d][router_cols_pad]: W_shr, W_g, mu_1..mu_B (fp32)

@@ -262,11 +262,13 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
   DeviceGuard dg(L->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = L->stage_ev;
-  // The output accumulator is all zero between forwards (each combine zeroes
-  // the rows it reads). A forward that returned before launching its
-  // combine leaves it dirty: clear it all first.
-  if (L->y_dirty)
+  // The output accumulator and the grouping counters are all zero between
+  // forwards (each combine zeroes them). A forward that returned before
+  // launching its combine leaves them dirty: clear them first.
+  if (L->y_dirty) {
     CK(cudaMemsetAsync(L->ws.y32, 0, sizeof(float) * (size_t)L->max_tokens * L->d, s));
+    if (L->fused_group) CK(cudaMemsetAsync(L->ws.grp_fill, 0, sizeof(int32_t) * L->G, s));
+  }
   L->y_dirty = true;
   if (ev[0]) CK(cudaEventRecord(ev[0], s));
   if (L->dtype == UNIF_MOE_BF16) {
