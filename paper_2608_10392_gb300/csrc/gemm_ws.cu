@@ -1,9 +1,10 @@
 // Weight-stationary grouped expert GEMMs (tcgen05 + TMEM) for bf16 layers
 // whose per-group weight slice fits in shared memory.
 //
-// The permute step sorts the tile list by group g = (expert e, block b), so
-// consecutive tiles mostly share one weight slice: K_e[:, H_b] (M x d) for the
-// up projection, V_e[H_b, :] (d x M) for the down projection (Eqs. 16, 28-29).
+// Tiles are numbered group by group, g = (expert e, block b) (from the
+// router's group sizes, or the grouping kernels' tile list), so consecutive
+// tiles mostly share one weight slice: K_e[:, H_b] (M x d) for the up
+// projection, V_e[H_b, :] (d x M) for the down projection (Eqs. 16, 28-29).
 // Each CTA takes an equal contiguous run of tiles and keeps the current
 // group's slice resident in shared memory, reloading it only when the group
 // changes, slab by slab as the last MMAs of the previous group release each

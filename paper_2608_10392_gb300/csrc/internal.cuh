@@ -67,7 +67,7 @@ struct Workspace {
   int32_t* tile_rows = nullptr;  // [max_tiles] rows of the tile that are not padding
   int32_t* row_tok = nullptr;    // [max_rows], or [G][region] when the router groups (-1 = padding)
   float* row_w = nullptr;        // same layout
-  // Look-back state of the grouping inside the router (bf16 layers).
+  // Fill counters of the grouping inside the router (bf16 layers).
   int32_t* grp_fill = nullptr;   // [G] rows reserved per group (the group sizes once the router completed)
   // Intermediate activations h = GeLU(x K_e[:, H_b]) per row, and the fp32
   // output accumulator.
