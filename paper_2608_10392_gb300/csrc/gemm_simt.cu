@@ -133,7 +133,7 @@ cudaError_t launch_gemms_simt(unif_moe_layer* L, const void* x, int T, cudaEvent
       static_cast<const float*>(x), static_cast<const float*>(L->w_up), h, a);
   if (mid) cudaEventRecord(mid, s);
   simt_gemm_kernel<1, float, float, float><<<grid, kThreads, 0, s>>>(
-      h, static_cast<const float*>(L->w_down), h, a);
+      h, static_cast<const float*>(L->w_down), nullptr, a);  // (output: the accumulator)
   return cudaGetLastError();
 }
 

@@ -274,7 +274,6 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       }
       if (!wait_warp(accf_bar(acc), acc_phase, abort_flag, p.status, p.wait_limit)) break;
       tc_fence_after();
-      const int row = row0 + q * 32 + lane;
       const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)acc * kAccStride;
       const int c_begin = half * cols;
       if (MODE == 0) {

@@ -362,7 +362,7 @@ int unif_moe_get_routing(unif_moe_t L, float* alpha, uint64_t* shared_mask, uint
   if (L->last_T < 0) { set_error("no forward has run"); return UNIF_MOE_ERR_STATE; }
   DeviceGuard dg(L->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const size_t T = (size_t)L->last_T, K = (size_t)L->K;
+  const size_t T = (size_t)L->last_T;
   const cudaMemcpyKind dd = cudaMemcpyDeviceToDevice;
   if (T > 0) {
     if (alpha) CK(cudaMemcpyAsync(alpha, L->ws.alpha, sizeof(float) * T, dd, s));
