@@ -71,6 +71,10 @@ struct Params {
   const int32_t* fill;
   int G, region;
   int per_cta;  // room for this many tiles of a CTA's run in the shared tile table
+  // Down projection with n_slices > 1: the work items are (column slice s,
+  // tile), slice-major, each with one sub-tile (n_sub = 1) of bn columns at
+  // s bn; only one slice's weight slabs are resident at a time.
+  int n_slices;
   const int32_t* n_tiles;
   const int32_t* tile_group;
   const int32_t* tile_row0;  // first row of each tile in row_tok / row_w
@@ -153,7 +157,7 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     if (MODE == 0) grid_dep_wait();
     tile_table(p.fill, p.G, p.region, lane, first_s, gcnt_s);
     __syncwarp();
-    const int nt = first_s[p.G];
+    const int nt = p.n_slices == 1 ? first_s[p.G] : 0;  // (slices: cursors, below)
     const int tb = (int)(((long long)blockIdx.x * nt) / gridDim.x);
     const int te = (int)(((long long)(blockIdx.x + 1) * nt) / gridDim.x);
     for (int k = tb + lane; k < te; k += 32) {
@@ -178,21 +182,42 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 
   // This CTA's contiguous run of tiles (sizes differ by at most one).
   const int n_tiles = p.fill ? first_s[p.G] : p.n_tiles[0];
-  const int t_begin = (int)(((long long)blockIdx.x * n_tiles) / gridDim.x);
-  const int t_end = (int)(((long long)(blockIdx.x + 1) * n_tiles) / gridDim.x);
-  // group, first row and real rows of tile k (t_begin <= k < t_end)
-  auto tile_of = [&](int k, int& g, int& r0, int& rows) {
-    if (p.fill) {
-      const int j = k - t_begin;
+  // work items: tiles, or (slice, tile) pairs slice-major; "tile" below
+  // names an item index
+  const int n_items = n_tiles * p.n_slices;
+  const int t_begin = (int)(((long long)blockIdx.x * n_items) / gridDim.x);
+  const int t_end = (int)(((long long)(blockIdx.x + 1) * n_items) / gridDim.x);
+  // For item v (t_begin <= v < t_end): the weight-slab key (slice * G +
+  // group), the tile's first row and real rows. With slices, each thread's
+  // lookups move forward through the items, so a cursor over the group table
+  // finds the group in amortised constant time.
+  int cur_g = 0;
+  auto tile_of = [&](int v, int& key, int& r0, int& rows) {
+    const int slice = v / n_tiles, k = v - slice * n_tiles;
+    int g;
+    if (p.fill && p.n_slices == 1) {
+      const int j = v - t_begin;
       g = run_s[j];
       r0 = run_s[p.per_cta + j];
       rows = run_s[2 * p.per_cta + j];
+    } else if (p.fill) {
+      if (k < first_s[cur_g]) cur_g = 0;
+      while (first_s[cur_g + 1] <= k) ++cur_g;  // first_s[G] = n_tiles > k
+      g = cur_g;
+      const int i = k - first_s[g];
+      r0 = g * p.region + 128 * i;
+      rows = min(128, gcnt_s[g] - 128 * i);
     } else {
       g = p.tile_group[k];
       r0 = p.tile_row0[k];
       rows = p.tile_rows[k];
     }
+    key = slice * p.G + g;
   };
+  // items of the down projection read h tile (v mod n_tiles); their output
+  // columns start at slice * n_sub * bn
+  auto item_tile = [&](int v) { return v % n_tiles; };
+  auto item_col0 = [&](int v) { return (v / n_tiles) * p.n_sub * p.bn; };
 
   if (MODE == 0 && warp < kProducerWarps) {
     // ---------------- up: A stage owners (x rows gathered) -----------------
@@ -262,7 +287,7 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             break;
           }
           mbar_expect_tx(fullA(stage), kStageA);
-          tma_load_2d(sA + stage * kStageA, &tmA, fullA(stage), kb * kBK, tile * kBM);
+          tma_load_2d(sA + stage * kStageA, &tmA, fullA(stage), kb * kBK, item_tile(tile) * kBM);
           if (++stage == kStagesA) { stage = 0; phase ^= 1u; }
         }
       }
@@ -280,7 +305,10 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         tile_of(tile, g, r0_unused, rows_unused);
         if (g == g_prev) continue;
         g_prev = g;
-        const int e = g / p.B, blk = g % p.B;
+        // key = slice * G + group; group = e * B + blk
+        const int slice = g / p.G, grp = g - slice * p.G;
+        const int e = grp / p.B, blk = grp % p.B;
+        const int col0 = slice * p.n_sub * p.bn;  // the slice's first output column
         for (int s = 0; s < n_slabs; ++s) {
           const int ns = s / p.num_kb, kb = s % p.num_kb;
           if (run > 0 &&
@@ -292,7 +320,8 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           if (MODE == 0)  // w_up viewed [(K+1) H][d]
             tma_load_2d(sB + s * slab_bytes, &tmB, wfull(s), kb * kBK, e * p.H + blk * p.M + ns * p.bn);
           else            // w_down viewed [(K+1) d][H]
-            tma_load_2d(sB + s * slab_bytes, &tmB, wfull(s), blk * p.M + kb * kBK, e * p.d + ns * p.bn);
+            tma_load_2d(sB + s * slab_bytes, &tmB, wfull(s), blk * p.M + kb * kBK,
+                        e * p.d + col0 + ns * p.bn);
         }
         ++run;
       }
@@ -313,6 +342,10 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // current stage's MMAs go out and read back after.
     const int m = warp - kMmaWarp;
     const bool split_n = !(MODE == 1 && p.n_sub == 2);
+    // A stages read by one sub-tile only are freed after their MMAs (the up
+    // projection, and sliced down projections); otherwise after the tile's
+    // last sub-tile
+    const bool a_once = MODE == 0 || p.n_sub == 1;
     const int n_mma = split_n ? p.bn / 2 : p.bn;
     const uint32_t idesc = idesc_bf16(kBM, n_mma);
     // B rows and accumulator columns this warp covers (split_n), in 16-byte
@@ -372,7 +405,7 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             // the stage after this one, in ring order (the next tile's first
             // stage after the last k-block); read back after the MMAs
             const uint32_t next_done =
-                first_pass && (MODE == 0 || kb + 1 < p.num_kb) ? mbar_test(fullA(st_n), ph_n) : 0u;
+                first_pass && (a_once || kb + 1 < p.num_kb) ? mbar_test(fullA(st_n), ph_n) : 0u;
             tc_fence_after();
             // descriptor start addresses advance in 16-byte units: +2 per 32 bytes
             const uint64_t a_desc = a_desc0 + (uint64_t)(st * (kStageA >> 4));
@@ -382,7 +415,7 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               for (int k = 0; k < kBK / 16; ++k)
                 umma_bf16(d_tmem, a_desc + 2 * k, b_desc + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
               if (release) umma_commit(wempty(s));
-              if (MODE == 0) umma_commit(emptyA(st));  // one pass over A: free it now
+              if (a_once) umma_commit(emptyA(st));  // one pass over A: free it now
             }
             ready = __all_sync(0xffffffffu, next_done != 0u);
             st = st_n;
@@ -398,16 +431,16 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
       }
       if (!ok) break;
-      // advance the A ring past this tile; the down projection frees its
-      // stages only after both sub-tiles read them
+      // advance the A ring past this tile; a down projection with several
+      // sub-tiles frees its stages only after all of them read them
       for (int kb = 0; kb < p.num_kb; ++kb) {
-        if (MODE == 1) {
+        if (!a_once) {
           if (elect_one()) umma_commit(emptyA(stage));
           __syncwarp();
         }
         if (++stage == kStagesA) { stage = 0; phase ^= 1u; }
       }
-      if (MODE == 1) ready = false;
+      if (!a_once) ready = false;
     }
   } else if (warp >= kFirstEpiWarp) {
     // ---------------- epilogue ----------------------------------------------
@@ -486,7 +519,7 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           // add 4 rows x 128 contiguous bytes per instruction.
           float* stf = reinterpret_cast<float*>(stg);
           const int r_sub = lane >> 3, c8 = lane & 7;
-          float* ybase = p.y32 + ns * p.bn + c_begin;
+          float* ybase = p.y32 + item_col0(tile) + ns * p.bn + c_begin;
           for (int c = 0; c < cols; c += 32) {
             float v[32];
             tmem_ld32(t_row + c_begin + c, v);
@@ -557,18 +590,49 @@ int gemm_ws_setup(unif_moe_layer* L) {
     L->up_ws = true;
     L->up_ws_smem = (uint32_t)up_smem;
   }
+  // Down: every sub-tile's slabs resident (the h tile feeds all of them),
+  // where they fit; else one column slice of the output at a time (items =
+  // (slice, tile)), with the widest slice whose slabs fit. Slices re-read
+  // each h tile once per slice: they pay off only where the h tile fits the
+  // A ring (measured on GB300: ViT-B 440 -> 378 us; BERT-base, whose h tile
+  // needs 6 stages, and the stress layer, whose 1.2 GB h is read from HBM,
+  // ran slower than the streaming kernel).
   const int down_kb = L->M / tc::kBK;
   const uint64_t down_slabs = (uint64_t)L->down_nsub * down_kb;
   const uint64_t down_smem =
       Cfg<1>::kFixed + down_slabs * (uint64_t)L->down_bn * tc::kBK * 2 + table;
+  int bn = 0, nsub = 0, slices = 0;
+  uint64_t smem = 0;
   if (down_kb <= Cfg<1>::kStagesA && down_slabs <= (uint64_t)kMaxSlabs && down_smem <= kMaxSmem) {
+    bn = L->down_bn; nsub = L->down_nsub; slices = 1; smem = down_smem;
+  } else if (down_kb <= Cfg<1>::kStagesA) {
+    const uint64_t small_table =
+        L->fused_group ? ((uint64_t)(2 * L->G + 1) * 4 + 15) / 16 * 16 : 0;
+    for (int b = 256; b >= 64; b -= 64) {
+      if (L->d % b != 0) continue;
+      const uint64_t sm = Cfg<1>::kFixed + (uint64_t)down_kb * b * tc::kBK * 2 + small_table;
+      if (sm <= kMaxSmem) {
+        bn = b; nsub = 1; slices = L->d / b; smem = sm;
+        break;
+      }
+    }
+  }
+  if (bn > 0) {
     if (cudaFuncSetAttribute(ws_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)down_smem) != cudaSuccess) {
+                             (int)smem) != cudaSuccess) {
       set_error("cudaFuncSetAttribute failed for the weight-stationary down kernel");
       return UNIF_MOE_ERR_CUDA;
     }
+    if (!encode_bf16_map(&L->tm_wdown_ws, L->w_down, L->H, ((uint64_t)L->K + 1) * L->d, tc::kBK,
+                         bn, 128)) {
+      set_error("cuTensorMapEncodeTiled failed for the down weight slabs");
+      return UNIF_MOE_ERR_CUDA;
+    }
     L->down_ws = true;
-    L->down_ws_smem = (uint32_t)down_smem;
+    L->down_ws_smem = (uint32_t)smem;
+    L->ws_down_bn = bn;
+    L->ws_down_nsub = nsub;
+    L->down_slices = slices;
   }
   return UNIF_MOE_OK;
 }
@@ -579,6 +643,7 @@ static tc::ws::Params ws_params(unif_moe_layer* L, const void* x) {
   p.G = L->G;
   p.region = L->region_rows;
   p.per_cta = (int)((L->max_tiles + L->n_sm - 1) / L->n_sm);
+  p.n_slices = 1;
   p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group; p.tile_row0 = L->ws.tile_row0;
   p.tile_rows = L->ws.tile_rows; p.row_tok = L->ws.row_tok; p.row_w = L->ws.row_w;
   p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;
@@ -599,9 +664,10 @@ cudaError_t launch_up_ws(unif_moe_layer* L, const void* x, cudaStream_t s) {
 
 cudaError_t launch_down_ws(unif_moe_layer* L, cudaStream_t s) {
   tc::ws::Params p = ws_params(L, nullptr);
-  p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
+  p.n_sub = L->ws_down_nsub; p.bn = L->ws_down_bn; p.num_kb = L->M / tc::kBK;
+  p.n_slices = L->down_slices;
   return launch_dependent(tc::ws::ws_gemm_kernel<1>, dim3(L->n_sm), dim3(tc::ws::Cfg<1>::kThreads),
-                          L->down_ws_smem, s, L->tm_h, L->tm_wdown, p);
+                          L->down_ws_smem, s, L->tm_h, L->tm_wdown_ws, p);
 }
 
 }  // namespace unif

@@ -124,6 +124,10 @@ struct unif_moe_layer {
   // memory) and their dynamic shared-memory sizes.
   bool up_ws = false, down_ws = false;
   uint32_t up_ws_smem = 0, down_ws_smem = 0;
+  // weight-stationary down projection: sub-tile width and count, and the
+  // number of output column slices run as separate work items
+  int ws_down_bn = 0, ws_down_nsub = 0, down_slices = 1;
+  CUtensorMap tm_wdown_ws;  // w_down slabs of ws_down_bn rows
   // Optional caller-owned timing events recorded at the stage boundaries.
   cudaEvent_t stage_ev[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
 };

@@ -348,3 +348,32 @@ def test_repeated_forwards_match_streaming_kernels(monkeypatch):
         assert L.sync_status() == 0
         rel = (y - ref).abs().amax(1) / ref.abs().amax(1).clamp_min(1e-6)
         assert float(rel.max()) < 1e-2, int((rel >= 1e-2).sum())
+
+
+def test_repeated_forwards_sliced_down_projection(monkeypatch):
+    """A ViT-B-shaped layer (d = 768: the weight-stationary down projection
+    runs in three 256-column slices) agrees with the streaming kernels over
+    repeated forwards, and with the oracle on sampled tokens."""
+    s = workloads.spec("vit_b", tokens=3000)
+    wl = workloads.make_workload(s)
+    dev = torch.device("cuda")
+
+    def layer():
+        L = make_layer(s)
+        L.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
+        return L
+
+    x = wl.x.to(dev)
+    monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
+    ref = layer().forward(x).float()
+    monkeypatch.delenv("UNIF_MOE_GEMM_KERNELS")
+    L = layer()
+    for _ in range(5):
+        y = L.forward(x).float()
+        torch.cuda.synchronize()
+        assert L.sync_status() == 0
+        rel = (y - ref).abs().amax(1) / ref.abs().amax(1).clamp_min(1e-6)
+        assert float(rel.max()) < 1e-2, int((rel >= 1e-2).sum())
+    g = run_gpu(wl, layer=L)
+    assert_parity(wl, g, compare(wl, g, sample=300))
+
