@@ -308,9 +308,8 @@ __host__ __device__ constexpr int group_rows_smem_ints(int NW, int G) {
 // the chunk's member bits of the group (token order) and writes those rows
 // one after another.
 template <int NW>
-__device__ void group_rows(const GroupArgs& a, int tid, int w, int lane, int t0,
-                           const uint32_t* masks, const float* dec_s, int dec_stride, int32_t* sm,
-                           uint32_t bar) {
+__device__ void group_rows(const GroupArgs& a, int tid, int t0, const uint32_t* masks,
+                           const float* dec_s, int dec_stride, int32_t* sm, uint32_t bar) {
   constexpr int NT = NW * 32;
   const int G = a.G, B = a.B;
   int32_t* cnt_s = sm;                    // [NW][G] chunk counts

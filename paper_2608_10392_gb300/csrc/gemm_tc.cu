@@ -514,7 +514,7 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
       named_bar(1, 128);
       if (row == 0) misc_s[7] = *abort_flag;  // one reading for all four warps
       named_bar(1, 128);
-      if (!misc_s[7]) group_rows<4>(p.grp, row, q, lane, t0, cscr, ss, 2 * K + 1, gsm, 1);
+      if (!misc_s[7]) group_rows<4>(p.grp, row, t0, cscr, ss, 2 * K + 1, gsm, 1);
     }
   }
   tc_fence_before();
