@@ -123,6 +123,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
   }
+  __syncwarp();  // every warp converged before the CTA barrier
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -340,6 +341,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
     }
   }
+  __syncwarp();  // every warp converged before the CTA barrier
   tc_fence_before();
   __syncthreads();
   if (warp == kMmaWarp) {
@@ -428,6 +430,7 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     tmem_alloc(smem_u32(tmem_slot), p.tmem_cols);
     tmem_relinquish();
   }
+  __syncwarp();  // every warp converged before the CTA barrier
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -517,6 +520,7 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
       if (!misc_s[7]) group_rows<4>(p.grp, row, t0, cscr, ss, 2 * K + 1, gsm, 1);
     }
   }
+  __syncwarp();  // every warp converged before the CTA barrier
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {

@@ -168,6 +168,9 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       run_s[2 * p.per_cta + k - tb] = rows;
     }
   }
+  // every warp converged before the CTA barrier (lane 0 of warp 0 ran the
+  // barrier setup, the table warp's lanes ran different trip counts)
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -548,6 +551,9 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
     if (MODE == 0 && lane == 0) bulk_wait_all();  // h complete before the CTA retires
   }
+  // every warp converged before the CTA barrier (an epilogue warp's lane 0
+  // may still wait for its h stores)
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == kMmaWarp) {
