@@ -86,8 +86,9 @@ __device__ __forceinline__ void decide_token_rt(const DecideArgs& a, int t, bool
       sv[j] = expf(l[j] - m);
       den += sv[j];
     }
+    const float inv_den = 1.0f / den;
     for (int j = 0; j < K; ++j) {
-      sv[j] = sv[j] / den;
+      sv[j] = sv[j] * inv_den;
       a.s[(size_t)t * K + j] = sv[j];
     }
     // Eqs. 25-27: rank the experts by affinity (by logit, which orders them
@@ -129,6 +130,22 @@ __device__ __forceinline__ void decide_token_rt(const DecideArgs& a, int t, bool
   }
   shr_out = shr;
   em_out = em;
+}
+
+// A token's KC affinities (KC a multiple of 8, dst 32-byte aligned): one
+// 32-byte store per 8, so that each store fills a whole sector instead of a
+// warp's store instruction touching 32 sectors partially.
+template <int KC>
+__device__ __forceinline__ void store_affinities(float* dst, const float (&e)[KC]) {
+  static_assert(KC % 8 == 0, "whole 32-byte sectors");
+#pragma unroll
+  for (int j = 0; j < KC; j += 8)
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst + j),
+                 "r"(__float_as_uint(e[j])), "r"(__float_as_uint(e[j + 1])),
+                 "r"(__float_as_uint(e[j + 2])), "r"(__float_as_uint(e[j + 3])),
+                 "r"(__float_as_uint(e[j + 4])), "r"(__float_as_uint(e[j + 5])),
+                 "r"(__float_as_uint(e[j + 6])), "r"(__float_as_uint(e[j + 7]))
+                 : "memory");
 }
 
 // The same decisions with K and B known at compile time: the priorities,
@@ -177,12 +194,13 @@ __device__ __forceinline__ void decide_token_ct(const DecideArgs& a, int t, bool
       e[j] = expf(l[j] - m);
       den += e[j];
     }
+    const float inv_den = 1.0f / den;
 #pragma unroll
     for (int j = 0; j < KC; ++j) {
-      e[j] = e[j] / den;
+      e[j] = e[j] * inv_den;
       sv[j] = e[j];
-      a.s[(size_t)t * KC + j] = e[j];
     }
+    store_affinities<KC>(a.s + (size_t)t * KC, e);
     const float beta = isnan(a.beta_fixed) ? 1.0f - alpha : a.beta_fixed;
     int rk[KC];
     int kcount = KC;
@@ -214,7 +232,8 @@ __device__ __forceinline__ void decide_token_ct(const DecideArgs& a, int t, bool
   } else if (t < a.T) {
     a.alpha[t] = 0.f; a.b[t] = 0; a.k[t] = 0; a.shr[t] = 0ull; a.emask[t] = 0ull;
 #pragma unroll
-    for (int j = 0; j < KC; ++j) a.s[(size_t)t * KC + j] = 0.f;
+    for (int j = 0; j < KC; j += 4)
+      *reinterpret_cast<float4*>(a.s + (size_t)t * KC + j) = make_float4(0.f, 0.f, 0.f, 0.f);
     if (a.bcnt) a.bcnt[t] = 0;
     if (a.kcnt) a.kcnt[t] = 0;
   }
@@ -239,9 +258,9 @@ __device__ __forceinline__ void decide_token(const DecideArgs& a, int t, bool va
 // scratch is 128 words of this warp's shared memory. One ballot per block
 // (lanes sharing it) and per residual expert (lanes selecting it); a group's
 // count is then a population count of their intersection.
-__device__ __forceinline__ void count_chunk_pairs(const DecideArgs& a, int lane, uint64_t shr,
-                                                  uint64_t em, uint32_t* scratch, int32_t* out,
-                                                  int stride) {
+__device__ __forceinline__ void count_chunk_pairs_rt(const DecideArgs& a, int lane, uint64_t shr,
+                                                     uint64_t em, uint32_t* scratch, int32_t* out,
+                                                     int stride) {
   const int K = a.K, B = a.B;
   for (int blk = 0; blk < B; ++blk) {
     const uint32_t m = __ballot_sync(0xffffffffu, (shr >> blk) & 1ull);
@@ -260,6 +279,49 @@ __device__ __forceinline__ void count_chunk_pairs(const DecideArgs& a, int lane,
     out[(size_t)g * stride] = c;
   }
   __syncwarp();
+}
+
+// The same counts with K and B known at compile time: the ballots issue
+// back to back, lane 0 stores all masks at once, and the group loop unrolls
+// with shifts for the divisions, so its shared-memory reads are all in
+// flight together.
+template <int KC, int BC>
+__device__ __forceinline__ void count_chunk_pairs_ct(int lane, uint64_t shr, uint64_t em,
+                                                     uint32_t* scratch, int32_t* out, int stride) {
+  uint32_t mb[BC], me[KC];
+#pragma unroll
+  for (int blk = 0; blk < BC; ++blk) mb[blk] = __ballot_sync(0xffffffffu, (shr >> blk) & 1ull);
+#pragma unroll
+  for (int e = 0; e < KC; ++e) me[e] = __ballot_sync(0xffffffffu, (em >> e) & 1ull);
+  if (lane == 0) {
+#pragma unroll
+    for (int blk = 0; blk < BC; ++blk) scratch[blk] = mb[blk];
+#pragma unroll
+    for (int e = 0; e < KC; ++e) scratch[64 + e] = me[e];
+  }
+  __syncwarp();
+  constexpr int G = (KC + 1) * BC;
+#pragma unroll
+  for (int g0 = 0; g0 < G; g0 += 32) {
+    const int g = g0 + lane;
+    if (g < G) {
+      const int e = g / BC, blk = g % BC;
+      const uint32_t sh = scratch[blk];
+      out[(size_t)g * stride] = e == 0 ? __popc(sh) : __popc(scratch[64 + e - 1] & ~sh);
+    }
+  }
+  __syncwarp();
+}
+
+__device__ __forceinline__ void count_chunk_pairs(const DecideArgs& a, int lane, uint64_t shr,
+                                                  uint64_t em, uint32_t* scratch, int32_t* out,
+                                                  int stride) {
+  if (a.K == 8 && a.B == 8)
+    count_chunk_pairs_ct<8, 8>(lane, shr, em, scratch, out, stride);
+  else if (a.K == 16 && a.B == 16)
+    count_chunk_pairs_ct<16, 16>(lane, shr, em, scratch, out, stride);
+  else
+    count_chunk_pairs_rt(a, lane, shr, em, scratch, out, stride);
 }
 
 // ---------------------------------------------------------------------------
