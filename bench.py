@@ -132,6 +132,43 @@ def measured_traffic(workload, kernel):
     return rec.get(kernel)
 
 
+def l2_reduction_ceiling(T, d, n_rows, dev, reps=10):
+    """TB/s of fp32 row reductions into a [T][d] accumulator in the down
+    projection epilogue's pattern (n_rows random rows of d values, 4 rows x
+    128 bytes per warp instruction), measured live with the probe library
+    (lib/libunif_probe.so); None where it is not built."""
+    import ctypes
+    import torch
+    path = os.path.join(ROOT, "paper_2608_10392_gb300", "lib", "libunif_probe.so")
+    if not os.path.exists(path) or d % 32 != 0:
+        return None
+    lib = ctypes.CDLL(path)
+    f = lib.unif_probe_l2_reductions
+    f.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                  ctypes.c_void_p]
+    g = torch.Generator().manual_seed(20260810)
+    tok = torch.randint(0, T, (n_rows,), generator=g, dtype=torch.int32).to(dev)
+    y = torch.zeros(T, d, dtype=torch.float32, device=dev)
+    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
+    stream = torch.cuda.current_stream(dev)
+
+    def launch():
+        rc = f(y.data_ptr(), tok.data_ptr(), n_rows, d, n_sm, ctypes.c_void_p(stream.cuda_stream))
+        if rc != 0:
+            raise RuntimeError("reduction probe launch failed (%d)" % rc)
+    for _ in range(3):
+        launch()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        launch()
+    b.record(stream)
+    b.synchronize()
+    ms = a.elapsed_time(b) / reps
+    return n_rows * d * 4 / (ms / 1e3) / 1e12
+
+
 # ----------------------------------------------------------------- clocks
 
 class ClockSampler:
@@ -389,6 +426,11 @@ def main():
     dom = "up_gemm" if stage_ms["up_gemm"] >= stage_ms["down_gemm"] else "down_gemm"
     ach = gemm_flops / (stage_ms[dom] / 1e3) / 1e12
     traffic = measured_traffic(s.name, dom)
+    # the down projection's fp32 reductions into the accumulator (one row of
+    # d values per (token, pair)) against the live-measured rate of the same
+    # reductions alone
+    red_bytes = 4.0 * d * sum_cb
+    red_peak = l2_reduction_ceiling(T, d, sum_cb, dev) if s.dtype == "bf16" else None
     router_bytes = T * d * elt + T * (4 * 3 + 8 * 2 + 12 * s.n_experts)
     combine_bytes = T * d * (4 + elt)
     permute_bytes = sum_cb * 8
@@ -419,6 +461,12 @@ def main():
                      "peak_kind": "%s bf16 sustained" % peak_kind},
         "stages": stages,
         "hbm_peak_gbs": hbm,
+        "reduction_bound": None if red_peak is None else {
+            "kernel": "down_gemm", "bytes": red_bytes,
+            "achieved": red_bytes / (stage_ms["down_gemm"] / 1e3) / 1e12, "peak": red_peak,
+            "unit": "TB/s", "frac": red_bytes / (stage_ms["down_gemm"] / 1e3) / 1e12 / red_peak,
+            "peak_kind": "live probe: the same number of random fp32 rows reduced alone in the "
+                         "epilogue's pattern"},
         "e2e": None if not e2e_ms else {
             "value": T_valid / (statistics.fmean(e2e_ms) / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
