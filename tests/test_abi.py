@@ -48,6 +48,23 @@ def test_only_declared_symbols_are_exported(lib):
     assert ours == declared_symbols()
 
 
+def test_measurement_probe_library(lib):
+    """The reduction probe bench.py times is built into its own library,
+    exports only its launcher, and rejects bad arguments before any CUDA
+    call (so this runs without a GPU)."""
+    import subprocess
+    from paper_2608_10392_gb300 import build
+    assert os.path.exists(build.PROBE_LIB)
+    out = subprocess.run(["nm", "-D", "--defined-only", build.PROBE_LIB], capture_output=True,
+                         text=True).stdout
+    assert [l.split()[-1] for l in out.splitlines() if " T unif_" in l] == ["unif_probe_l2_reductions"]
+    f = C.CDLL(build.PROBE_LIB).unif_probe_l2_reductions
+    f.argtypes = [C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_void_p]
+    assert f(None, None, 10, 384, 152, None) == -1          # null buffers
+    assert f(C.c_void_p(16), C.c_void_p(16), 10, 100, 152, None) == -1   # d not a multiple of 32
+    assert f(C.c_void_p(16), C.c_void_p(16), 0, 384, 152, None) == -1    # no rows
+
+
 def test_argument_errors_without_gpu(lib):
     import paper_2608_10392_gb300 as pkg
     th = pkg.Thresholds()
