@@ -430,7 +430,7 @@ def main():
     # d values per (token, pair)) against the live-measured rate of the same
     # reductions alone
     red_bytes = 4.0 * d * sum_cb
-    red_peak = l2_reduction_ceiling(T, d, sum_cb, dev) if s.dtype == "bf16" else None
+    red_peak = l2_reduction_ceiling(T, d, sum_cb, dev) if s.dtype == "bf16" and sum_cb > 0 else None
     router_bytes = T * d * elt + T * (4 * 3 + 8 * 2 + 12 * s.n_experts)
     combine_bytes = T * d * (4 + elt)
     permute_bytes = sum_cb * 8
