@@ -9,7 +9,10 @@ paper equation by equation (Eqs. 16-30); this module only compiles it, moves
 arrays in and out with ctypes, and chains the steps:
     prototypes (Eq. 20) -> route (Eqs. 17-27) -> forward (Eqs. 16, 28-30).
 `groups` lists the (expert, block) pairs the output sums over, grouped by
-pair (the bookkeeping behind Eq. 35).
+pair (the bookkeeping behind Eq. 35). `upcycle` and `sublayer` place the
+layer the way the paper's backbones use it (Sec. III: experts initialised
+from one dense FFN; Sec. B.1: converted FFN layers of DeiT-S, normalised
+first, and of BERT, normalised after the residual sum).
 """
 from __future__ import annotations
 
@@ -59,6 +62,7 @@ def _load():
             lib.oracle_forward.argtypes = [C.c_int] * 5 + [P] * 10
             lib.oracle_groups.argtypes = [C.c_int] * 3 + [P] * 9 + [C.c_longlong]
             lib.oracle_groups.restype = C.c_longlong
+            lib.oracle_layernorm.argtypes = [C.c_int, C.c_int, P, P, P, P, C.c_double, C.c_int, P]
             _lib = lib
     return _lib
 
@@ -233,3 +237,49 @@ def with_decisions(r: Routing, shr_mask: np.ndarray, expert_mask: np.ndarray, B:
     return Routing(alpha=r.alpha.copy(), beta=r.beta.copy(), b=b, k=k,
                    shr_mask=np.asarray(shr_mask, np.uint64).copy(), q=q, p=p, s=r.s.copy(),
                    u=r.u.copy(), margin=r.margin.copy())
+
+
+def layernorm(v, gamma, beta, eps: float, mask=None, round_mode: int = ROUND_NONE) -> np.ndarray:
+    """Layer normalisation of each token over its d features (biased variance,
+    eps inside the square root), rounded per round_mode; padding rows give 0."""
+    va = _f64(v)
+    T, d = va.shape
+    g = _f64(gamma).reshape(d)
+    b = _f64(beta).reshape(d)
+    m = _u8(mask)
+    out = np.empty((T, d), dtype=np.float64)
+    rc = _load().oracle_layernorm(T, d, _p(va), _p(m), _p(g), _p(b), float(eps), round_mode,
+                                  _p(out))
+    if rc != 0:
+        raise ValueError("oracle_layernorm: bad arguments")
+    return out
+
+
+def upcycle(w_up_dense, w_down_dense, K: int):
+    """Sec. III: every expert (the shared one and the K residual ones) starts
+    as the same dense FFN: K+1 copies of its up projection [H][d] and down
+    projection [d][H]."""
+    wu = _f64(w_up_dense)
+    wd = _f64(w_down_dense)
+    return (np.ascontiguousarray(np.broadcast_to(wu, (K + 1,) + wu.shape)),
+            np.ascontiguousarray(np.broadcast_to(wd, (K + 1,) + wd.shape)))
+
+
+def sublayer(x, w_router, w_up, w_down, B: int, gamma, beta, eps: float, norm_first: bool,
+             th: Optional[Thresholds] = None, mask=None, bias=None,
+             round_mode: int = ROUND_NONE):
+    """The layer as a Transformer sublayer (Sec. B.1 backbones):
+    norm_first (DeiT-S): out = x + F(LN(x)), LN(x) kept in the layer's input
+    precision (round_mode); otherwise (BERT): out = LN(x + F(x)). Padding
+    tokens give 0. Returns (out [T][d], Routing)."""
+    xa = _f64(x)
+    if norm_first:
+        xn = layernorm(xa, gamma, beta, eps, mask, round_mode)
+        y, r = layer(xn, w_router, w_up, w_down, B, th, mask, bias, round_mode)
+        out = xa + y
+    else:
+        y, r = layer(xa, w_router, w_up, w_down, B, th, mask, bias, round_mode)
+        out = layernorm(xa + y, gamma, beta, eps, mask, ROUND_NONE)
+    if mask is not None:
+        out[_u8(mask) == 0] = 0.0
+    return out, r

@@ -332,3 +332,33 @@ long long oracle_groups(int T, int K, int B, const uint8_t* mask, const double* 
   }
   return total;
 }
+
+/* The layer inside a Transformer sublayer (the converted FFN layers of the
+ * paper's DeiT-S and BERT backbones, Sec. B.1): layer normalisation of each
+ * token over its d features, in the standard form
+ *   LN(v) = gamma * (v - mean(v)) / sqrt(var(v) + eps) + beta,
+ * mean and var over the d features, var the biased (1/d) second central
+ * moment. Rows whose mask entry is 0 (padding) give 0. The result is
+ * rounded per round_mode (the precision the layer's inputs are kept in).
+ * v, out [T][d]; gamma, beta [d]; mask [T] or NULL. */
+int oracle_layernorm(int T, int d, const double* v, const uint8_t* mask, const double* gamma,
+                     const double* beta, double eps, int round_mode, double* out) {
+  if (T < 0 || d <= 0 || !v || !gamma || !beta || !out || !(eps >= 0.0)) return -1;
+  for (int t = 0; t < T; ++t) {
+    const double* row = v + (size_t)t * d;
+    double* o = out + (size_t)t * d;
+    if (mask && !mask[t]) {
+      for (int i = 0; i < d; ++i) o[i] = 0.0;
+      continue;
+    }
+    double mean = 0.0;
+    for (int i = 0; i < d; ++i) mean += row[i];
+    mean /= (double)d;
+    double var = 0.0;
+    for (int i = 0; i < d; ++i) var += (row[i] - mean) * (row[i] - mean);
+    var /= (double)d;
+    const double inv = 1.0 / sqrt(var + eps);
+    for (int i = 0; i < d; ++i) o[i] = round_to(gamma[i] * (row[i] - mean) * inv + beta[i], round_mode);
+  }
+  return 0;
+}

@@ -42,6 +42,14 @@ MUTANTS = {
     "b_truncated": ("int b = (int)nearbyint((double)B * alpha);", "int b = (int)((double)B * alpha);"),
     # GeLU without the 1/sqrt(2) scaling
     "gelu_scale": ("erf(v * M_SQRT1_2)", "erf(v)"),
+    # layer normalisation with the unbiased (1/(d-1)) variance
+    "ln_unbiased_variance": ("    var /= (double)d;", "    var /= (double)(d - 1);"),
+    # eps added outside the square root
+    "ln_eps_outside": ("const double inv = 1.0 / sqrt(var + eps);",
+                       "const double inv = 1.0 / (sqrt(var) + eps);"),
+    # beta scaled by gamma (the affine step applied before the shift)
+    "ln_beta_scaled": ("o[i] = round_to(gamma[i] * (row[i] - mean) * inv + beta[i], round_mode);",
+                       "o[i] = round_to(gamma[i] * ((row[i] - mean) * inv + beta[i]), round_mode);"),
 }
 
 

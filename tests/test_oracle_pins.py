@@ -393,3 +393,103 @@ def test_margins_flag_near_ties(oracle_mod):
         frac = 8 * r.alpha[t] - math.floor(8 * r.alpha[t])
         assert r.margin[t, 0] == pytest.approx(abs(frac - 0.5) / 8, abs=1e-15)
         assert (r.margin[t] >= 0).all()
+
+
+# --------------------------------------------------------------------------
+# The layer as a Transformer sublayer (Sec. B.1) and upcycled experts
+# (Sec. III)
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("eps", [0.0, 1e-5, 0.3])
+def test_layernorm_moments(oracle_mod, eps):
+    """With gamma = 1, beta = 0 every normalised row has mean 0 and variance
+    var / (var + eps), var the row's biased variance (closed form)."""
+    rng = np.random.default_rng(11)
+    d = 48
+    v = rng.standard_normal((40, d)) * rng.uniform(0.2, 3.0, (40, 1)) + rng.normal(0, 2, (40, 1))
+    out = oracle_mod.layernorm(v, np.ones(d), np.zeros(d), eps)
+    var = v.var(axis=1)  # numpy's default is the biased (1/d) variance
+    np.testing.assert_allclose(out.mean(axis=1), 0.0, atol=1e-12)
+    np.testing.assert_allclose(out.var(axis=1), var / (var + eps), rtol=1e-12)
+
+
+def test_layernorm_affine_constant_padding_rounding(oracle_mod):
+    """gamma and beta act after the normalisation; a constant row normalises
+    to beta; padding rows give 0; round_mode rounds to bf16 values."""
+    rng = np.random.default_rng(12)
+    d = 32
+    v = rng.standard_normal((6, d))
+    v[3] = 2.5  # constant row
+    g = rng.uniform(0.5, 2.0, d)
+    b = rng.standard_normal(d)
+    unit = oracle_mod.layernorm(v, np.ones(d), np.zeros(d), 1e-5)
+    out = oracle_mod.layernorm(v, g, b, 1e-5)
+    np.testing.assert_allclose(out, unit * g + b, rtol=1e-13, atol=1e-13)
+    np.testing.assert_array_equal(out[3], b)
+    mask = np.array([1, 1, 0, 1, 1, 1], np.uint8)
+    np.testing.assert_array_equal(oracle_mod.layernorm(v, g, b, 1e-5, mask)[2], 0.0)
+    r = oracle_mod.layernorm(v, g, b, 1e-5, round_mode=oracle_mod.ROUND_BF16)
+    import torch
+    as_bf16 = torch.tensor(out).to(torch.bfloat16).double().numpy()  # library rounding
+    np.testing.assert_array_equal(r, as_bf16)
+
+
+@pytest.mark.parametrize("norm_first", [True, False])
+def test_sublayer_with_silent_experts(oracle_mod, norm_first):
+    """Experts with zero up-projections output nothing (GeLU(0) = 0), so the
+    sublayer reduces to the residual path: x itself when normalised first,
+    LN(x) when normalised after the sum. Padding rows give 0."""
+    rng = np.random.default_rng(13)
+    d, H, K, B = 16, 32, 3, 4
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, T=20)
+    w_up[:] = 0.0
+    g = rng.uniform(0.5, 2.0, d)
+    b = rng.standard_normal(d)
+    mask = np.ones(20, np.uint8)
+    mask[[4, 9]] = 0
+    out, _ = oracle_mod.sublayer(x, w_router, w_up, w_down, B, g, b, 1e-5, norm_first, mask=mask)
+    ref = x if norm_first else oracle_mod.layernorm(x, g, b, 1e-5)
+    keep = mask == 1
+    np.testing.assert_allclose(out[keep], ref[keep], rtol=1e-13, atol=1e-13)
+    np.testing.assert_array_equal(out[~keep], 0.0)
+
+
+def test_sublayer_order_of_norm_and_residual(oracle_mod):
+    """Normalised first, the residual adds the raw input to the layer's output
+    on the normalised input; normalised after, the norm sees the sum. Both
+    against the layer oracle composed by hand."""
+    rng = np.random.default_rng(14)
+    d, H, K, B = 16, 32, 3, 4
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, T=24)
+    g = rng.uniform(0.5, 2.0, d)
+    b = rng.standard_normal(d)
+    pre, _ = oracle_mod.sublayer(x, w_router, w_up, w_down, B, g, b, 1e-5, True)
+    xn = oracle_mod.layernorm(x, g, b, 1e-5)
+    np.testing.assert_allclose(pre, x + oracle_mod.layer(xn, w_router, w_up, w_down, B)[0],
+                               rtol=1e-13, atol=1e-13)
+    post, _ = oracle_mod.sublayer(x, w_router, w_up, w_down, B, g, b, 1e-5, False)
+    y = oracle_mod.layer(x, w_router, w_up, w_down, B)[0]
+    np.testing.assert_allclose(post, oracle_mod.layernorm(x + y, g, b, 1e-5), rtol=1e-13,
+                               atol=1e-13)
+
+
+def test_upcycled_experts_closed_form(oracle_mod):
+    """Sec. III: experts upcycled from one dense FFN are identical, so the
+    layer output is alpha times the dense FFN's shared blocks plus P_k (the
+    selected residual mass) times its complementary blocks, whatever experts
+    were selected (block outputs by dense matrix products, GeLU from the
+    normal CDF)."""
+    rng = np.random.default_rng(15)
+    d, H, K, B = 24, 48, 4, 4
+    x, w_router, _, _ = rand_layer(rng, d, H, K, B, T=40)
+    w1 = rng.standard_normal((H, d)) / math.sqrt(d)
+    w2 = rng.standard_normal((d, H)) / math.sqrt(H)
+    wu, wd = oracle_mod.upcycle(w1, w2, K)
+    assert wu.shape == (K + 1, H, d) and wd.shape == (K + 1, d, H)
+    y, r = oracle_mod.layer(x, w_router, wu, wd, B)
+    Eb = block_outputs_dense(x, w1[None], w2[None], B)[:, 0]  # [T][B][d]
+    for t in range(x.shape[0]):
+        shr = [(int(r.shr_mask[t]) >> blk) & 1 for blk in range(B)]
+        Pk = float(np.sum(r.p[t, :r.k[t]]))
+        ref = sum(r.alpha[t] * Eb[t, blk] if shr[blk] else Pk * Eb[t, blk] for blk in range(B))
+        np.testing.assert_allclose(y[t], ref, rtol=1e-12, atol=1e-12)
