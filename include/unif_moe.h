@@ -98,6 +98,19 @@ UNIF_MOE_API int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_e
 UNIF_MOE_API int unif_moe_load_weights(unif_moe_t h, const void* w_router_dev, const void* w_up_dev,
                           const void* w_down_dev, const float* router_bias_dev, void* stream);
 
+/* Upcycling (Sec. III: all experts start from the same dense FFN): loads the
+ * dense FFN's projections into every expert, the shared one and the K
+ * residual ones, then the router as unif_moe_load_weights does:
+ *   w_router_dev    [d][K+1]  as in unif_moe_load_weights
+ *   w_up_dense_dev  [H][d]    the dense FFN's keys, copied to every expert
+ *   w_down_dense_dev [d][H]   the dense FFN's values, copied to every expert
+ *   router_bias_dev [K+1] float or NULL
+ * Layer dtype, device memory; copied, so the caller may free its buffers
+ * once `stream` has passed this call. Errors: ERR_ARG (NULL weight), ERR_CUDA. */
+UNIF_MOE_API int unif_moe_load_upcycled(unif_moe_t h, const void* w_router_dev,
+                                        const void* w_up_dense_dev, const void* w_down_dense_dev,
+                                        const float* router_bias_dev, void* stream);
+
 /* One forward pass over T tokens (Eqs. 17-30):
  *   x_dev   [T][d] input tokens
  *   out_dev [T][d] output y (layer dtype); padding tokens give 0
@@ -112,6 +125,26 @@ UNIF_MOE_API int unif_moe_load_weights(unif_moe_t h, const void* w_router_dev, c
 UNIF_MOE_API int unif_moe_forward(unif_moe_t h, const void* x_dev, void* out_dev, int T,
                      const uint8_t* token_mask_dev, int32_t* shared_counts_dev,
                      int32_t* residual_counts_dev, void* stream);
+
+/* The layer as a Transformer sublayer, the way the paper's backbones hold
+ * the converted FFN layers (Appendix A, Architecture details: DeiT-S normalises first, BERT after
+ * the residual sum). With F the layer (Eqs. 16-30) and
+ * LN(v) = gamma (v - mean(v)) / sqrt(var(v) + eps) + beta over each token's
+ * d features (biased variance, fp32 statistics):
+ *   norm_first != 0:  out = x + F(LN(x)), LN(x) kept in the layer dtype
+ *   norm_first == 0:  out = LN(x + F(x))
+ * ln_gamma_dev, ln_beta_dev [d] in the layer dtype (device); eps >= 0.
+ * Padding tokens (mask 0) give 0. The routing decisions and counts are
+ * those of F's input. x, out, counts, mask and errors as unif_moe_forward;
+ * also ERR_ARG (NULL gamma or beta, bad eps), ERR_SHAPE (d > 1024). A
+ * norm-first call allocates a [max_tokens][d] buffer for LN(x) on first
+ * use. */
+UNIF_MOE_API int unif_moe_sublayer_forward(unif_moe_t h, const void* x_dev, void* out_dev, int T,
+                                           const uint8_t* token_mask_dev,
+                                           int32_t* shared_counts_dev,
+                                           int32_t* residual_counts_dev, const void* ln_gamma_dev,
+                                           const void* ln_beta_dev, float eps, int norm_first,
+                                           void* stream);
 
 /* The same forward from host buffers: copies x_host (and token_mask_host if
  * not NULL) to the handle's device staging buffers, runs the forward, copies

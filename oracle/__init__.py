@@ -11,7 +11,7 @@ arrays in and out with ctypes, and chains the steps:
 `groups` lists the (expert, block) pairs the output sums over, grouped by
 pair (the bookkeeping behind Eq. 35). `upcycle` and `sublayer` place the
 layer the way the paper's backbones use it (Sec. III: experts initialised
-from one dense FFN; Sec. B.1: converted FFN layers of DeiT-S, normalised
+from one dense FFN; Appendix A, Architecture details: converted FFN layers of DeiT-S, normalised
 first, and of BERT, normalised after the residual sum).
 """
 from __future__ import annotations
@@ -268,7 +268,7 @@ def upcycle(w_up_dense, w_down_dense, K: int):
 def sublayer(x, w_router, w_up, w_down, B: int, gamma, beta, eps: float, norm_first: bool,
              th: Optional[Thresholds] = None, mask=None, bias=None,
              round_mode: int = ROUND_NONE):
-    """The layer as a Transformer sublayer (Sec. B.1 backbones):
+    """The layer as a Transformer sublayer (backbones of Appendix A, Architecture details):
     norm_first (DeiT-S): out = x + F(LN(x)), LN(x) kept in the layer's input
     precision (round_mode); otherwise (BERT): out = LN(x + F(x)). Padding
     tokens give 0. Returns (out [T][d], Routing)."""

@@ -334,8 +334,8 @@ long long oracle_groups(int T, int K, int B, const uint8_t* mask, const double* 
 }
 
 /* The layer inside a Transformer sublayer (the converted FFN layers of the
- * paper's DeiT-S and BERT backbones, Sec. B.1): layer normalisation of each
- * token over its d features, in the standard form
+ * paper's DeiT-S and BERT backbones, Appendix A, Architecture details):
+ * layer normalisation of each token over its d features, in the standard form
  *   LN(v) = gamma * (v - mean(v)) / sqrt(var(v) + eps) + beta,
  * mean and var over the d features, var the biased (1/d) second central
  * moment. Rows whose mask entry is 0 (padding) give 0. The result is

@@ -29,7 +29,8 @@ ERR = {0: "OK", -1: "ERR_ARG", -2: "ERR_SHAPE", -3: "ERR_CAPACITY", -4: "ERR_CUD
 
 # Every symbol include/unif_moe.h declares.
 EXPORTS = ["unif_moe_default_thresholds", "unif_moe_create", "unif_moe_load_weights",
-           "unif_moe_forward", "unif_moe_forward_host", "unif_moe_get_routing",
+           "unif_moe_load_upcycled", "unif_moe_forward", "unif_moe_sublayer_forward",
+           "unif_moe_forward_host", "unif_moe_get_routing",
            "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_kernels_per_forward",
            "unif_moe_set_stage_events",
            "unif_moe_sync_status", "unif_moe_selftest_timeout", "unif_moe_group_noalloc",
@@ -63,6 +64,8 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_create.argtypes = [C.POINTER(P), I, I, I, I, C.POINTER(Thresholds), I, I]
         L.unif_moe_load_weights.argtypes = [P, P, P, P, P, P]
         L.unif_moe_forward.argtypes = [P, P, P, I, P, P, P, P]
+        L.unif_moe_load_upcycled.argtypes = [P, P, P, P, P, P]
+        L.unif_moe_sublayer_forward.argtypes = [P, P, P, I, P, P, P, P, P, C.c_float, I, P]
         L.unif_moe_forward_host.argtypes = [P, P, P, I, P, P, P, P]
         L.unif_moe_get_routing.argtypes = [P, P, P, P, P, P, P]
         L.unif_moe_get_groups.argtypes = [P, P, P, P, P, C.POINTER(C.c_int64), P]
@@ -139,6 +142,36 @@ class Layer:
         self._keep = (w_router, w_up, w_down, router_bias)  # alive until the copy ran
         _check(lib().unif_moe_load_weights(self._h, _ptr(w_router), _ptr(w_up), _ptr(w_down),
                                            _ptr(router_bias), _stream(stream)))
+
+    def load_upcycled(self, w_router: torch.Tensor, w_up_dense: torch.Tensor,
+                      w_down_dense: torch.Tensor, router_bias: Optional[torch.Tensor] = None,
+                      stream=None):
+        """Every expert starts as the dense FFN (w_up_dense [H][d], w_down_dense [d][H])."""
+        for t in (w_router, w_up_dense, w_down_dense):
+            assert t.is_cuda and t.dtype == self.torch_dtype and t.is_contiguous()
+        if router_bias is not None:
+            assert router_bias.is_cuda and router_bias.dtype == torch.float32
+        self._keep = (w_router, w_up_dense, w_down_dense, router_bias)
+        _check(lib().unif_moe_load_upcycled(self._h, _ptr(w_router), _ptr(w_up_dense),
+                                            _ptr(w_down_dense), _ptr(router_bias),
+                                            _stream(stream)))
+
+    def sublayer_forward(self, x: torch.Tensor, ln_gamma: torch.Tensor, ln_beta: torch.Tensor,
+                         eps: float, norm_first: bool, out: Optional[torch.Tensor] = None,
+                         mask: Optional[torch.Tensor] = None,
+                         shared_counts: Optional[torch.Tensor] = None,
+                         residual_counts: Optional[torch.Tensor] = None,
+                         stream=None) -> torch.Tensor:
+        """x + F(LN(x)) (norm_first) or LN(x + F(x)), F this layer."""
+        T = x.shape[0]
+        if out is None:
+            out = torch.empty_like(x)
+        _check(lib().unif_moe_sublayer_forward(self._h, _ptr(x), _ptr(out), T, _ptr(mask),
+                                               _ptr(shared_counts), _ptr(residual_counts),
+                                               _ptr(ln_gamma), _ptr(ln_beta), float(eps),
+                                               1 if norm_first else 0, _stream(stream)))
+        self.last_T = T
+        return out
 
     def forward(self, x: torch.Tensor, out: Optional[torch.Tensor] = None,
                 mask: Optional[torch.Tensor] = None, shared_counts: Optional[torch.Tensor] = None,

@@ -74,6 +74,7 @@ struct Workspace {
   void* hbuf = nullptr;          // [max_rows][M] (layer dtype)
   float* y32 = nullptr;          // [max_tokens][d]
   // Host-buffer forward staging.
+  void* xn = nullptr;             // [max_tokens][d] LN(x) of a norm-first sublayer (on first use)
   void* x_stage = nullptr;
   void* out_stage = nullptr;
   uint8_t* mask_stage = nullptr;
@@ -144,6 +145,12 @@ cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask,
                           int32_t* b_out, int32_t* k_out, cudaStream_t s);
 cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s);
 cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s);
+cudaError_t launch_layernorm(unif_moe_layer* L, const void* x, void* out, const uint8_t* mask,
+                             const void* gamma, const void* beta, float eps, int T,
+                             cudaStream_t s);
+cudaError_t launch_combine_residual(unif_moe_layer* L, const void* x, void* out,
+                                    const uint8_t* mask, const void* gamma, const void* beta,
+                                    float eps, bool norm, int T, cudaStream_t s);
 // Tile list from the router's group sizes, for streaming grouped GEMMs.
 cudaError_t launch_tile_list(unif_moe_layer* L, cudaStream_t s);
 cudaError_t launch_sort_affinities(unif_moe_layer* L, int T, int32_t* q, float* p,

@@ -11,6 +11,8 @@
 //   combine : casts the fp32 accumulator of Eq. 30 to the layer dtype.
 #include <math.h>
 
+#include <algorithm>
+
 #include "decide.cuh"
 #include "internal.cuh"
 
@@ -543,6 +545,111 @@ __global__ void cast_out_bf16(float4* __restrict__ y, uint2* __restrict__ out, s
   }
 }
 
+// ---------------------------------------------------------------------------
+// The layer as a Transformer sublayer (converted FFN layers of the paper's
+// DeiT-S and BERT backbones, Appendix A, Architecture details): layer
+// normalisation LN(v) = gamma (v - mean) / sqrt(var + eps) + beta over each token's d
+// features (fp32 statistics: the mean, then the biased variance of the
+// centred values), and the residual sum. One warp per token row; a lane
+// keeps the row's features lane, lane + 32, ... (d <= 1024) in registers.
+// ---------------------------------------------------------------------------
+constexpr int kRowMax = 32;  // features per lane: d <= 32 * kRowMax
+
+template <typename T> __device__ __forceinline__ T from_f32(float v);
+template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) {
+  return __float2bfloat16_rn(v);
+}
+
+// In place: v[0 .. d) of this lane's features -> LN(v) (the whole warp calls).
+template <typename T>
+__device__ __forceinline__ void layernorm_warp(float (&v)[kRowMax], int d, int lane,
+                                               const T* __restrict__ gamma,
+                                               const T* __restrict__ beta, float eps) {
+  float sum = 0.f;
+#pragma unroll
+  for (int j = 0; j < kRowMax; ++j)
+    if (j * 32 + lane < d) sum += v[j];
+  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  const float mean = sum / (float)d;
+  float sq = 0.f;
+#pragma unroll
+  for (int j = 0; j < kRowMax; ++j)
+    if (j * 32 + lane < d) sq += (v[j] - mean) * (v[j] - mean);
+  for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+  const float inv = 1.0f / sqrtf(sq / (float)d + eps);
+#pragma unroll
+  for (int j = 0; j < kRowMax; ++j) {
+    const int i = j * 32 + lane;
+    if (i < d) v[j] = to_f32(gamma[i]) * ((v[j] - mean) * inv) + to_f32(beta[i]);
+  }
+}
+
+// out = LN(x), rows of padding (mask 0) give 0.
+template <typename T>
+__global__ void __launch_bounds__(256)
+layernorm_rows(const T* __restrict__ x, T* __restrict__ out, const uint8_t* __restrict__ mask,
+               const T* __restrict__ gamma, const T* __restrict__ beta, float eps, int n_rows,
+               int d) {
+  const int lane = threadIdx.x & 31;
+  const int warps = gridDim.x * (blockDim.x >> 5);
+  for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n_rows; r += warps) {
+    const size_t base = (size_t)r * d;
+    const bool pad = mask != nullptr && mask[r] == 0;
+    float v[kRowMax];
+#pragma unroll
+    for (int j = 0; j < kRowMax; ++j) {
+      const int i = j * 32 + lane;
+      v[j] = (i < d && !pad) ? to_f32(x[base + i]) : 0.f;
+    }
+    if (!pad) layernorm_warp<T>(v, d, lane, gamma, beta, eps);
+#pragma unroll
+    for (int j = 0; j < kRowMax; ++j) {
+      const int i = j * 32 + lane;
+      if (i < d) out[base + i] = from_f32<T>(pad ? 0.f : v[j]);
+    }
+  }
+}
+
+// The sublayer's combine: v = y + x (accumulator row plus the residual
+// input), out = LN(v) (NORM) or v; padding rows give 0. Zeroes the
+// accumulator rows and, in block 0, hands the group sizes on and zeroes the
+// grouping counters, as cast_out_bf16 does.
+template <typename T, bool NORM>
+__global__ void __launch_bounds__(256)
+combine_residual(float* __restrict__ y, const T* __restrict__ x, T* __restrict__ out,
+                 const uint8_t* __restrict__ mask, const T* __restrict__ gamma,
+                 const T* __restrict__ beta, float eps, int n_rows, int d, int32_t* fill,
+                 int32_t* counts, int n_fill, int region) {
+  grid_dep_wait();  // the down projection's sums are complete
+  if (blockIdx.x == 0)
+    for (int i = threadIdx.x; i < n_fill; i += blockDim.x) {
+      counts[i] = min(fill[i], region);
+      fill[i] = 0;
+    }
+  const int lane = threadIdx.x & 31;
+  const int warps = gridDim.x * (blockDim.x >> 5);
+  for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n_rows; r += warps) {
+    const size_t base = (size_t)r * d;
+    const bool pad = mask != nullptr && mask[r] == 0;
+    float v[kRowMax];
+#pragma unroll
+    for (int j = 0; j < kRowMax; ++j) {
+      const int i = j * 32 + lane;
+      v[j] = (i < d && !pad) ? y[base + i] + to_f32(x[base + i]) : 0.f;
+    }
+    if (NORM && !pad) layernorm_warp<T>(v, d, lane, gamma, beta, eps);
+#pragma unroll
+    for (int j = 0; j < kRowMax; ++j) {
+      const int i = j * 32 + lane;
+      if (i < d) {
+        out[base + i] = from_f32<T>(pad ? 0.f : v[j]);
+        y[base + i] = 0.f;
+      }
+    }
+  }
+}
+
 __global__ void copy_out_f32(float4* __restrict__ y, float4* __restrict__ out, size_t n4) {
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4;
        i += (size_t)gridDim.x * blockDim.x) {
@@ -668,6 +775,43 @@ cudaError_t launch_tile_list(unif_moe_layer* L, cudaStream_t s) {
   tile_list_kernel<<<1, 256, sizeof(int32_t) * (2 * (size_t)L->G + 1), s>>>(
       w.grp_fill, L->G, L->region_rows, w.n_tiles, w.tile_group, w.tile_row0, w.tile_rows);
   return cudaGetLastError();
+}
+
+cudaError_t launch_layernorm(unif_moe_layer* L, const void* x, void* out, const uint8_t* mask,
+                             const void* gamma, const void* beta, float eps, int T,
+                             cudaStream_t s) {
+  const int grid = std::min((T + 7) / 8, L->n_sm * 8);
+  if (L->dtype == UNIF_MOE_BF16)
+    layernorm_rows<__nv_bfloat16><<<grid, 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(x), static_cast<__nv_bfloat16*>(out), mask,
+        static_cast<const __nv_bfloat16*>(gamma), static_cast<const __nv_bfloat16*>(beta), eps, T,
+        L->d);
+  else
+    layernorm_rows<float><<<grid, 256, 0, s>>>(
+        static_cast<const float*>(x), static_cast<float*>(out), mask,
+        static_cast<const float*>(gamma), static_cast<const float*>(beta), eps, T, L->d);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine_residual(unif_moe_layer* L, const void* x, void* out,
+                                    const uint8_t* mask, const void* gamma, const void* beta,
+                                    float eps, bool norm, int T, cudaStream_t s) {
+  const int grid = std::min((T + 7) / 8, L->n_sm * 8);
+  const int n_fill = L->fused_group ? L->G : 0;
+  float* y = L->ws.y32;
+  if (L->dtype == UNIF_MOE_BF16) {
+    using B = __nv_bfloat16;
+    auto k = norm ? combine_residual<B, true> : combine_residual<B, false>;
+    return launch_dependent(k, dim3(grid), dim3(256), 0, s, y, static_cast<const B*>(x),
+                            static_cast<B*>(out), mask, static_cast<const B*>(gamma),
+                            static_cast<const B*>(beta), eps, T, L->d, L->ws.grp_fill,
+                            L->ws.grp_cnt, n_fill, L->region_rows);
+  }
+  auto k = norm ? combine_residual<float, true> : combine_residual<float, false>;
+  return launch_dependent(k, dim3(grid), dim3(256), 0, s, y, static_cast<const float*>(x),
+                          static_cast<float*>(out), mask, static_cast<const float*>(gamma),
+                          static_cast<const float*>(beta), eps, T, L->d, L->ws.grp_fill,
+                          L->ws.grp_cnt, n_fill, L->region_rows);
 }
 
 cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s) {

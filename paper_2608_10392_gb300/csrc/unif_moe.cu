@@ -68,7 +68,7 @@ void free_all(unif_moe_layer* L) {
                   L->ws.shr_mask, L->ws.exp_mask, L->ws.s, L->ws.chunk_cnt,
                   L->ws.grp_cnt, L->ws.grp_off, L->ws.n_tiles, L->ws.tile_group,
                   L->ws.tile_row0, L->ws.row_tok, L->ws.row_w, L->ws.hbuf, L->ws.y32,
-                  L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
+                  L->ws.xn, L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
                   L->ws.k_stage, L->ws.status, L->ws.grp_fill,
                   L->ws.tile_rows};
   for (void* q : ptrs)
@@ -239,9 +239,18 @@ int unif_moe_load_weights(unif_moe_t L, const void* w_router, const void* w_up,
   return UNIF_MOE_OK;
 }
 
-int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_t* token_mask,
-                     int32_t* shared_counts, int32_t* residual_counts, void* stream) {
-  unif::g_err[0] = 0;
+// The residual epilogue of a Transformer sublayer: out = res + y, then LN
+// when `norm` (the layer's combine otherwise).
+struct SublayerEpilogue {
+  const void* res;
+  const void* gamma;
+  const void* beta;
+  float eps;
+  bool norm;
+};
+
+static int forward_checks(unif_moe_t L, const void* x, void* out, int T,
+                          int32_t* shared_counts, int32_t* residual_counts) {
   if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
   if (T < 0) { set_error("T < 0"); return UNIF_MOE_ERR_ARG; }
   if (T > L->max_tokens) {
@@ -259,8 +268,14 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
     set_error("count buffers must be 16-byte aligned");
     return UNIF_MOE_ERR_ARG;
   }
-  DeviceGuard dg(L->device);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  return UNIF_MOE_OK;
+}
+
+// The forward after the argument checks (T > 0); `sub` replaces the combine
+// with a sublayer's residual epilogue.
+static int forward_core(unif_moe_t L, const void* x, void* out, int T, const uint8_t* token_mask,
+                        int32_t* shared_counts, int32_t* residual_counts, cudaStream_t s,
+                        const SublayerEpilogue* sub) {
   cudaEvent_t* ev = L->stage_ev;
   // The output accumulator and the grouping counters are all zero between
   // forwards (each combine zeroes them). A forward that returned before
@@ -286,11 +301,74 @@ int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_
     CK(unif::launch_gemms_simt(L, x, T, ev[3], s));
   }
   if (ev[4]) CK(cudaEventRecord(ev[4], s));
-  CK(unif::launch_combine(L, out, T, s));
+  if (sub)
+    CK(unif::launch_combine_residual(L, sub->res, out, token_mask, sub->gamma, sub->beta,
+                                     sub->eps, sub->norm, T, s));
+  else
+    CK(unif::launch_combine(L, out, T, s));
   L->y_dirty = false;
   if (ev[5]) CK(cudaEventRecord(ev[5], s));
   L->last_T = T;
   return UNIF_MOE_OK;
+}
+
+int unif_moe_load_upcycled(unif_moe_t L, const void* w_router, const void* w_up_dense,
+                           const void* w_down_dense, const float* router_bias, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L || !w_router || !w_up_dense || !w_down_dense) {
+    set_error("NULL handle or weight");
+    return UNIF_MOE_ERR_ARG;
+  }
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // every expert, the shared one and the K residual ones, starts as the
+  // dense FFN: K + 1 copies of each projection
+  const size_t bytes = elt_size(L) * (size_t)L->H * L->d;
+  for (int e = 0; e <= L->K; ++e) {
+    CK(cudaMemcpyAsync(static_cast<char*>(L->w_up) + e * bytes, w_up_dense, bytes,
+                       cudaMemcpyDeviceToDevice, s));
+    CK(cudaMemcpyAsync(static_cast<char*>(L->w_down) + e * bytes, w_down_dense, bytes,
+                       cudaMemcpyDeviceToDevice, s));
+  }
+  CK(unif::launch_prototypes(L, w_router, router_bias, s));
+  L->loaded = true;
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_t* token_mask,
+                     int32_t* shared_counts, int32_t* residual_counts, void* stream) {
+  unif::g_err[0] = 0;
+  const int rc = forward_checks(L, x, out, T, shared_counts, residual_counts);
+  if (rc != UNIF_MOE_OK || T == 0) return rc;
+  DeviceGuard dg(L->device);
+  return forward_core(L, x, out, T, token_mask, shared_counts, residual_counts,
+                      static_cast<cudaStream_t>(stream), nullptr);
+}
+
+int unif_moe_sublayer_forward(unif_moe_t L, const void* x, void* out, int T,
+                              const uint8_t* token_mask, int32_t* shared_counts,
+                              int32_t* residual_counts, const void* ln_gamma,
+                              const void* ln_beta, float eps, int norm_first, void* stream) {
+  unif::g_err[0] = 0;
+  const int rc = forward_checks(L, x, out, T, shared_counts, residual_counts);
+  if (rc != UNIF_MOE_OK) return rc;
+  if (!ln_gamma || !ln_beta) { set_error("ln_gamma or ln_beta is NULL"); return UNIF_MOE_ERR_ARG; }
+  if (!(eps >= 0.f) || !isfinite(eps)) { set_error("eps must be finite and >= 0"); return UNIF_MOE_ERR_ARG; }
+  if (L->d > 1024) { set_error("the sublayer needs d <= 1024 (d=%d)", L->d); return UNIF_MOE_ERR_SHAPE; }
+  if (T == 0) return UNIF_MOE_OK;
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const SublayerEpilogue sub{x, ln_gamma, ln_beta, eps, !norm_first};
+  if (!norm_first)  // out = LN(x + F(x))
+    return forward_core(L, x, out, T, token_mask, shared_counts, residual_counts, s, &sub);
+  // out = x + F(LN(x)); LN(x) in the layer dtype, in a buffer made on first use
+  if (!L->ws.xn) {
+    const int arc = dalloc(reinterpret_cast<char**>(&L->ws.xn),
+                           elt_size(L) * (size_t)L->max_tokens * L->d);
+    if (arc != UNIF_MOE_OK) return arc;
+  }
+  CK(unif::launch_layernorm(L, x, L->ws.xn, token_mask, ln_gamma, ln_beta, eps, T, s));
+  return forward_core(L, L->ws.xn, out, T, token_mask, shared_counts, residual_counts, s, &sub);
 }
 
 // The device address of pinned, mapped host memory (nullptr for any other

@@ -82,6 +82,9 @@ def test_argument_errors_without_gpu(lib):
     assert lib.unif_moe_create(C.byref(h), 64, 256, 4, 4, C.byref(bad), 1, 16) == -1
     assert lib.unif_moe_forward(None, None, None, 4, None, None, None, None) == -1
     assert lib.unif_moe_load_weights(None, None, None, None, None, None) == -1
+    assert lib.unif_moe_load_upcycled(None, None, None, None, None, None) == -1
+    assert lib.unif_moe_sublayer_forward(None, None, None, 4, None, None, None, None, None,
+                                         1e-5, 1, None) == -1
     assert lib.unif_moe_sync_status(None, None) == -1
     assert lib.unif_moe_max_rows(None) == -1
     assert lib.unif_moe_kernels_per_forward(None) == -1

@@ -396,7 +396,7 @@ def test_margins_flag_near_ties(oracle_mod):
 
 
 # --------------------------------------------------------------------------
-# The layer as a Transformer sublayer (Sec. B.1) and upcycled experts
+# The layer as a Transformer sublayer (Appendix A, Architecture details) and upcycled experts
 # (Sec. III)
 # --------------------------------------------------------------------------
 
