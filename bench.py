@@ -278,6 +278,9 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=50)
     ap.add_argument("--routing", default="adaptive", choices=sorted(ROUTINGS),
                     help="routing variant (Table IV ablations, fixed thresholds)")
+    ap.add_argument("--sublayer", default="none", choices=["none", "pre", "post"],
+                    help="time the layer inside a Transformer sublayer: x + F(LN(x)) (pre) or "
+                         "LN(x + F(x)) (post), seeded LayerNorm parameters")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -330,8 +333,19 @@ def main():
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
     flush_r = torch.zeros(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
 
+    if args.sublayer == "none":
+        def step():
+            layer.forward(xd, out=out, mask=md, shared_counts=bcnt, residual_counts=kcnt)
+    else:
+        gen = torch.Generator().manual_seed(7)
+        ln_g = (0.5 + torch.rand(s.d_model, generator=gen)).to(xd.dtype).to(dev)
+        ln_b = (0.1 * torch.randn(s.d_model, generator=gen)).to(xd.dtype).to(dev)
+
+        def step():
+            layer.sublayer_forward(xd, ln_g, ln_b, 1e-5, args.sublayer == "pre", out=out,
+                                   mask=md, shared_counts=bcnt, residual_counts=kcnt)
     for _ in range(args.warmup):
-        layer.forward(xd, out=out, mask=md, shared_counts=bcnt, residual_counts=kcnt)
+        step()
     torch.cuda.synchronize(dev)
     if layer.sync_status() != 0:
         raise RuntimeError("device status word set during warm-up")
@@ -362,7 +376,7 @@ def main():
         flush.zero_()  # L2 flush between steps (outside the timed events)
         flush_r.max()
         starts[i].record(stream)
-        layer.forward(xd, out=out, mask=md, shared_counts=bcnt, residual_counts=kcnt)
+        step()
         ends[i].record(stream)
     torch.cuda.synchronize(dev)
     if dist:
@@ -378,7 +392,7 @@ def main():
         flush.zero_()
         flush_r.max()
         layer.set_stage_events(stage_ev[i])
-        layer.forward(xd, out=out, mask=md, shared_counts=bcnt, residual_counts=kcnt)
+        step()
     torch.cuda.synchronize(dev)
     layer.set_stage_events(None)
 
@@ -399,7 +413,9 @@ def main():
     for _ in range(3):
         layer.forward_host(xh, oh, mh, bh, kh)
     e2e_ms = []
-    for _ in range(args.e2e_steps):
+    # (the host-buffer entry point runs the layer alone: no end-to-end line
+    # for a sublayer run)
+    for _ in range(args.e2e_steps if args.sublayer == "none" else 0):
         a, b = mk(), mk()
         a.record(stream)
         layer.forward_host(xh, oh, mh, bh, kh)
@@ -451,6 +467,9 @@ def main():
         "vs_baseline": None, "dtype": s.dtype, "data": "synthetic (seeded; stands in for DeiT-S "
         "tokens on DomainBed, which are not available)",
         "config": dict(workload_desc(s, T_valid), parallelism="dp%d (independent batches)" % world,
+                       sublayer={"none": "no (the layer alone)",
+                                 "pre": "x + F(LN(x)), LN eps 1e-5",
+                                 "post": "LN(x + F(x)), LN eps 1e-5"}[args.sublayer],
                        l2="flushed between steps (512 MB write + 256 MB read, outside the "
                           "timed events)"),
         "activated_tflops": tflops,

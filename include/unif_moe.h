@@ -136,7 +136,8 @@ UNIF_MOE_API int unif_moe_forward(unif_moe_t h, const void* x_dev, void* out_dev
  * ln_gamma_dev, ln_beta_dev [d] in the layer dtype (device); eps >= 0.
  * Padding tokens (mask 0) give 0. The routing decisions and counts are
  * those of F's input. x, out, counts, mask and errors as unif_moe_forward;
- * also ERR_ARG (NULL gamma or beta, bad eps), ERR_SHAPE (d > 1024). A
+ * also ERR_ARG (NULL or not 16-byte aligned gamma or beta, bad eps),
+ * ERR_SHAPE (d > 1024 or not a multiple of 8). A
  * norm-first call allocates a [max_tokens][d] buffer for LN(x) on first
  * use. */
 UNIF_MOE_API int unif_moe_sublayer_forward(unif_moe_t h, const void* x_dev, void* out_dev, int T,

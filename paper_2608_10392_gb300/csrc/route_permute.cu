@@ -548,12 +548,13 @@ __global__ void cast_out_bf16(float4* __restrict__ y, uint2* __restrict__ out, s
 // ---------------------------------------------------------------------------
 // The layer as a Transformer sublayer (converted FFN layers of the paper's
 // DeiT-S and BERT backbones, Appendix A, Architecture details): layer
-// normalisation LN(v) = gamma (v - mean) / sqrt(var + eps) + beta over each token's d
-// features (fp32 statistics: the mean, then the biased variance of the
-// centred values), and the residual sum. One warp per token row; a lane
-// keeps the row's features lane, lane + 32, ... (d <= 1024) in registers.
+// normalisation LN(v) = gamma (v - mean) / sqrt(var + eps) + beta over each
+// token's d features (fp32 statistics: the mean, then the biased variance of
+// the centred values), and the residual sum. One warp per token row; lane l
+// keeps the row's 8-feature groups l, l + 32, ... (d a multiple of 8, at
+// most 1024) in registers and moves each group with 16-byte accesses.
 // ---------------------------------------------------------------------------
-constexpr int kRowMax = 32;  // features per lane: d <= 32 * kRowMax
+constexpr int kGroups = 4;  // 8-feature groups per lane: d <= 32 * 8 * kGroups
 
 template <typename T> __device__ __forceinline__ T from_f32(float v);
 template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
@@ -561,27 +562,53 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
   return __float2bfloat16_rn(v);
 }
 
-// In place: v[0 .. d) of this lane's features -> LN(v) (the whole warp calls).
+// (load8, the router's 8-value loader, reads the groups)
+__device__ __forceinline__ void store8(float* p, const float (&v)[8]) {
+  reinterpret_cast<float4*>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+  reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+__device__ __forceinline__ void store8(__nv_bfloat16* p, const float (&v)[8]) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    w[i] = *reinterpret_cast<uint32_t*>(&h);
+  }
+  *reinterpret_cast<uint4*>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// In place: this lane's groups of v (features 8 (32 j + lane) ..) -> LN(v);
+// the whole warp calls.
 template <typename T>
-__device__ __forceinline__ void layernorm_warp(float (&v)[kRowMax], int d, int lane,
+__device__ __forceinline__ void layernorm_warp(float (&v)[kGroups][8], int d, int lane,
                                                const T* __restrict__ gamma,
                                                const T* __restrict__ beta, float eps) {
   float sum = 0.f;
 #pragma unroll
-  for (int j = 0; j < kRowMax; ++j)
-    if (j * 32 + lane < d) sum += v[j];
+  for (int j = 0; j < kGroups; ++j)
+    if (8 * (32 * j + lane) < d)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) sum += v[j][i];
   for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
   const float mean = sum / (float)d;
   float sq = 0.f;
 #pragma unroll
-  for (int j = 0; j < kRowMax; ++j)
-    if (j * 32 + lane < d) sq += (v[j] - mean) * (v[j] - mean);
+  for (int j = 0; j < kGroups; ++j)
+    if (8 * (32 * j + lane) < d)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) sq += (v[j][i] - mean) * (v[j][i] - mean);
   for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
   const float inv = 1.0f / sqrtf(sq / (float)d + eps);
 #pragma unroll
-  for (int j = 0; j < kRowMax; ++j) {
-    const int i = j * 32 + lane;
-    if (i < d) v[j] = to_f32(gamma[i]) * ((v[j] - mean) * inv) + to_f32(beta[i]);
+  for (int j = 0; j < kGroups; ++j) {
+    const int f = 8 * (32 * j + lane);
+    if (f < d) {
+      float g[8], b[8];
+      load8(gamma + f, g);
+      load8(beta + f, b);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[j][i] = g[i] * ((v[j][i] - mean) * inv) + b[i];
+    }
   }
 }
 
@@ -596,17 +623,22 @@ layernorm_rows(const T* __restrict__ x, T* __restrict__ out, const uint8_t* __re
   for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n_rows; r += warps) {
     const size_t base = (size_t)r * d;
     const bool pad = mask != nullptr && mask[r] == 0;
-    float v[kRowMax];
+    float v[kGroups][8];
 #pragma unroll
-    for (int j = 0; j < kRowMax; ++j) {
-      const int i = j * 32 + lane;
-      v[j] = (i < d && !pad) ? to_f32(x[base + i]) : 0.f;
+    for (int j = 0; j < kGroups; ++j) {
+      const int f = 8 * (32 * j + lane);
+      if (f < d && !pad) {
+        load8(x + base + f, v[j]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[j][i] = 0.f;
+      }
     }
     if (!pad) layernorm_warp<T>(v, d, lane, gamma, beta, eps);
 #pragma unroll
-    for (int j = 0; j < kRowMax; ++j) {
-      const int i = j * 32 + lane;
-      if (i < d) out[base + i] = from_f32<T>(pad ? 0.f : v[j]);
+    for (int j = 0; j < kGroups; ++j) {
+      const int f = 8 * (32 * j + lane);
+      if (f < d) store8(out + base + f, v[j]);
     }
   }
 }
@@ -629,22 +661,32 @@ combine_residual(float* __restrict__ y, const T* __restrict__ x, T* __restrict__
     }
   const int lane = threadIdx.x & 31;
   const int warps = gridDim.x * (blockDim.x >> 5);
+  const float zero[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n_rows; r += warps) {
     const size_t base = (size_t)r * d;
     const bool pad = mask != nullptr && mask[r] == 0;
-    float v[kRowMax];
+    float v[kGroups][8];
 #pragma unroll
-    for (int j = 0; j < kRowMax; ++j) {
-      const int i = j * 32 + lane;
-      v[j] = (i < d && !pad) ? y[base + i] + to_f32(x[base + i]) : 0.f;
+    for (int j = 0; j < kGroups; ++j) {
+      const int f = 8 * (32 * j + lane);
+      if (f < d && !pad) {
+        float a[8];
+        load8(y + base + f, v[j]);
+        load8(x + base + f, a);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[j][i] += a[i];
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[j][i] = 0.f;
+      }
     }
     if (NORM && !pad) layernorm_warp<T>(v, d, lane, gamma, beta, eps);
 #pragma unroll
-    for (int j = 0; j < kRowMax; ++j) {
-      const int i = j * 32 + lane;
-      if (i < d) {
-        out[base + i] = from_f32<T>(pad ? 0.f : v[j]);
-        y[base + i] = 0.f;
+    for (int j = 0; j < kGroups; ++j) {
+      const int f = 8 * (32 * j + lane);
+      if (f < d) {
+        store8(out + base + f, v[j]);
+        store8(y + base + f, zero);
       }
     }
   }

@@ -354,7 +354,14 @@ int unif_moe_sublayer_forward(unif_moe_t L, const void* x, void* out, int T,
   if (rc != UNIF_MOE_OK) return rc;
   if (!ln_gamma || !ln_beta) { set_error("ln_gamma or ln_beta is NULL"); return UNIF_MOE_ERR_ARG; }
   if (!(eps >= 0.f) || !isfinite(eps)) { set_error("eps must be finite and >= 0"); return UNIF_MOE_ERR_ARG; }
-  if (L->d > 1024) { set_error("the sublayer needs d <= 1024 (d=%d)", L->d); return UNIF_MOE_ERR_SHAPE; }
+  if (!aligned16(ln_gamma) || !aligned16(ln_beta)) {
+    set_error("ln_gamma and ln_beta must be 16-byte aligned");
+    return UNIF_MOE_ERR_ARG;
+  }
+  if (L->d > 1024 || L->d % 8 != 0) {
+    set_error("the sublayer needs d <= 1024, a multiple of 8 (d=%d)", L->d);
+    return UNIF_MOE_ERR_SHAPE;
+  }
   if (T == 0) return UNIF_MOE_OK;
   DeviceGuard dg(L->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
