@@ -490,7 +490,8 @@ def main():
             "value": T_valid / (statistics.fmean(e2e_ms) / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": statistics.fmean(e2e_ms)},
-        "gpu_launches": layer.kernels_per_forward() * K,
+        # (a norm-first sublayer adds its layer-normalisation kernel)
+        "gpu_launches": (layer.kernels_per_forward() + (args.sublayer == "pre")) * K,
         "clocks": clocks,
     }
     if not args.no_cpu_baseline and world >= 1:
