@@ -154,3 +154,29 @@ def test_upcycled_experts():
     denom = np.abs(y_ref).max(axis=1)
     err = np.abs(out - y_ref).max(axis=1)
     assert float((err / np.maximum(denom, 1e-12)).max()) <= TOL["bf16"]
+
+
+def test_sublayer_argument_errors():
+    """Misaligned LayerNorm parameters and a bad eps are refused before any
+    launch, and the handle stays usable."""
+    from paper_2608_10392_gb300 import UnifMoeError
+    wl = workloads.make_workload(workloads.spec("vit_s", tokens=256))
+    s = wl.spec
+    dev = torch.device("cuda")
+    layer = make_layer(s)
+    layer.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
+    gamma, beta = ln_params(s.d_model, torch.bfloat16)
+    gd, bd = gamma.to(dev), beta.to(dev)
+    x = wl.x.to(dev)
+    shifted = torch.empty(s.d_model + 1, dtype=torch.bfloat16, device=dev)[1:]  # 2-byte offset
+    shifted.copy_(gd)
+    with pytest.raises(UnifMoeError) as e:
+        layer.sublayer_forward(x, shifted, bd, EPS, True)
+    assert e.value.code == -1
+    for eps in (-1.0, float("nan")):
+        with pytest.raises(UnifMoeError) as e:
+            layer.sublayer_forward(x, gd, bd, eps, False)
+        assert e.value.code == -1
+    out = layer.sublayer_forward(x, gd, bd, EPS, True)
+    torch.cuda.synchronize()
+    assert layer.sync_status() == 0 and torch.isfinite(out.float()).all()
