@@ -1,7 +1,8 @@
 """The pins must catch plausible mistakes in the oracle. Each case below
 plants one mistake in a copy of the oracle's C source (on the CPU, in a
 temporary directory), builds it, and runs the pin suite against it with the
-wrapper pointed at the broken library: at least one pin has to fail."""
+wrapper pointed at the broken library, or plants it in a copy of the Python
+wrapper and runs the pins next to it: at least one pin has to fail."""
 import os
 import shutil
 import subprocess
@@ -50,6 +51,35 @@ MUTANTS = {
     # beta scaled by gamma (the affine step applied before the shift)
     "ln_beta_scaled": ("o[i] = round_to(gamma[i] * (row[i] - mean) * inv + beta[i], round_mode);",
                        "o[i] = round_to(gamma[i] * ((row[i] - mean) * inv + beta[i]), round_mode);"),
+    # prefix block selection counted from the last block (Table IV: the first b)
+    "prefix_from_end": ("shr |= 1ull << (prefix_blocks ? r : uorder[r]);",
+                        "shr |= 1ull << (prefix_blocks ? B - 1 - r : uorder[r]);"),
+    # prefix switch ignored (prototype TopK always)
+    "prefix_ignored": ("shr |= 1ull << (prefix_blocks ? r : uorder[r]);",
+                       "shr |= 1ull << uorder[r];"),
+    # router bias left out of the logits
+    "bias_dropped": ("z[j] = acc + (bias ? bias[j] : 0.0);", "z[j] = acc;"),
+    # router bias added to the neighbouring column
+    "bias_wrong_column": ("z[j] = acc + (bias ? bias[j] : 0.0);",
+                          "z[j] = acc + (bias ? bias[(j + 1) % (K + 1)] : 0.0);"),
+    # margin (ii) measured from the top priority instead of the b-th
+    "margin_ii_wrong_rank": ("u[uorder[b - 1]] - u[uorder[b]]", "u[uorder[0]] - u[uorder[b]]"),
+    # margin (iii) with P_k in place of P_{k-1} on the lower side
+    "margin_iii_prefix": ("for (int i = 0; i < k - 1; ++i) prev += p[i];",
+                          "for (int i = 0; i < k; ++i) prev += p[i];"),
+    # margin (iii) one-sided (only the distance above beta)
+    "margin_iii_one_sided": ("mg[2] = fmin(P_k - beta, beta - prev);", "mg[2] = P_k - beta;"),
+}
+
+# Mistakes planted in the Python side of the oracle (oracle/__init__.py).
+PY_MUTANTS = {
+    # given experts listed by increasing affinity
+    "with_decisions_ascending": ("sel.sort(key=lambda j: (-r.s[t, j], j))",
+                                 "sel.sort(key=lambda j: (r.s[t, j], j))"),
+    # the unselected experts placed first, so the first k are the wrong ones
+    "with_decisions_rest_first": ("order = sel + rest", "order = rest + sel"),
+    # affinities left in expert order instead of following q
+    "with_decisions_p_unsorted": ("p[t] = r.s[t, order]", "p[t] = r.s[t]"),
 }
 
 
@@ -67,4 +97,39 @@ def test_pins_catch_mutant(name, tmp_path):
     res = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
                           os.path.join(ROOT, "tests", "test_oracle_pins.py")],
                          cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert res.returncode != 0, "no pin caught mutant %s:\n%s" % (name, res.stdout[-2000:])
+
+
+def run_pins_in_copy(tmp_path, old, new):
+    """Runs the pins in a tree of their own holding a copy of the oracle
+    package whose Python source has `old` replaced by `new`."""
+    src = open(os.path.join(ROOT, "oracle", "__init__.py")).read()
+    assert src.count(old) == 1, "mutation anchor not found: " + old
+    (tmp_path / "oracle").mkdir()
+    (tmp_path / "oracle" / "__init__.py").write_text(src.replace(old, new))
+    shutil.copy(SRC, tmp_path / "oracle" / "unif_moe_oracle.c")
+    (tmp_path / "tests").mkdir()
+    for f in ("conftest.py", "test_oracle_pins.py"):
+        shutil.copy(os.path.join(ROOT, "tests", f), tmp_path / "tests" / f)
+    shutil.copytree(os.path.join(ROOT, "tests", "golden"), tmp_path / "tests" / "golden")
+    env = dict(os.environ, OMP_NUM_THREADS="2")
+    env.pop("UNIF_MOE_ORACLE_LIB", None)
+    return subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+                           str(tmp_path / "tests" / "test_oracle_pins.py")],
+                          cwd=str(tmp_path), env=env, capture_output=True, text=True, timeout=600)
+
+
+def test_unmutated_copy_passes(tmp_path):
+    """Control for the Python mutants: the copied tree itself passes, so a
+    mutant's failure comes from its planted mistake."""
+    res = run_pins_in_copy(tmp_path, "order = sel + rest", "order = sel + rest")
+    assert res.returncode == 0, res.stdout[-2000:]
+
+
+@pytest.mark.parametrize("name", sorted(PY_MUTANTS))
+def test_pins_catch_python_mutant(name, tmp_path):
+    """The same check for the Python wrapper: a copy of the oracle package
+    with one planted mistake, next to copies of the pins."""
+    old, new = PY_MUTANTS[name]
+    res = run_pins_in_copy(tmp_path, old, new)
     assert res.returncode != 0, "no pin caught mutant %s:\n%s" % (name, res.stdout[-2000:])

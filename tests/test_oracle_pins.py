@@ -110,12 +110,14 @@ def test_hand_example_groups(oracle_mod):
 # Exhaustive search on tiny layers (Eqs. 18-30 by enumeration)
 # --------------------------------------------------------------------------
 
-def brute_force(x, w_router, w_up, w_down, B, th: Thresholds):
+def brute_force(x, w_router, w_up, w_down, B, th: Thresholds, bias=None):
     """Decisions by exhaustive search and the output as a masked sum of dense
     block outputs. No sorting: the shared set is the b-subset with the
-    largest total priority, the residual set the smallest subset of experts
-    whose affinity mass reaches beta (largest mass among subsets of that
-    size)."""
+    largest total priority (with prefix selection, Table IV, the blocks
+    0..b-1), the residual set the smallest subset of experts whose affinity
+    mass reaches beta (largest mass among subsets of that size; with a fixed
+    top-k, the k-subset of largest mass). `bias` is added to the router
+    logits x W* column by column."""
     T, d = x.shape
     K = w_up.shape[0] - 1
     H = w_up.shape[1]
@@ -125,18 +127,25 @@ def brute_force(x, w_router, w_up, w_down, B, th: Thresholds):
     blocks = block_outputs_dense(x, w_up, w_down, B)
     ys, bs, ks, shr_sets, exp_sets = [], [], [], [], []
     for t in range(T):
-        z = x[t] @ w_router
+        z = x[t] @ w_router + (0.0 if bias is None else bias)
         alpha = tau + (1 - 2 * tau) * expit(z[0]) if math.isnan(th.alpha_fixed) else th.alpha_fixed
         b = int(np.rint(B * alpha))
         u = mu @ x[t]
-        best = max(itertools.combinations(range(B), b), key=lambda S: sum(u[i] for i in S))
-        shr = set(best)
+        if th.prefix_blocks:
+            shr = set(range(b))
+        else:
+            best = max(itertools.combinations(range(B), b), key=lambda S: sum(u[i] for i in S))
+            shr = set(best)
         s = softmax(z[1:])
         beta = 1 - alpha if math.isnan(th.beta_fixed) else th.beta_fixed
         chosen = None
         for n in range(1, K + 1):
             S = max(itertools.combinations(range(K), n), key=lambda S: sum(s[j] for j in S))
-            if sum(s[j] for j in S) >= beta or n == K:
+            if th.topk_fixed:
+                if n == th.topk_fixed:
+                    chosen = S
+                    break
+            elif sum(s[j] for j in S) >= beta or n == K:
                 chosen = S
                 break
         y = alpha * sum(blocks[t, 0, blk] for blk in shr) if shr else np.zeros(d)
@@ -169,14 +178,130 @@ def test_brute_force_tiny(oracle_mod, d, H, K, B, seed):
 
 
 @pytest.mark.parametrize("th", [Thresholds(beta_fixed=0.7), Thresholds(alpha_fixed=0.4),
-                                Thresholds(tau=0.1)])
+                                Thresholds(tau=0.1), Thresholds(prefix_blocks=1),
+                                Thresholds(topk_fixed=2),
+                                Thresholds(prefix_blocks=1, topk_fixed=3, alpha_fixed=0.3)])
 def test_brute_force_threshold_variants(oracle_mod, th):
+    """The Table IV ablation switches (fixed alpha, fixed top-k, prefix block
+    selection) and the fixed thresholds, against exhaustive search."""
     rng = np.random.default_rng(7)
     x, w_router, w_up, w_down = rand_layer(rng, 6, 16, 4, 4, router_scale=3.0, T=40)
     y, r = oracle.layer(x, w_router, w_up, w_down, 4, th)
-    yb, bb, kb, _, _ = brute_force(x, w_router, w_up, w_down, 4, th)
+    yb, bb, kb, shr, exps = brute_force(x, w_router, w_up, w_down, 4, th)
     assert r.b.tolist() == bb.tolist() and r.k.tolist() == kb.tolist()
+    em = r.expert_mask()
+    for t in range(x.shape[0]):
+        assert {blk for blk in range(4) if (int(r.shr_mask[t]) >> blk) & 1} == shr[t]
+        assert {j for j in range(4) if (int(em[t]) >> j) & 1} == exps[t]
     np.testing.assert_allclose(y, yb, rtol=1e-11, atol=1e-13)
+
+
+def test_prefix_selection_ignores_priorities(oracle_mod):
+    """Prefix block selection (Table IV) shares blocks 0..b-1 even when the
+    priorities rank the last blocks highest; the default TopK picks those."""
+    d, H, K, B = 4, 8, 2, 8
+    x = np.array([[1.0, 0.0, 0.0, 0.0]])
+    w_router = np.zeros((d, K + 1))
+    w_up = np.zeros((K + 1, H, d))
+    w_up[0, :, 0] = np.arange(H, dtype=np.float64)  # M = 1: u_b = b, last blocks first
+    w_down = np.zeros((K + 1, d, H))
+    th = Thresholds(alpha_fixed=0.375)  # b = 3
+    _, r = oracle.layer(x, w_router, w_up, w_down, B, th)
+    assert r.b[0] == 3 and int(r.shr_mask[0]) == 0b11100000
+    _, rp = oracle.layer(x, w_router, w_up, w_down, B,
+                         Thresholds(alpha_fixed=0.375, prefix_blocks=1))
+    assert rp.b[0] == 3 and int(rp.shr_mask[0]) == 0b00000111
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_router_bias_brute_force(oracle_mod, seed):
+    """A bias per router column enters the logits before Eqs. 18 and 24:
+    decisions and output against exhaustive search with the bias added to
+    x W* by a dense product."""
+    rng = np.random.default_rng(40 + seed)
+    K, B = 4, 4
+    x, w_router, w_up, w_down = rand_layer(rng, 6, 16, K, B, router_scale=2.0, T=40)
+    bias = rng.normal(0.0, 1.5, K + 1)
+    y, r = oracle.layer(x, w_router, w_up, w_down, B, bias=bias)
+    yb, bb, kb, shr, exps = brute_force(x, w_router, w_up, w_down, B, Thresholds(), bias=bias)
+    assert r.b.tolist() == bb.tolist() and r.k.tolist() == kb.tolist()
+    em = r.expert_mask()
+    for t in range(x.shape[0]):
+        assert {j for j in range(K) if (int(em[t]) >> j) & 1} == exps[t]
+    np.testing.assert_allclose(y, yb, rtol=1e-11, atol=1e-13)
+    # the bias changes decisions here (it is not a no-op on this layer)
+    _, r0 = oracle.layer(x, w_router, w_up, w_down, B)
+    assert (r0.k != r.k).any() or (r0.b != r.b).any()
+
+
+@pytest.mark.parametrize("j", [0, 2])
+def test_router_bias_closed_form(oracle_mod, j):
+    """A large bias on one residual expert's column makes its affinity 1 (to
+    rounding), so it alone is selected: k = 1, q_1 = j (Eqs. 24-27). A large
+    bias on the shared column drives alpha to its bounds tau and 1 - tau
+    (Eq. 18): with B = 4, tau = 3/16, b = round(4 * 13/16) = 3 or
+    round(4 * 3/16) = 1."""
+    rng = np.random.default_rng(3)
+    K, B = 3, 4
+    x, w_router, w_up, w_down = rand_layer(rng, 8, 16, K, B, T=30)
+    for sign, b_want in ((1.0, 3), (-1.0, 1)):
+        bias = np.zeros(K + 1)
+        bias[0] = 60.0 * sign
+        bias[1 + j] = 60.0
+        _, r = oracle.layer(x, w_router, w_up, w_down, B, bias=bias)
+        assert (r.k == 1).all() and (r.q[:, 0] == j).all()
+        np.testing.assert_allclose(r.p[:, 0], 1.0, rtol=0, atol=1e-15)
+        assert (r.b == b_want).all()
+        alpha_bound = 13 / 16 if sign > 0 else 3 / 16
+        np.testing.assert_allclose(r.alpha, alpha_bound, rtol=0, atol=1e-15)
+
+
+def test_with_decisions_hand_case(oracle_mod):
+    """with_decisions keeps this oracle's scores and takes the given discrete
+    decisions: q lists the given residual experts by decreasing affinity
+    (ties to the lower index), then the rest; p follows q; k counts the given
+    experts; b counts the given shared blocks (hand example)."""
+    s = np.array([[0.1, 0.5, 0.4], [0.25, 0.5, 0.25]])
+    T, K, B = 2, 3, 4
+    r = oracle.Routing(alpha=np.array([0.6, 0.3]), beta=np.array([0.4, 0.7]),
+                       b=np.array([2, 1], np.int32), k=np.array([1, 2], np.int32),
+                       shr_mask=np.array([0b0011, 0b0001], np.uint64),
+                       q=np.zeros((T, K), np.int32), p=np.zeros((T, K)), s=s,
+                       u=np.zeros((T, B)), margin=np.zeros((T, 4)))
+    f = oracle.with_decisions(r, np.array([0b1010, 0b0111], np.uint64),
+                              np.array([0b101, 0b101], np.uint64), B)
+    assert f.q.tolist() == [[2, 0, 1], [0, 2, 1]]
+    np.testing.assert_array_equal(f.p, [[0.4, 0.1, 0.5], [0.25, 0.25, 0.5]])
+    assert f.k.tolist() == [2, 2] and f.b.tolist() == [2, 3]
+    assert f.shr_mask.tolist() == [0b1010, 0b0111]
+    np.testing.assert_array_equal(f.alpha, r.alpha)
+
+
+def test_with_decisions_output_matches_brute_force(oracle_mod):
+    """The layer output for given decisions (other than the oracle's own)
+    equals the masked sum of dense block outputs with those sets (Eq. 30),
+    and the oracle's own decisions reproduce its own output."""
+    rng = np.random.default_rng(21)
+    K, B = 4, 4
+    x, w_router, w_up, w_down = rand_layer(rng, 6, 16, K, B, router_scale=3.0, T=30)
+    y, r = oracle.layer(x, w_router, w_up, w_down, B)
+    same = oracle.with_decisions(r, r.shr_mask, r.expert_mask(), B)
+    np.testing.assert_array_equal(oracle.forward(x, w_up, w_down, same, B), y)
+    shr = rng.integers(0, 2**B, 30).astype(np.uint64)
+    em = rng.integers(1, 2**K, 30).astype(np.uint64)
+    f = oracle.with_decisions(r, shr, em, B)
+    yf = oracle.forward(x, w_up, w_down, f, B)
+    blocks = block_outputs_dense(x, w_up, w_down, B)
+    for t in range(30):
+        want = np.zeros(x.shape[1])
+        for blk in range(B):
+            if (int(shr[t]) >> blk) & 1:
+                want += r.alpha[t] * blocks[t, 0, blk]
+            else:
+                for j in range(K):
+                    if (int(em[t]) >> j) & 1:
+                        want += r.s[t, j] * blocks[t, 1 + j, blk]
+        np.testing.assert_allclose(yf[t], want, rtol=1e-12, atol=1e-13)
 
 
 # --------------------------------------------------------------------------
@@ -378,6 +503,39 @@ def test_prototype_rounding(oracle_mod):
     w2 = np.array([[1.0], [2**-9], [0.0], [0.0]])  # mean of first block = (1 + 2^-9)/2
     mu2 = oracle.prototypes(w2, 2, oracle.ROUND_BF16)[:, 0]
     assert mu2[0] == 0.5  # (1+2^-9)/2 = 0.5 + 2^-10, below the halfway point 0.5 + 2^-9
+
+
+def test_margins_hand_case(oracle_mod):
+    """All four margins on two hand-built tokens. M = 1, so the priority of
+    block b is key b of the shared expert; x is a unit vector, so the logits
+    are one row of W*: residual logits ln(0.5, 0.3, 0.2) and ln(0.65, 0.25,
+    0.1) give those affinities exactly (to rounding). alpha fixed at 0.5
+    (B = 4: b = 2, margin (i) not applicable), beta fixed at 0.6.
+      token 0: u = (0.9, 0.5, 0.45, 0.1): (ii) = 0.5 - 0.45 = 0.05;
+               P = 0.5, 0.8: k = 2, (iii) = min(0.8 - 0.6, 0.6 - 0.5) = 0.1;
+               (iv) = p_2 - p_3 = 0.1
+      token 1: u = (0.2, 0.8, 0.1, 0.3): (ii) = 0.3 - 0.2 = 0.1;
+               P_1 = 0.65: k = 1, (iii) = min(0.65 - 0.6, 0.6 - 0) = 0.05;
+               (iv) = 0.65 - 0.25 = 0.4"""
+    d, H, K, B = 4, 4, 3, 4
+    x = np.eye(d)[:2]
+    w_router = np.zeros((d, K + 1))
+    w_router[0, 1:] = np.log([0.5, 0.3, 0.2])
+    w_router[1, 1:] = np.log([0.65, 0.25, 0.1])
+    w_up = np.zeros((K + 1, H, d))
+    w_up[0, :, 0] = [0.9, 0.5, 0.45, 0.1]
+    w_up[0, :, 1] = [0.2, 0.8, 0.1, 0.3]
+    w_down = np.zeros((K + 1, d, H))
+    _, r = oracle.layer(x, w_router, w_up, w_down, B, Thresholds(alpha_fixed=0.5, beta_fixed=0.6))
+    assert r.b.tolist() == [2, 2] and r.k.tolist() == [2, 1]
+    assert np.isinf(r.margin[:, 0]).all()
+    np.testing.assert_allclose(r.margin[:, 1], [0.05, 0.1], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(r.margin[:, 2], [0.1, 0.05], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(r.margin[:, 3], [0.1, 0.4], rtol=0, atol=1e-15)
+    # a fixed top-k has no cutoff margin; prefix selection no priority margin
+    _, r2 = oracle.layer(x, w_router, w_up, w_down, B,
+                         Thresholds(alpha_fixed=0.5, topk_fixed=2, prefix_blocks=1))
+    assert np.isinf(r2.margin[:, 1]).all() and np.isinf(r2.margin[:, 2]).all()
 
 
 def test_margins_flag_near_ties(oracle_mod):
