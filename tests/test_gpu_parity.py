@@ -39,7 +39,7 @@ def test_tiny_f32_full():
 def test_vit_s_full_size():
     wl = workloads.make_workload(workloads.spec("vit_s"))
     g = run_gpu(wl)
-    rep = compare(wl, g, sample=1500)
+    rep = compare(wl, g)
     print(rep)
     assert_parity(wl, g, rep)
 
@@ -51,7 +51,7 @@ def test_bert_base_padding():
     assert (g.b[m == 0] == 0).all() and (g.k[m == 0] == 0).all()
     assert (g.y[m == 0] == 0).all()
     assert np.isfinite(g.y).all()
-    rep = compare(wl, g, sample=1000)
+    rep = compare(wl, g)
     print(rep)
     assert_parity(wl, g, rep)
 
@@ -60,7 +60,7 @@ def test_bert_base_padding():
 def test_vit_b_thresholds(theta):
     wl = workloads.make_workload(workloads.spec("vit_b", beta_fixed=theta))
     g = run_gpu(wl)
-    rep = compare(wl, g, sample=400)
+    rep = compare(wl, g, label="theta %s" % theta)
     print(theta, rep)
     assert_parity(wl, g, rep)
 
@@ -68,7 +68,7 @@ def test_vit_b_thresholds(theta):
 def test_stress_full_size():
     wl = workloads.make_workload(workloads.spec("stress"))
     g = run_gpu(wl)
-    rep = compare(wl, g, sample=200)
+    rep = compare(wl, g)
     print(rep, "b range", g.b.min(), g.b.max(), "k range", g.k.min(), g.k.max())
     assert g.b.min() == 1 and g.b.max() == 15  # the mixture spans every shared count
     assert_parity(wl, g, rep)
@@ -312,7 +312,7 @@ def test_gemm_variants_many_group_runs(kernels, monkeypatch):
     wl = workloads.make_workload(small(tokens=6000, d_model=128, d_ff=512, n_experts=8,
                                        n_blocks=4))
     g = run_gpu(wl)
-    assert_parity(wl, g, compare(wl, g, sample=1500))
+    assert_parity(wl, g, compare(wl, g, label=kernels))
 
 
 def test_vit_s_streaming_kernels(monkeypatch):
@@ -320,7 +320,7 @@ def test_vit_s_streaming_kernels(monkeypatch):
     monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
     wl = workloads.make_workload(workloads.spec("vit_s", tokens=4000))
     g = run_gpu(wl)
-    assert_parity(wl, g, compare(wl, g, sample=800))
+    assert_parity(wl, g, compare(wl, g, label="streaming"))
 
 
 def test_repeated_forwards_match_streaming_kernels(monkeypatch):
@@ -353,7 +353,7 @@ def test_repeated_forwards_match_streaming_kernels(monkeypatch):
 def test_repeated_forwards_sliced_down_projection(monkeypatch):
     """A ViT-B-shaped layer (d = 768: the weight-stationary down projection
     runs in three 256-column slices) agrees with the streaming kernels over
-    repeated forwards, and with the oracle on sampled tokens."""
+    repeated forwards, and with the oracle on every token."""
     s = workloads.spec("vit_b", tokens=3000)
     wl = workloads.make_workload(s)
     dev = torch.device("cuda")
@@ -375,5 +375,5 @@ def test_repeated_forwards_sliced_down_projection(monkeypatch):
         rel = (y - ref).abs().amax(1) / ref.abs().amax(1).clamp_min(1e-6)
         assert float(rel.max()) < 1e-2, int((rel >= 1e-2).sum())
     g = run_gpu(wl, layer=L)
-    assert_parity(wl, g, compare(wl, g, sample=300))
+    assert_parity(wl, g, compare(wl, g, label="sliced down projection"))
 
