@@ -132,43 +132,6 @@ def measured_traffic(workload, kernel):
     return rec.get(kernel)
 
 
-def l2_reduction_ceiling(T, d, n_rows, dev, reps=10):
-    """TB/s of fp32 row reductions into a [T][d] accumulator in the down
-    projection epilogue's pattern (n_rows random rows of d values, 4 rows x
-    128 bytes per warp instruction), measured live with the probe library
-    (lib/libunif_probe.so); None where it is not built."""
-    import ctypes
-    import torch
-    path = os.path.join(ROOT, "paper_2608_10392_gb300", "lib", "libunif_probe.so")
-    if not os.path.exists(path) or d % 32 != 0:
-        return None
-    lib = ctypes.CDLL(path)
-    f = lib.unif_probe_l2_reductions
-    f.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_int,
-                  ctypes.c_void_p]
-    g = torch.Generator().manual_seed(20260810)
-    tok = torch.randint(0, T, (n_rows,), generator=g, dtype=torch.int32).to(dev)
-    y = torch.zeros(T, d, dtype=torch.float32, device=dev)
-    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
-    stream = torch.cuda.current_stream(dev)
-
-    def launch():
-        rc = f(y.data_ptr(), tok.data_ptr(), n_rows, d, n_sm, ctypes.c_void_p(stream.cuda_stream))
-        if rc != 0:
-            raise RuntimeError("reduction probe launch failed (%d)" % rc)
-    for _ in range(3):
-        launch()
-    a = torch.cuda.Event(enable_timing=True)
-    b = torch.cuda.Event(enable_timing=True)
-    a.record(stream)
-    for _ in range(reps):
-        launch()
-    b.record(stream)
-    b.synchronize()
-    ms = a.elapsed_time(b) / reps
-    return n_rows * d * 4 / (ms / 1e3) / 1e12
-
-
 # ----------------------------------------------------------------- clocks
 
 class ClockSampler:
@@ -178,10 +141,11 @@ class ClockSampler:
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, interval_ms=50):
+        import tempfile
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", "clocks_bench.csv")
+        fd, self.path = tempfile.mkstemp(prefix="unif_moe_clocks_", suffix=".csv")
+        os.close(fd)
         try:
-            os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "--query-gpu=" + self.FIELDS,
                                           "--format=csv,noheader,nounits", "-lms", str(interval_ms)],
@@ -199,7 +163,10 @@ class ClockSampler:
             self.proc.kill()
         self.f.close()
         sm, mx, reasons = [], [], set()
-        for line in open(self.path):
+        with open(self.path) as f:
+            lines = f.read().splitlines()
+        os.unlink(self.path)
+        for line in lines:
             parts = [p.strip() for p in line.split(",")]
             if len(parts) < 9 or not parts[0].isdigit() or int(parts[0]) != gpu_index:
                 continue
@@ -258,6 +225,29 @@ class OracleRunner:
             _, t, k = self.time(tokens)
             dt, n, repeat = dt + t, n + k, repeat + 1
         return n / dt, dt, n, tokens, repeat
+
+
+def decision_check(wl, gpu, tokens):
+    """The oracle's decisions on the first `tokens` token slots against the
+    GPU's (b, k, shared block set, residual expert set): near-ties (oracle
+    margin <= 1e-3), tokens whose decisions differ, and those among them
+    with a margin above 1e-3."""
+    import numpy as np
+    import oracle
+    s = wl.spec
+    rm = oracle.ROUND_BF16 if s.dtype == "bf16" else oracle.ROUND_F32
+    th = oracle.Thresholds(s.tau, s.alpha_fixed, s.beta_fixed, s.topk_fixed, s.prefix_blocks)
+    m = None if wl.mask is None else wl.mask[:tokens]
+    mu = oracle.prototypes(wl.w_up, s.n_blocks, rm)
+    r = oracle.route(wl.x[:tokens], wl.w_router, mu, s.n_experts, s.n_blocks, th, m,
+                     wl.router_bias)
+    valid = np.ones(tokens, bool) if m is None else m.numpy() != 0
+    same = ((gpu["b"][:tokens] == r.b) & (gpu["k"][:tokens] == r.k) &
+            (gpu["shr"][:tokens] == r.shr_mask) & (gpu["em"][:tokens] == r.expert_mask()))
+    near = r.margin.min(axis=1) <= 1e-3
+    return {"tokens": int(valid.sum()), "near_ties_margin_le_1e-3": int((near & valid).sum()),
+            "decisions_differ": int((~same).sum()),
+            "differ_with_margin_gt_1e-3": int((~same & ~near).sum())}
 
 
 def oracle_cores():
@@ -350,6 +340,10 @@ def main():
     if layer.sync_status() != 0:
         raise RuntimeError("device status word set during warm-up")
     b_h, k_h = bcnt.cpu().long(), kcnt.cpu().long()
+    rt = layer.routing()
+    gpu_dec = {"b": bcnt.cpu().numpy(), "k": kcnt.cpu().numpy(),
+               "shr": rt["shared_mask"].cpu().numpy().view("uint64"),
+               "em": rt["expert_mask"].cpu().numpy().view("uint64")}
     B, M, d = s.n_blocks, s.block_width, s.d_model
     cb = b_h + k_h * (B - b_h)
     if mask is not None:
@@ -435,32 +429,52 @@ def main():
     ms = total_ms / K
     value = job_throughput(total_valid, ms)
     tflops = act_flops / (ms / 1e3) / 1e12
-    peak_tf = peaks["bf16_tflops_sustained"]
+    # the per-kernel pass times each kernel alone (events between kernels):
+    # the burst bf16 peak applies to the GEMMs; the whole step is set
+    # against the sustained one
+    peak_tf = peaks["bf16_tflops"]
+    peak_tf_sus = peaks["bf16_tflops_sustained"]
     hbm = peaks["hbm_gbs"]
+    hbm_nominal = 8000.0
     # roofline of the dominant kernel (the larger grouped GEMM), timed in the
     # per-kernel pass
     dom = "up_gemm" if stage_ms["up_gemm"] >= stage_ms["down_gemm"] else "down_gemm"
     ach = gemm_flops / (stage_ms[dom] / 1e3) / 1e12
     traffic = measured_traffic(s.name, dom)
-    # the down projection's fp32 reductions into the accumulator (one row of
-    # d values per (token, pair)) against the live-measured rate of the same
-    # reductions alone
-    red_bytes = 4.0 * d * sum_cb
-    red_peak = l2_reduction_ceiling(T, d, sum_cb, dev) if s.dtype == "bf16" and sum_cb > 0 else None
-    router_bytes = T * d * elt + T * (4 * 3 + 8 * 2 + 12 * s.n_experts)
+    # algorithmic bytes of the memory-bound kernels (per forward): the router
+    # reads x and writes each token's records (alpha, b, k, two masks, K
+    # affinities; b and k also to the caller) and, when it groups the pairs,
+    # one (token, weight) row per pair; the permute writes those rows; the
+    # combine reads the fp32 accumulator and writes the output
+    fused = layer.kernels_per_forward() <= 5 and s.dtype == "bf16"
+    router_bytes = (T * d * elt + T * (4 * 3 + 8 * 2 + 4 * s.n_experts + 8) +
+                    (8 * sum_cb if fused else 0))
     combine_bytes = T * d * (4 + elt)
     permute_bytes = sum_cb * 8
+
+    def hbm_stage(ms_, nbytes):
+        gbs = nbytes / ms_ / 1e6
+        return {"ms": ms_, "bytes": nbytes, "GB/s": gbs, "frac_of_measured_hbm": gbs / hbm,
+                "frac_of_nominal_8tbs": gbs / hbm_nominal}
+
     stages = {
-        "router": {"ms": stage_ms["router"], "GB/s": router_bytes / stage_ms["router"] / 1e6},
-        "permute": ({"ms": stage_ms["permute"], "GB/s": permute_bytes / stage_ms["permute"] / 1e6}
-                    if layer.kernels_per_forward() > 4 else
+        "router": hbm_stage(stage_ms["router"], router_bytes),
+        "permute": (hbm_stage(stage_ms["permute"], permute_bytes) if not fused else
                     {"ms": 0.0, "fused_into": "router", "event_gap_ms": stage_ms["permute"]}),
-        "up_gemm": {"ms": stage_ms["up_gemm"],
-                    "TFLOP/s": gemm_flops / stage_ms["up_gemm"] / 1e9},
+        "up_gemm": {"ms": stage_ms["up_gemm"], "TFLOP/s": gemm_flops / stage_ms["up_gemm"] / 1e9,
+                    "frac_of_burst_bf16": gemm_flops / stage_ms["up_gemm"] / 1e9 / peak_tf},
         "down_gemm": {"ms": stage_ms["down_gemm"],
-                      "TFLOP/s": gemm_flops / stage_ms["down_gemm"] / 1e9},
-        "combine": {"ms": stage_ms["combine"], "GB/s": combine_bytes / stage_ms["combine"] / 1e6},
+                      "TFLOP/s": gemm_flops / stage_ms["down_gemm"] / 1e9,
+                      "frac_of_burst_bf16": gemm_flops / stage_ms["down_gemm"] / 1e9 / peak_tf},
+        "combine": hbm_stage(stage_ms["combine"], combine_bytes),
     }
+    import numpy as np
+    valid = np.ones(T, bool) if mask is None else mask.numpy() != 0
+    cb_np = cb.numpy()
+
+    def hist(v):
+        vals, counts = np.unique(v[valid], return_counts=True)
+        return {str(int(a)): int(c) for a, c in zip(vals, counts)}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -473,19 +487,17 @@ def main():
                        l2="flushed between steps (512 MB write + 256 MB read, outside the "
                           "timed events)"),
         "activated_tflops": tflops,
-        "activated_frac_of_bf16_peak": tflops / peak_tf,
+        "activated_frac_of_bf16_peak": tflops / peak_tf_sus,
+        "activated_frac_kind": "%s bf16 sustained (whole step)" % peak_kind,
         "mean_C_B": sum_cb / T_valid,
+        "decisions": {"hist_b": hist(b_h.numpy()), "hist_k": hist(k_h.numpy()),
+                      "hist_C_B": hist(cb_np)},
         "roofline": {"bound": "tensor", "kernel": dom, "achieved": ach, "peak": peak_tf,
                      "unit": "TFLOP/s", "frac": ach / peak_tf, "traffic": traffic,
-                     "peak_kind": "%s bf16 sustained" % peak_kind},
+                     "peak_kind": "%s bf16 burst (kernel timed alone)" % peak_kind,
+                     "frac_of_sustained": ach / peak_tf_sus},
         "stages": stages,
         "hbm_peak_gbs": hbm,
-        "reduction_bound": None if red_peak is None else {
-            "kernel": "down_gemm", "bytes": red_bytes,
-            "achieved": red_bytes / (stage_ms["down_gemm"] / 1e3) / 1e12, "peak": red_peak,
-            "unit": "TB/s", "frac": red_bytes / (stage_ms["down_gemm"] / 1e3) / 1e12 / red_peak,
-            "peak_kind": "live probe: the same number of random fp32 rows reduced alone in the "
-                         "epilogue's pattern"},
         "e2e": None if not e2e_ms else {
             "value": T_valid / (statistics.fmean(e2e_ms) / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
@@ -500,7 +512,9 @@ def main():
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": oracle_cores(), "kind": "oracle",
                                 "sample": "first %d of the workload's %d token slots, %d passes "
                                           "(%d valid tokens in all, %.1f s)"
-                                          % (tokens, T, repeat, n, dt)}
+                                          % (tokens, T, repeat, n, dt),
+                                # the oracle's decisions on every token against the GPU's
+                                "parity_check": decision_check(wl, gpu_dec, T)}
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()

@@ -74,16 +74,49 @@ typedef struct {
 /* Fills *th with the paper's adaptive settings (all NaN / 0). */
 UNIF_MOE_API void unif_moe_default_thresholds(unif_moe_thresholds* th);
 
+/* Optional parts of a handle, chosen at create time (not in the paper; they
+ * decide which workspaces unif_moe_create_ex allocates up front). */
+enum {
+  UNIF_MOE_FEATURE_NORM_FIRST = 1, /* unif_moe_sublayer_forward with norm_first:
+                                      a [max_tokens][d] buffer for LN(x) */
+  UNIF_MOE_FEATURE_HOST_IO = 2,    /* unif_moe_forward_host: device staging
+                                      buffers for x, y, the mask and the counts */
+  UNIF_MOE_FEATURES_ALL = 3
+};
+/* Grouped GEMM kernels: the library picks the weight-stationary kernels
+ * where a group's weight slice fits in shared memory, else the streaming
+ * ones (AUTO); STREAMING always takes the streaming ones (both compute the
+ * same products; the fp32 sums into the output differ only in order). */
+enum { UNIF_MOE_GEMM_AUTO = 0, UNIF_MOE_GEMM_STREAMING = 1 };
+
+typedef struct {
+  unsigned int features; /* UNIF_MOE_FEATURE_* bits */
+  int gemm_kernels;      /* UNIF_MOE_GEMM_AUTO or UNIF_MOE_GEMM_STREAMING */
+} unif_moe_options;
+
+/* Fills *opts with the defaults of unif_moe_create: every feature, AUTO. */
+UNIF_MOE_API void unif_moe_default_options(unif_moe_options* opts);
+
 /* Creates a layer (Sec. III-A): d_model = d, d_ff = H, n_experts = K residual
  * experts (one shared expert is added), n_blocks = B, max_tokens = largest T
  * a forward will be given. th may be NULL (adaptive defaults).
  * Limits: 2 <= B <= 64, 1 <= K <= 64, H % B == 0, d % 8 == 0; for
  * UNIF_MOE_BF16 also d % 64 == 0 and M = H/B a multiple of 64.
  * Device workspace for max_tokens is allocated here, sized for the largest
- * possible C_B (Eq. 35) under th; nothing is allocated by later calls.
+ * possible C_B (Eq. 35) under th, with every optional feature's buffers
+ * (UNIF_MOE_FEATURES_ALL); no later call allocates device memory.
  * Errors: ERR_ARG (out == NULL, bad values), ERR_SHAPE, ERR_CUDA (allocation). */
 UNIF_MOE_API int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n_blocks,
                     const unif_moe_thresholds* th, unif_moe_dtype dtype, int max_tokens);
+
+/* unif_moe_create with options (NULL = the defaults above). A handle made
+ * without a feature refuses the calls that need it with ERR_STATE, so no
+ * later call allocates device memory either. Errors as unif_moe_create, and
+ * ERR_ARG for unknown feature bits or GEMM kind. */
+UNIF_MOE_API int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts,
+                                    int n_blocks, const unif_moe_thresholds* th,
+                                    unif_moe_dtype dtype, int max_tokens,
+                                    const unif_moe_options* opts);
 
 /* Loads weights from device memory (copied into the handle; the caller may
  * free its buffers once `stream` has passed this call):
@@ -137,9 +170,9 @@ UNIF_MOE_API int unif_moe_forward(unif_moe_t h, const void* x_dev, void* out_dev
  * Padding tokens (mask 0) give 0. The routing decisions and counts are
  * those of F's input. x, out, counts, mask and errors as unif_moe_forward;
  * also ERR_ARG (NULL or not 16-byte aligned gamma or beta, bad eps),
- * ERR_SHAPE (d > 1024 or not a multiple of 8). A
- * norm-first call allocates a [max_tokens][d] buffer for LN(x) on first
- * use. */
+ * ERR_SHAPE (d > 1024 or not a multiple of 8), ERR_STATE (norm_first on a
+ * handle created without UNIF_MOE_FEATURE_NORM_FIRST; LN(x) goes to the
+ * buffer allocated for it at create time). */
 UNIF_MOE_API int unif_moe_sublayer_forward(unif_moe_t h, const void* x_dev, void* out_dev, int T,
                                            const uint8_t* token_mask_dev,
                                            int32_t* shared_counts_dev,
@@ -153,7 +186,9 @@ UNIF_MOE_API int unif_moe_sublayer_forward(unif_moe_t h, const void* x_dev, void
  * residual_counts_host (each may be NULL), and synchronises `stream` before
  * returning. Host buffers should be pinned for asynchronous copies; output
  * buffers (out_host and the counts) in pinned host memory the device can
- * address are written by the kernels directly, with no copy back. */
+ * address are written by the kernels directly, with no copy back. The
+ * staging buffers are allocated at create time (UNIF_MOE_FEATURE_HOST_IO;
+ * ERR_STATE on a handle created without it). */
 UNIF_MOE_API int unif_moe_forward_host(unif_moe_t h, const void* x_host, void* out_host, int T,
                           const uint8_t* token_mask_host, int32_t* shared_counts_host,
                           int32_t* residual_counts_host, void* stream);

@@ -19,7 +19,8 @@ from typing import Optional
 
 import torch
 
-__all__ = ["Layer", "lib", "UnifMoeError", "ERR", "EXPORTS"]
+__all__ = ["Layer", "lib", "UnifMoeError", "ERR", "EXPORTS", "Options", "FEATURE_NORM_FIRST",
+           "FEATURE_HOST_IO", "FEATURES_ALL"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "lib", "libunif_moe.so")
@@ -28,7 +29,8 @@ ERR = {0: "OK", -1: "ERR_ARG", -2: "ERR_SHAPE", -3: "ERR_CAPACITY", -4: "ERR_CUD
        -5: "ERR_TIMEOUT", -6: "ERR_STATE"}
 
 # Every symbol include/unif_moe.h declares.
-EXPORTS = ["unif_moe_default_thresholds", "unif_moe_create", "unif_moe_load_weights",
+EXPORTS = ["unif_moe_default_thresholds", "unif_moe_default_options", "unif_moe_create",
+           "unif_moe_create_ex", "unif_moe_load_weights",
            "unif_moe_load_upcycled", "unif_moe_forward", "unif_moe_sublayer_forward",
            "unif_moe_forward_host", "unif_moe_get_routing",
            "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_kernels_per_forward",
@@ -48,6 +50,14 @@ class Thresholds(C.Structure):
                 ("topk_fixed", C.c_int), ("prefix_blocks", C.c_int)]
 
 
+class Options(C.Structure):
+    _fields_ = [("features", C.c_uint), ("gemm_kernels", C.c_int)]
+
+
+FEATURE_NORM_FIRST, FEATURE_HOST_IO, FEATURES_ALL = 1, 2, 3
+GEMM_KERNELS = {"auto": 0, "streaming": 1}
+
+
 _lib = None
 
 
@@ -62,6 +72,10 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_default_thresholds.argtypes = [C.POINTER(Thresholds)]
         L.unif_moe_default_thresholds.restype = None
         L.unif_moe_create.argtypes = [C.POINTER(P), I, I, I, I, C.POINTER(Thresholds), I, I]
+        L.unif_moe_default_options.argtypes = [C.POINTER(Options)]
+        L.unif_moe_default_options.restype = None
+        L.unif_moe_create_ex.argtypes = [C.POINTER(P), I, I, I, I, C.POINTER(Thresholds), I, I,
+                                         C.POINTER(Options)]
         L.unif_moe_load_weights.argtypes = [P, P, P, P, P, P]
         L.unif_moe_forward.argtypes = [P, P, P, I, P, P, P, P]
         L.unif_moe_load_upcycled.argtypes = [P, P, P, P, P, P]
@@ -80,7 +94,8 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_destroy.restype = None
         L.unif_moe_last_error.restype = C.c_char_p
         for name in EXPORTS:
-            if name not in ("unif_moe_default_thresholds", "unif_moe_destroy",
+            if name not in ("unif_moe_default_thresholds", "unif_moe_default_options",
+                            "unif_moe_destroy",
                             "unif_moe_last_error", "unif_moe_max_rows"):
                 getattr(L, name).restype = C.c_int
         _lib = L
@@ -105,20 +120,25 @@ def _stream(stream) -> Optional[int]:
 class Layer:
     """One UniF-MoE layer (Sec. III): K residual experts plus one shared
     expert, FFN width H split into B blocks. dtype "bf16" (tensor cores) or
-    "f32" (CUDA-core FMA)."""
+    "f32" (CUDA-core FMA). `features` (FEATURE_* bits) picks the optional
+    workspaces allocated at create time; `gemm_kernels` "auto" or
+    "streaming"."""
 
     def __init__(self, d_model: int, d_ff: int, n_experts: int, n_blocks: int,
                  dtype: str = "bf16", max_tokens: int = 65536, tau: float = math.nan,
                  alpha_fixed: float = math.nan, beta_fixed: float = math.nan,
-                 topk_fixed: int = 0, prefix_blocks: int = 0):
+                 topk_fixed: int = 0, prefix_blocks: int = 0, features: int = FEATURES_ALL,
+                 gemm_kernels: str = "auto"):
         self.d, self.H, self.K, self.B = d_model, d_ff, n_experts, n_blocks
         self.dtype = dtype
         self.torch_dtype = torch.bfloat16 if dtype == "bf16" else torch.float32
         self.max_tokens = max_tokens
         th = Thresholds(tau, alpha_fixed, beta_fixed, topk_fixed, prefix_blocks)
+        opts = Options(features, GEMM_KERNELS[gemm_kernels])
         h = C.c_void_p()
-        _check(lib().unif_moe_create(C.byref(h), d_model, d_ff, n_experts, n_blocks, C.byref(th),
-                                     1 if dtype == "bf16" else 0, max_tokens))
+        _check(lib().unif_moe_create_ex(C.byref(h), d_model, d_ff, n_experts, n_blocks,
+                                        C.byref(th), 1 if dtype == "bf16" else 0, max_tokens,
+                                        C.byref(opts)))
         self._h = h
         self.last_T = 0
 

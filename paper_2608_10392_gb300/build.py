@@ -1,9 +1,8 @@
 """Builds libunif_moe.so (the C-ABI library) in-tree for sm_103a with nvcc.
 
 Each translation unit compiles in its own nvcc process (in parallel); the
-objects link into paper_2608_10392_gb300/lib/libunif_moe.so. The
-measurement probe (csrc/probe_l2.cu, used by bench.py) links into its own
-lib/libunif_probe.so. Nothing is installed outside the repository.
+objects link into paper_2608_10392_gb300/lib/libunif_moe.so. Nothing is
+installed outside the repository.
 """
 from __future__ import annotations
 
@@ -18,8 +17,6 @@ CSRC = os.path.join(HERE, "csrc")
 LIBDIR = os.path.join(HERE, "lib")
 LIB = os.path.join(LIBDIR, "libunif_moe.so")
 SOURCES = ["unif_moe.cu", "route_permute.cu", "gemm_simt.cu", "gemm_tc.cu", "gemm_ws.cu"]
-PROBE_LIB = os.path.join(LIBDIR, "libunif_probe.so")
-PROBE_SOURCE = "probe_l2.cu"
 HEADERS = ["internal.cuh", "decide.cuh", "tc_common.cuh", os.path.join("..", "..", "include", "unif_moe.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
@@ -60,20 +57,9 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
             sys.stderr.write(r.stdout + r.stderr)
         return r
 
-    probe = os.path.join(CSRC, PROBE_SOURCE)
-    if force or _stale(PROBE_LIB, [probe]):
-        jobs.append(None)  # built below, alongside the library's objects
-
-    def job(cmd):
-        if cmd is not None:
-            return run(cmd)
-        tmp = PROBE_LIB + ".tmp%d" % os.getpid()
-        run([nvcc()] + ARCH + flags + ["-shared", probe, "-o", tmp])
-        os.replace(tmp, PROBE_LIB)
-
-    with cf.ThreadPoolExecutor(max_workers=len(SOURCES) + 1) as ex:
-        list(ex.map(job, jobs))
-    if force or any(j is not None for j in jobs) or _stale(LIB, objs):
+    with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
+        list(ex.map(run, jobs))
+    if force or jobs or _stale(LIB, objs):
         tmp = LIB + ".tmp%d" % os.getpid()
         run([nvcc()] + ARCH + ["-shared", "-o", tmp] + objs)
         os.replace(tmp, LIB)

@@ -569,12 +569,11 @@ ws_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 // allow: the up projection needs the whole block width in one accumulator
 // (M <= 256); the down projection reuses each h tile across all output
 // column sub-tiles, so the tile's M / 64 reduction stages must fit its A ring.
-// UNIF_MOE_GEMM_KERNELS=streaming keeps the streaming kernels.
+// A handle created with UNIF_MOE_GEMM_STREAMING keeps the streaming kernels.
 int gemm_ws_setup(unif_moe_layer* L) {
   using namespace tc::ws;
   L->up_ws = L->down_ws = false;
-  const char* env = getenv("UNIF_MOE_GEMM_KERNELS");
-  if (env && strcmp(env, "streaming") == 0) return UNIF_MOE_OK;
+  if (L->gemm_streaming) return UNIF_MOE_OK;
   // the tile table (first tile and size of every group, the tiles of one
   // CTA's run) follows the barriers
   const uint64_t per_cta = (uint64_t)((L->max_tiles + L->n_sm - 1) / L->n_sm);

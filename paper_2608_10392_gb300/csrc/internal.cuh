@@ -74,7 +74,8 @@ struct Workspace {
   void* hbuf = nullptr;          // [max_rows][M] (layer dtype)
   float* y32 = nullptr;          // [max_tokens][d]
   // Host-buffer forward staging.
-  void* xn = nullptr;             // [max_tokens][d] LN(x) of a norm-first sublayer (on first use)
+  void* xn = nullptr;             // [max_tokens][d] LN(x) of a norm-first sublayer
+  // Staging buffers of the host-buffer forward.
   void* x_stage = nullptr;
   void* out_stage = nullptr;
   uint8_t* mask_stage = nullptr;
@@ -103,6 +104,8 @@ struct unif_moe_layer {
   bool fused_group = false;
   int region_rows = 0;
   bool tile_list = false;  // a streaming GEMM reads the tile list: build it after the router
+  unsigned features = 0;        // UNIF_MOE_FEATURE_* workspaces allocated at create time
+  bool gemm_streaming = false;  // UNIF_MOE_GEMM_STREAMING: never the weight-stationary kernels
   int device = 0;
   bool loaded = false;
   bool y_dirty = false;  // accumulator / grouping counters may hold state of a forward cut short

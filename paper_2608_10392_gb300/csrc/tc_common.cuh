@@ -205,7 +205,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 // ---- GeLU on pairs with packed fp32x2 arithmetic ----
 // GeLU(x) = x Phi(x), Phi(x) = (1 + tanh(g(x))) / 2 with g(x) = atanh(2 Phi(x) - 1)
 // approximated by x P(x^2), P of degree 4 (coefficients and their fit in
-// gelu_coeffs.py; |Phi error| < 2e-6 before the hardware tanh, whose own
+// tests/gelu_fit.py; |Phi error| < 2e-6 before the hardware tanh, whose own
 // error, about 2^-11, dominates). g increases monotonically, so large |x|
 // saturates cleanly to x or 0. Evaluated as h = x/2 + (x/2) tanh(g).
 __device__ __forceinline__ uint64_t pk2(float lo, float hi) {

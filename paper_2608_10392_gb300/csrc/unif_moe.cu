@@ -94,11 +94,32 @@ void unif_moe_default_thresholds(unif_moe_thresholds* th) {
 
 const char* unif_moe_last_error(void) { return unif::g_err; }
 
+void unif_moe_default_options(unif_moe_options* opts) {
+  if (!opts) return;
+  opts->features = UNIF_MOE_FEATURES_ALL;
+  opts->gemm_kernels = UNIF_MOE_GEMM_AUTO;
+}
+
 int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n_blocks,
                     const unif_moe_thresholds* th, unif_moe_dtype dtype, int max_tokens) {
+  return unif_moe_create_ex(out, d_model, d_ff, n_experts, n_blocks, th, dtype, max_tokens,
+                            nullptr);
+}
+
+int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n_blocks,
+                       const unif_moe_thresholds* th, unif_moe_dtype dtype, int max_tokens,
+                       const unif_moe_options* opts) {
   unif::g_err[0] = 0;
   if (!out) { set_error("out is NULL"); return UNIF_MOE_ERR_ARG; }
   *out = nullptr;
+  unif_moe_options o;
+  unif_moe_default_options(&o);
+  if (opts) o = *opts;
+  if ((o.features & ~(unsigned)UNIF_MOE_FEATURES_ALL) != 0u ||
+      (o.gemm_kernels != UNIF_MOE_GEMM_AUTO && o.gemm_kernels != UNIF_MOE_GEMM_STREAMING)) {
+    set_error("bad options: features 0x%x, gemm_kernels %d", o.features, o.gemm_kernels);
+    return UNIF_MOE_ERR_ARG;
+  }
   if (dtype != UNIF_MOE_F32 && dtype != UNIF_MOE_BF16) { set_error("bad dtype"); return UNIF_MOE_ERR_ARG; }
   if (d_model <= 0 || d_ff <= 0 || n_experts < 1 || n_experts > 64 || n_blocks < 2 ||
       n_blocks > 64 || max_tokens < 1) {
@@ -137,6 +158,8 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   L->d = d_model; L->H = d_ff; L->K = n_experts; L->B = n_blocks; L->M = M;
   L->G = (n_experts + 1) * n_blocks;
   L->dtype = dtype; L->max_tokens = max_tokens; L->th = t;
+  L->features = o.features;
+  L->gemm_streaming = o.gemm_kernels == UNIF_MOE_GEMM_STREAMING;
   L->tau = isnan(t.tau) ? (float)((double)(n_blocks - 1) / ((double)n_blocks * n_blocks)) : t.tau;
   const int kmax = t.topk_fixed > 0 ? t.topk_fixed : n_experts;
   L->cb_max = kmax * n_blocks;  // C_B = b + k (B - b) <= k B for every b >= 0 (Eq. 35)
@@ -199,6 +222,16 @@ int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n
   w.hbuf = hb;
   ALLOC(w.y32, T * d_model);
   ALLOC(w.status, 1);
+  // optional features: every buffer a later call needs, so that no later
+  // call allocates
+  if (o.features & UNIF_MOE_FEATURE_NORM_FIRST) {
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.xn), es * T * d_model);
+  }
+  if (o.features & UNIF_MOE_FEATURE_HOST_IO) {
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.x_stage), es * T * d_model);
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.out_stage), es * T * d_model);
+    ALLOC(w.mask_stage, T); ALLOC(w.b_stage, T); ALLOC(w.k_stage, T);
+  }
 #undef ALLOC
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
                             cudaMemset(w.y32, 0, sizeof(float) * T * d_model) != cudaSuccess ||
@@ -368,11 +401,10 @@ int unif_moe_sublayer_forward(unif_moe_t L, const void* x, void* out, int T,
   const SublayerEpilogue sub{x, ln_gamma, ln_beta, eps, !norm_first};
   if (!norm_first)  // out = LN(x + F(x))
     return forward_core(L, x, out, T, token_mask, shared_counts, residual_counts, s, &sub);
-  // out = x + F(LN(x)); LN(x) in the layer dtype, in a buffer made on first use
+  // out = x + F(LN(x)); LN(x) in the layer dtype, in the buffer made at create
   if (!L->ws.xn) {
-    const int arc = dalloc(reinterpret_cast<char**>(&L->ws.xn),
-                           elt_size(L) * (size_t)L->max_tokens * L->d);
-    if (arc != UNIF_MOE_OK) return arc;
+    set_error("norm-first sublayer on a handle created without UNIF_MOE_FEATURE_NORM_FIRST");
+    return UNIF_MOE_ERR_STATE;
   }
   CK(unif::launch_layernorm(L, x, L->ws.xn, token_mask, ln_gamma, ln_beta, eps, T, s));
   return forward_core(L, L->ws.xn, out, T, token_mask, shared_counts, residual_counts, s, &sub);
@@ -402,21 +434,16 @@ int unif_moe_forward_host(unif_moe_t L, const void* x_host, void* out_host, int 
     return T < 0 ? UNIF_MOE_ERR_ARG : UNIF_MOE_ERR_CAPACITY;
   }
   if (!L->loaded) { set_error("forward before load_weights"); return UNIF_MOE_ERR_STATE; }
+  if (!(L->features & UNIF_MOE_FEATURE_HOST_IO)) {
+    set_error("host-buffer forward on a handle created without UNIF_MOE_FEATURE_HOST_IO");
+    return UNIF_MOE_ERR_STATE;
+  }
   if (T == 0) return UNIF_MOE_OK;
   if (!x_host || !out_host) { set_error("x or out is NULL"); return UNIF_MOE_ERR_ARG; }
   DeviceGuard dg(L->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   unif::Workspace& w = L->ws;
   const size_t es = elt_size(L);
-  const size_t n = (size_t)L->max_tokens;
-  if (!w.x_stage) {  // staging buffers are created on first use
-    int rc = dalloc(reinterpret_cast<char**>(&w.x_stage), es * n * L->d);
-    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.out_stage), es * n * L->d);
-    if (rc == UNIF_MOE_OK) rc = dalloc(&w.mask_stage, n);
-    if (rc == UNIF_MOE_OK) rc = dalloc(&w.b_stage, n);
-    if (rc == UNIF_MOE_OK) rc = dalloc(&w.k_stage, n);
-    if (rc != UNIF_MOE_OK) return rc;
-  }
   const size_t xb = es * (size_t)T * L->d;
   CK(cudaMemcpyAsync(w.x_stage, x_host, xb, cudaMemcpyHostToDevice, s));
   if (mask_host) CK(cudaMemcpyAsync(w.mask_stage, mask_host, (size_t)T, cudaMemcpyHostToDevice, s));

@@ -12,7 +12,8 @@ On the GPU, tanh is the hardware approximation tanh.approx.f32, whose error
 (about 2^-11) dominates the polynomial's (below 2e-6 on Phi): the GeLU
 error stays a small fraction of the bf16 rounding that h receives next.
 
-Run:  python paper_2608_10392_gb300/csrc/gelu_coeffs.py
+Run:  python tests/gelu_fit.py   (prints the constants the epilogue in
+csrc/tc_common.cuh holds; tests/test_gelu_epilogue.py checks them)
 """
 import struct
 

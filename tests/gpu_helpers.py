@@ -55,18 +55,19 @@ class GpuRun:
     layer: object
 
 
-def make_layer(s, max_tokens=None):
+def make_layer(s, max_tokens=None, **kw):
     from paper_2608_10392_gb300 import Layer
     return Layer(s.d_model, s.d_ff, s.n_experts, s.n_blocks, dtype=s.dtype,
                  max_tokens=max_tokens or s.tokens, tau=s.tau, alpha_fixed=s.alpha_fixed,
-                 beta_fixed=s.beta_fixed, topk_fixed=s.topk_fixed, prefix_blocks=s.prefix_blocks)
+                 beta_fixed=s.beta_fixed, topk_fixed=s.topk_fixed, prefix_blocks=s.prefix_blocks,
+                 **kw)
 
 
-def run_gpu(wl, layer=None, x=None, mask="default") -> GpuRun:
+def run_gpu(wl, layer=None, x=None, mask="default", **layer_kw) -> GpuRun:
     s = wl.spec
     dev = torch.device("cuda")
     if layer is None:
-        layer = make_layer(s, max_tokens=max(s.tokens, 1))
+        layer = make_layer(s, max_tokens=max(s.tokens, 1), **layer_kw)
         bias = None if wl.router_bias is None else wl.router_bias.to(dev)
         layer.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev), bias)
     x = wl.x if x is None else x

@@ -48,23 +48,6 @@ def test_only_declared_symbols_are_exported(lib):
     assert ours == declared_symbols()
 
 
-def test_measurement_probe_library(lib):
-    """The reduction probe bench.py times is built into its own library,
-    exports only its launcher, and rejects bad arguments before any CUDA
-    call (so this runs without a GPU)."""
-    import subprocess
-    from paper_2608_10392_gb300 import build
-    assert os.path.exists(build.PROBE_LIB)
-    out = subprocess.run(["nm", "-D", "--defined-only", build.PROBE_LIB], capture_output=True,
-                         text=True).stdout
-    assert [l.split()[-1] for l in out.splitlines() if " T unif_" in l] == ["unif_probe_l2_reductions"]
-    f = C.CDLL(build.PROBE_LIB).unif_probe_l2_reductions
-    f.argtypes = [C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_void_p]
-    assert f(None, None, 10, 384, 152, None) == -1          # null buffers
-    assert f(C.c_void_p(16), C.c_void_p(16), 10, 100, 152, None) == -1   # d not a multiple of 32
-    assert f(C.c_void_p(16), C.c_void_p(16), 0, 384, 152, None) == -1    # no rows
-
-
 def test_argument_errors_without_gpu(lib):
     import paper_2608_10392_gb300 as pkg
     th = pkg.Thresholds()
@@ -80,6 +63,12 @@ def test_argument_errors_without_gpu(lib):
     assert b"d_model" in lib.unif_moe_last_error()
     bad = pkg.Thresholds(math.nan, math.nan, math.nan, 5, 0)
     assert lib.unif_moe_create(C.byref(h), 64, 256, 4, 4, C.byref(bad), 1, 16) == -1
+    opts = pkg.Options()
+    lib.unif_moe_default_options(C.byref(opts))
+    assert opts.features == pkg.FEATURES_ALL and opts.gemm_kernels == 0
+    for o in (pkg.Options(8, 0), pkg.Options(3, 2), pkg.Options(3, -1)):  # unknown bit / kind
+        assert lib.unif_moe_create_ex(C.byref(h), 64, 256, 4, 4, None, 1, 16, C.byref(o)) == -1
+    assert b"options" in lib.unif_moe_last_error()
     assert lib.unif_moe_forward(None, None, None, 4, None, None, None, None) == -1
     assert lib.unif_moe_load_weights(None, None, None, None, None, None) == -1
     assert lib.unif_moe_load_upcycled(None, None, None, None, None, None) == -1
@@ -106,3 +95,11 @@ def test_product_code_never_touches_the_oracle():
                 text = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in text and "liboracle" not in text, f
                 assert "from oracle" not in text, f
+
+
+def test_library_reads_no_environment():
+    """Behaviour is set through the ABI only: no getenv in the library."""
+    csrc = os.path.join(ROOT, "paper_2608_10392_gb300", "csrc")
+    for f in os.listdir(csrc):
+        if f.endswith((".cu", ".cuh", ".h")):
+            assert "getenv" not in open(os.path.join(csrc, f)).read(), f

@@ -125,9 +125,9 @@ def test_kernels_per_forward():
     assert make_layer(small("f32", tokens=64)).kernels_per_forward() == 6
 
 
-def test_kernels_per_forward_streaming(monkeypatch):
-    monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
-    assert make_layer(small(tokens=500)).kernels_per_forward() == 5   # + tile list
+def test_kernels_per_forward_streaming():
+    L = make_layer(small(tokens=500), gemm_kernels="streaming")
+    assert L.kernels_per_forward() == 5   # + tile list
 
 
 @pytest.mark.parametrize("shape", [
@@ -251,6 +251,74 @@ def test_errors_are_reported():
         make_layer(wl.spec.with_(d_model=96))  # bf16 needs d % 64 == 0
 
 
+def test_forward_calls_allocate_nothing():
+    """Every buffer a forward-family call needs is allocated at create time:
+    the device's free memory does not move across a fresh handle's first
+    forward, norm-first and norm-after sublayer forwards and host-buffer
+    forwards (kernel modules loaded beforehand by another handle; every
+    torch output allocated beforehand)."""
+    s = workloads.spec("vit_s")
+    wl = workloads.make_workload(s)
+    dev = torch.device("cuda")
+    d = s.d_model
+    x = wl.x.to(dev)
+    out = torch.empty_like(x)
+    b = torch.empty(s.tokens, dtype=torch.int32, device=dev)
+    k = torch.empty_like(b)
+    gamma = torch.ones(d, dtype=torch.bfloat16, device=dev)
+    beta = torch.zeros(d, dtype=torch.bfloat16, device=dev)
+    xh = wl.x.pin_memory()
+    oh = torch.empty_like(xh).pin_memory()
+    xp, op = wl.x.clone(), torch.empty_like(wl.x)  # pageable: staging buffers and copies
+    bh = torch.empty(s.tokens, dtype=torch.int32)
+
+    def every_call(L):
+        L.forward(x, out=out, shared_counts=b, residual_counts=k)
+        L.sublayer_forward(x, gamma, beta, 1e-5, True, out=out)
+        L.sublayer_forward(x, gamma, beta, 1e-5, False, out=out)
+        L.forward_host(xh, oh, shared_counts_host=bh)
+        L.forward_host(xp, op, shared_counts_host=bh)
+        torch.cuda.synchronize()
+        assert L.sync_status() == 0
+
+    def fresh():
+        L = make_layer(s)
+        L.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
+        torch.cuda.synchronize()
+        return L
+
+    every_call(fresh())  # loads every kernel the calls launch
+    L = fresh()
+    free0 = torch.cuda.mem_get_info()[0]
+    every_call(L)
+    assert torch.cuda.mem_get_info()[0] == free0
+
+
+def test_features_left_out_are_refused():
+    """A handle created without the optional workspaces refuses the calls
+    that need them (ERR_STATE) and runs the rest."""
+    from paper_2608_10392_gb300 import UnifMoeError
+    wl = workloads.make_workload(small(tokens=256))
+    dev = torch.device("cuda")
+    L = make_layer(wl.spec, features=0)
+    L.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
+    x = wl.x.to(dev)
+    d = wl.spec.d_model
+    gamma = torch.ones(d, dtype=torch.bfloat16, device=dev)
+    beta = torch.zeros(d, dtype=torch.bfloat16, device=dev)
+    with pytest.raises(UnifMoeError) as e:
+        L.sublayer_forward(x, gamma, beta, 1e-5, True)
+    assert e.value.code == -6
+    with pytest.raises(UnifMoeError) as e:
+        L.forward_host(wl.x.clone(), torch.empty_like(wl.x))
+    assert e.value.code == -6
+    y = L.forward(x)
+    z = L.sublayer_forward(x, gamma, beta, 1e-5, False)
+    torch.cuda.synchronize()
+    assert L.sync_status() == 0
+    assert torch.isfinite(y.float()).all() and torch.isfinite(z.float()).all()
+
+
 def test_output_guard_bands():
     wl = workloads.make_workload(small(tokens=257))
     layer = make_layer(wl.spec)
@@ -304,26 +372,23 @@ def test_forward_host_pageable_buffers():
 # ------------------------------------------- GEMM kernel variants
 
 @pytest.mark.parametrize("kernels", ["weight_stationary", "streaming"])
-def test_gemm_variants_many_group_runs(kernels, monkeypatch):
+def test_gemm_variants_many_group_runs(kernels):
     """Enough tiles that every CTA walks several group runs (weight slabs
     reloaded mid-run), on both GEMM kernel families."""
-    if kernels == "streaming":
-        monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
     wl = workloads.make_workload(small(tokens=6000, d_model=128, d_ff=512, n_experts=8,
                                        n_blocks=4))
-    g = run_gpu(wl)
+    g = run_gpu(wl, gemm_kernels="auto" if kernels == "weight_stationary" else "streaming")
     assert_parity(wl, g, compare(wl, g, label=kernels))
 
 
-def test_vit_s_streaming_kernels(monkeypatch):
+def test_vit_s_streaming_kernels():
     """The ViT-S layer through the streaming GEMMs agrees with the oracle too."""
-    monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
     wl = workloads.make_workload(workloads.spec("vit_s", tokens=4000))
-    g = run_gpu(wl)
+    g = run_gpu(wl, gemm_kernels="streaming")
     assert_parity(wl, g, compare(wl, g, label="streaming"))
 
 
-def test_repeated_forwards_match_streaming_kernels(monkeypatch):
+def test_repeated_forwards_match_streaming_kernels():
     """Ten forwards of the ViT-S layer through the weight-stationary kernels
     agree with the streaming kernels token by token (the two differ only in
     the order of the fp32 additions into the accumulator): catches
@@ -332,16 +397,14 @@ def test_repeated_forwards_match_streaming_kernels(monkeypatch):
     wl = workloads.make_workload(s)
     dev = torch.device("cuda")
 
-    def layer():
-        L = make_layer(s)
+    def layer(kernels):
+        L = make_layer(s, gemm_kernels=kernels)
         L.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
         return L
 
     x = wl.x.to(dev)
-    monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
-    ref = layer().forward(x).float()
-    monkeypatch.delenv("UNIF_MOE_GEMM_KERNELS")
-    L = layer()
+    ref = layer("streaming").forward(x).float()
+    L = layer("auto")
     for _ in range(10):
         y = L.forward(x).float()
         torch.cuda.synchronize()
@@ -350,7 +413,7 @@ def test_repeated_forwards_match_streaming_kernels(monkeypatch):
         assert float(rel.max()) < 1e-2, int((rel >= 1e-2).sum())
 
 
-def test_repeated_forwards_sliced_down_projection(monkeypatch):
+def test_repeated_forwards_sliced_down_projection():
     """A ViT-B-shaped layer (d = 768: the weight-stationary down projection
     runs in three 256-column slices) agrees with the streaming kernels over
     repeated forwards, and with the oracle on every token."""
@@ -358,16 +421,14 @@ def test_repeated_forwards_sliced_down_projection(monkeypatch):
     wl = workloads.make_workload(s)
     dev = torch.device("cuda")
 
-    def layer():
-        L = make_layer(s)
+    def layer(kernels):
+        L = make_layer(s, gemm_kernels=kernels)
         L.load_weights(wl.w_router.to(dev), wl.w_up.to(dev), wl.w_down.to(dev))
         return L
 
     x = wl.x.to(dev)
-    monkeypatch.setenv("UNIF_MOE_GEMM_KERNELS", "streaming")
-    ref = layer().forward(x).float()
-    monkeypatch.delenv("UNIF_MOE_GEMM_KERNELS")
-    L = layer()
+    ref = layer("streaming").forward(x).float()
+    L = layer("auto")
     for _ in range(5):
         y = L.forward(x).float()
         torch.cuda.synchronize()

@@ -101,3 +101,31 @@ def test_noalloc_rejects_sizes_beyond_the_scratch():
                                       T * K * B + G * 127, None)
     assert rc == -3
     assert b"scratch" in lib().unif_moe_last_error()
+
+
+def test_noalloc_scratch_limit_is_exact():
+    """(K+1) B ceil(T/256) equal to the scratch's 262144 entries is accepted
+    (and groups every pair); one 256-token chunk more is refused with
+    ERR_CAPACITY before anything is enqueued."""
+    from paper_2608_10392_gb300 import lib
+    K, B = 63, 64
+    G = (K + 1) * B                      # 4096 groups
+    T = 262144 // G * 256                # 64 chunks of 256 tokens: exactly at the limit
+    dev = torch.device("cuda")
+    g = torch.Generator().manual_seed(3)
+    shr = torch.randint(0, 2**62, (T,), generator=g, dtype=torch.int64) & 0x0101  # blocks 0, 8
+    em = torch.randint(0, 2**62, (T,), generator=g, dtype=torch.int64) & 0x11     # experts 0, 4
+    alpha = torch.rand(T, generator=g)
+    s = torch.rand(T, K, generator=g)
+    n_shr = np.array([bin(int(v)).count("1") for v in shr])
+    n_em = np.array([bin(int(v)).count("1") for v in em])
+    pairs = int((n_shr + n_em * (B - n_shr)).sum())  # sum of C_B (Eq. 35)
+    counts, offsets, n_tiles, tok, w, tg, tr = noalloc_groups(
+        lib(), T, K, B, shr.to(dev), em.to(dev), alpha.to(dev), s.to(dev))
+    assert int(counts.sum()) == pairs
+    assert (tok >= 0).sum() == pairs
+    T1 = T + 1                           # 65 chunks
+    p = torch.zeros(8, dtype=torch.int64, device=dev).data_ptr()
+    rc = lib().unif_moe_group_noalloc(T1, K, B, p, p, p, p, p, p, p, p, p, p, p,
+                                      T1 * K * B + G * 127, None)
+    assert rc == -3 and b"scratch" in lib().unif_moe_last_error()
