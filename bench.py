@@ -351,6 +351,14 @@ def main():
     sum_cb = int(cb.sum())
     gemm_flops = 2.0 * d * M * sum_cb  # one of the two grouped GEMMs (Eq. 16)
     act_flops = 2.0 * gemm_flops       # activated FLOPs of the layer (Eq. 35 blocks)
+    # a forward of more than pass_tokens tokens runs in passes; the stage
+    # events of the per-kernel pass time the last one, tokens [last0, T)
+    P = layer.pass_tokens()
+    n_pass = (T + P - 1) // P
+    last0 = (n_pass - 1) * P
+    T_last = T - last0
+    cb_last = int(cb[last0:].sum())
+    stage_flops = 2.0 * d * M * cb_last  # one grouped GEMM launch of the last pass
 
     K = args.steps
     mk = lambda: torch.cuda.Event(enable_timing=True)
@@ -439,7 +447,7 @@ def main():
     # roofline of the dominant kernel (the larger grouped GEMM), timed in the
     # per-kernel pass
     dom = "up_gemm" if stage_ms["up_gemm"] >= stage_ms["down_gemm"] else "down_gemm"
-    ach = gemm_flops / (stage_ms[dom] / 1e3) / 1e12
+    ach = stage_flops / (stage_ms[dom] / 1e3) / 1e12
     traffic = measured_traffic(s.name, dom)
     # algorithmic bytes of the memory-bound kernels (per forward): the router
     # reads x and writes each token's records (alpha, b, k, two masks, K
@@ -447,10 +455,10 @@ def main():
     # one (token, weight) row per pair; the permute writes those rows; the
     # combine reads the fp32 accumulator and writes the output
     fused = layer.kernels_per_forward() <= 5 and s.dtype == "bf16"
-    router_bytes = (T * d * elt + T * (4 * 3 + 8 * 2 + 4 * s.n_experts + 8) +
-                    (8 * sum_cb if fused else 0))
-    combine_bytes = T * d * (4 + elt)
-    permute_bytes = sum_cb * 8
+    router_bytes = (T_last * d * elt + T_last * (4 * 3 + 8 * 2 + 4 * s.n_experts + 8) +
+                    (8 * cb_last if fused else 0))
+    combine_bytes = T_last * d * (4 + elt)
+    permute_bytes = cb_last * 8
 
     def hbm_stage(ms_, nbytes):
         gbs = nbytes / ms_ / 1e6
@@ -461,11 +469,13 @@ def main():
         "router": hbm_stage(stage_ms["router"], router_bytes),
         "permute": (hbm_stage(stage_ms["permute"], permute_bytes) if not fused else
                     {"ms": 0.0, "fused_into": "router", "event_gap_ms": stage_ms["permute"]}),
-        "up_gemm": {"ms": stage_ms["up_gemm"], "TFLOP/s": gemm_flops / stage_ms["up_gemm"] / 1e9,
-                    "frac_of_burst_bf16": gemm_flops / stage_ms["up_gemm"] / 1e9 / peak_tf},
+        "up_gemm": {"ms": stage_ms["up_gemm"], "TFLOP/s": stage_flops / stage_ms["up_gemm"] / 1e9,
+                    "frac_of_burst_bf16": stage_flops / stage_ms["up_gemm"] / 1e9 / peak_tf},
         "down_gemm": {"ms": stage_ms["down_gemm"],
-                      "TFLOP/s": gemm_flops / stage_ms["down_gemm"] / 1e9,
-                      "frac_of_burst_bf16": gemm_flops / stage_ms["down_gemm"] / 1e9 / peak_tf},
+                      "TFLOP/s": stage_flops / stage_ms["down_gemm"] / 1e9,
+                      "frac_of_burst_bf16": stage_flops / stage_ms["down_gemm"] / 1e9 / peak_tf},
+        "timed_pass": {"passes_per_forward": n_pass, "pass_tokens": P,
+                       "tokens": [last0, T]},
         "combine": hbm_stage(stage_ms["combine"], combine_bytes),
     }
     import numpy as np
@@ -503,7 +513,7 @@ def main():
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": statistics.fmean(e2e_ms)},
         # (a norm-first sublayer adds its layer-normalisation kernel)
-        "gpu_launches": (layer.kernels_per_forward() + (args.sublayer == "pre")) * K,
+        "gpu_launches": (layer.kernels_per_forward() * n_pass + (args.sublayer == "pre")) * K,
         "clocks": clocks,
     }
     if not args.no_cpu_baseline and world >= 1:

@@ -205,7 +205,9 @@ UNIF_MOE_API int unif_moe_get_routing(unif_moe_t h, float* alpha_dev, uint64_t* 
                          uint64_t* expert_mask_dev, int32_t* q_dev, float* p_dev,
                          void* stream);
 
-/* Copies the (expert, block) group table of the last forward to host memory.
+/* Copies the (expert, block) group table of the last forward to host memory
+ * (of its last pass, tokens [T - n, T), when it ran in passes: see
+ * unif_moe_pass_tokens).
  * Group g = e*B + b for e = 0 (shared expert) or e = 1+j (residual expert j),
  * G = (K+1)*B groups. counts_host [G] receives each group's row count; the
  * rows of group g are listed in increasing token order at
@@ -224,17 +226,28 @@ UNIF_MOE_API int unif_moe_get_groups(unif_moe_t h, int32_t* counts_host, int32_t
  * stream at the stage boundaries: [0] before the router, [1] after the
  * router (Eqs. 17-27), [2] after the permute (grouping of Eqs. 28-29),
  * [3] after the up-projection GEMM + GeLU, [4] after the down-projection
- * GEMM (Eq. 16), [5] after the combine (Eq. 30). NULL stops the recording.
+ * GEMM (Eq. 16), [5] after the combine (Eq. 30). A forward that runs in
+ * passes records them around its last pass. NULL stops the recording.
  * The caller keeps the events alive while they are set. */
 UNIF_MOE_API int unif_moe_set_stage_events(unif_moe_t h, void* const* events);
 
-/* Upper bound on group-table rows (padded) of a forward at max_tokens. */
+/* Upper bound on group-table rows (padded) of one pass of a forward. */
 UNIF_MOE_API int64_t unif_moe_max_rows(unif_moe_t h);
 
-/* Number of kernels one unif_moe_forward launches with T > 0 (the same for
- * every T): 4 for bf16 layers whose router also groups the pairs (router,
- * up projection, down projection, combine), else 6 (router, group scan,
- * group scatter, up, down, combine). -1 for a NULL handle. */
+/* Tokens per pass: bf16 layers run a forward of more tokens in consecutive
+ * passes of this many tokens (the last one shorter), each pass the whole
+ * layer (Eqs. 17-30) over its tokens, so that the fp32 output accumulator
+ * of one pass (pass_tokens * d * 4 bytes, at most 128 MiB) stays resident
+ * in L2. Results do not depend on it. max_tokens when a forward always runs
+ * in one pass; -1 for a NULL handle. */
+UNIF_MOE_API int unif_moe_pass_tokens(unif_moe_t h);
+
+/* Number of kernels one pass of unif_moe_forward launches (a forward of
+ * T > 0 tokens runs ceil(T / unif_moe_pass_tokens) passes): 4 for bf16
+ * layers whose router also groups the pairs (router, up projection, down
+ * projection, combine), 5 when a streaming GEMM reads a tile list, else 6
+ * (router, group scan, group scatter, up, down, combine). -1 for a NULL
+ * handle. */
 UNIF_MOE_API int unif_moe_kernels_per_forward(unif_moe_t h);
 
 /* Waits for `stream`, then reads and clears the handle's device status word.

@@ -33,7 +33,8 @@ EXPORTS = ["unif_moe_default_thresholds", "unif_moe_default_options", "unif_moe_
            "unif_moe_create_ex", "unif_moe_load_weights",
            "unif_moe_load_upcycled", "unif_moe_forward", "unif_moe_sublayer_forward",
            "unif_moe_forward_host", "unif_moe_get_routing",
-           "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_kernels_per_forward",
+           "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_pass_tokens",
+           "unif_moe_kernels_per_forward",
            "unif_moe_set_stage_events",
            "unif_moe_sync_status", "unif_moe_selftest_timeout", "unif_moe_group_noalloc",
            "unif_moe_destroy", "unif_moe_last_error"]
@@ -85,6 +86,7 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_get_groups.argtypes = [P, P, P, P, P, C.POINTER(C.c_int64), P]
         L.unif_moe_max_rows.argtypes = [P]
         L.unif_moe_max_rows.restype = C.c_int64
+        L.unif_moe_pass_tokens.argtypes = [P]
         L.unif_moe_kernels_per_forward.argtypes = [P]
         L.unif_moe_set_stage_events.argtypes = [P, P]
         L.unif_moe_sync_status.argtypes = [P, P]
@@ -232,6 +234,10 @@ class Layer:
 
     def max_rows(self) -> int:
         return int(lib().unif_moe_max_rows(self._h))
+
+    def pass_tokens(self) -> int:
+        """Tokens per pass: larger forwards run in passes of this many tokens."""
+        return int(lib().unif_moe_pass_tokens(self._h))
 
     def kernels_per_forward(self) -> int:
         return int(lib().unif_moe_kernels_per_forward(self._h))

@@ -104,12 +104,19 @@ struct unif_moe_layer {
   bool fused_group = false;
   int region_rows = 0;
   bool tile_list = false;  // a streaming GEMM reads the tile list: build it after the router
+  // A forward of more than pass_tokens tokens runs in passes of pass_tokens
+  // (bf16 layers): the fp32 accumulator rows of one pass stay in L2. rec0 is
+  // the first token of the pass being launched; the routing records of token
+  // t of the pass are at rec0 + t.
+  int pass_tokens = 0;
+  int rec0 = 0;
   unsigned features = 0;        // UNIF_MOE_FEATURE_* workspaces allocated at create time
   bool gemm_streaming = false;  // UNIF_MOE_GEMM_STREAMING: never the weight-stationary kernels
   int device = 0;
   bool loaded = false;
   bool y_dirty = false;  // accumulator / grouping counters may hold state of a forward cut short
   int last_T = -1;
+  int last_pass_T = 0;  // tokens of the last forward's last pass
   // Weights (device, owned).
   float* wr = nullptr;      // [d][router_cols_pad]: W_shr, W_g, mu_1..mu_B (fp32)
   __nv_bfloat16* wr_bf = nullptr;  // [router_cols_pad][d] the same matrix in bf16 (bf16 layers)

@@ -748,8 +748,9 @@ DecideArgs decide_args(unif_moe_layer* L, const uint8_t* mask, int T, int32_t* b
   a.bias = L->bias;
   a.tau = L->tau; a.alpha_fixed = L->th.alpha_fixed; a.beta_fixed = L->th.beta_fixed;
   a.topk_fixed = L->th.topk_fixed; a.prefix = L->th.prefix_blocks;
-  a.alpha = L->ws.alpha; a.b = L->ws.b; a.k = L->ws.k; a.shr = L->ws.shr_mask;
-  a.emask = L->ws.exp_mask; a.s = L->ws.s;
+  const size_t r0 = (size_t)L->rec0;  // the records of this pass's first token
+  a.alpha = L->ws.alpha + r0; a.b = L->ws.b + r0; a.k = L->ws.k + r0;
+  a.shr = L->ws.shr_mask + r0; a.emask = L->ws.exp_mask + r0; a.s = L->ws.s + r0 * L->K;
   a.bcnt = b_out; a.kcnt = k_out;
   a.chunk_cnt = L->ws.chunk_cnt; a.n_chunks = forward_chunks(T);
   return a;
@@ -799,9 +800,11 @@ cudaError_t router_setup(unif_moe_layer* L) {
 cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s) {
   const int n_chunks = forward_chunks(T);
   Workspace& w = L->ws;
+  const size_t r0 = (size_t)L->rec0;  // the records of this pass's first token
   chunk_scan_kernel<<<(L->G + 7) / 8, 256, 0, s>>>(L->G, n_chunks, w.chunk_cnt, w.grp_cnt);
   group_scatter_kernel<<<(n_chunks + 3) / 4, 128, scatter_smem(L), s>>>(
-      w.shr_mask, w.exp_mask, w.alpha, w.s, T, L->K, L->B, n_chunks, w.chunk_cnt, w.grp_cnt,
+      w.shr_mask + r0, w.exp_mask + r0, w.alpha + r0, w.s + r0 * L->K, T, L->K, L->B, n_chunks,
+      w.chunk_cnt, w.grp_cnt,
       w.grp_off, w.n_tiles, w.tile_group, w.tile_row0, w.tile_rows, w.row_tok, w.row_w);
   return cudaGetLastError();
 }

@@ -163,11 +163,22 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   L->tau = isnan(t.tau) ? (float)((double)(n_blocks - 1) / ((double)n_blocks * n_blocks)) : t.tau;
   const int kmax = t.topk_fixed > 0 ? t.topk_fixed : n_experts;
   L->cb_max = kmax * n_blocks;  // C_B = b + k (B - b) <= k B for every b >= 0 (Eq. 35)
-  const int64_t rows = (int64_t)max_tokens * L->cb_max + (int64_t)L->G * (unif::kTileRows - 1);
+  // bf16 layers: a forward runs in passes whose fp32 accumulator rows fit in
+  // 128 MiB, so that the down projection's reductions stay in the 129 MB L2
+  // (measured on GB300 for d = 1024: 62.5 us per 1,000 tokens at 65,536
+  // tokens in one pass, 54.7 at 32,768). The GEMM workspace is sized for one
+  // pass, the routing records for max_tokens.
+  L->pass_tokens = max_tokens;
+  if (dtype == UNIF_MOE_BF16) {
+    const long long fit = (128ll << 20) / (4ll * d_model) / unif::kTileRows * unif::kTileRows;
+    if (fit >= unif::kTileRows && fit < max_tokens) L->pass_tokens = (int)fit;
+  }
+  const int64_t rows =
+      (int64_t)L->pass_tokens * L->cb_max + (int64_t)L->G * (unif::kTileRows - 1);
   L->max_rows = (rows + unif::kTileRows - 1) / unif::kTileRows * unif::kTileRows;
   if (L->max_rows >= (int64_t)1 << 31) {
-    set_error("max_tokens=%d needs %lld group rows, above the int32 row index", max_tokens,
-              (long long)L->max_rows);
+    set_error("max_tokens=%d needs %lld group rows per pass, above the int32 row index",
+              max_tokens, (long long)L->max_rows);
     delete L;
     return UNIF_MOE_ERR_CAPACITY;
   }
@@ -213,14 +224,14 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   // max_tokens rows (rounded up to whole tiles) in the row arrays
   L->fused_group = dtype == UNIF_MOE_BF16 && L->router_cols_pad <= 160 &&
                    unif::router_can_group(L->router_cols_pad, L->K, L->G);
-  L->region_rows = (max_tokens + 127) / 128 * 128;
+  L->region_rows = (L->pass_tokens + 127) / 128 * 128;
   const size_t row_cap = L->fused_group ? (size_t)L->G * L->region_rows : (size_t)L->max_rows;
   ALLOC(w.row_tok, row_cap); ALLOC(w.row_w, row_cap);
   if (L->fused_group) ALLOC(w.grp_fill, (size_t)L->G);
   void* hb = nullptr;
   if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&hb), es * (size_t)L->max_rows * M);
   w.hbuf = hb;
-  ALLOC(w.y32, T * d_model);
+  ALLOC(w.y32, (size_t)L->pass_tokens * d_model);
   ALLOC(w.status, 1);
   // optional features: every buffer a later call needs, so that no later
   // call allocates
@@ -234,7 +245,8 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   }
 #undef ALLOC
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
-                            cudaMemset(w.y32, 0, sizeof(float) * T * d_model) != cudaSuccess ||
+                            cudaMemset(w.y32, 0, sizeof(float) * L->pass_tokens * d_model) !=
+                                cudaSuccess ||
                             (L->fused_group &&
                              (cudaMemset(w.grp_fill, 0, sizeof(int32_t) * L->G) != cudaSuccess ||
                               // rows hold token indices from the start, also any row a
@@ -304,20 +316,26 @@ static int forward_checks(unif_moe_t L, const void* x, void* out, int T,
   return UNIF_MOE_OK;
 }
 
-// The forward after the argument checks (T > 0); `sub` replaces the combine
-// with a sublayer's residual epilogue.
-static int forward_core(unif_moe_t L, const void* x, void* out, int T, const uint8_t* token_mask,
-                        int32_t* shared_counts, int32_t* residual_counts, cudaStream_t s,
-                        const SublayerEpilogue* sub) {
+// One pass of the forward over tokens [t0, t0 + T) of the caller's arrays
+// (x, out, mask, counts and, for a sublayer, the residual input already
+// offset to t0); `sub` replaces the combine with a sublayer's residual
+// epilogue. `timed`: record the stage events around this pass.
+static int forward_pass(unif_moe_t L, const void* x, void* out, int T, int t0,
+                        const uint8_t* token_mask, int32_t* shared_counts,
+                        int32_t* residual_counts, cudaStream_t s, const SublayerEpilogue* sub,
+                        bool timed) {
   cudaEvent_t* ev = L->stage_ev;
+  cudaEvent_t none[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+  if (!timed) ev = none;
   // The output accumulator and the grouping counters are all zero between
-  // forwards (each combine zeroes them). A forward that returned before
+  // passes (each combine zeroes them). A pass that returned before
   // launching its combine leaves them dirty: clear them first.
   if (L->y_dirty) {
-    CK(cudaMemsetAsync(L->ws.y32, 0, sizeof(float) * (size_t)L->max_tokens * L->d, s));
+    CK(cudaMemsetAsync(L->ws.y32, 0, sizeof(float) * (size_t)L->pass_tokens * L->d, s));
     if (L->fused_group) CK(cudaMemsetAsync(L->ws.grp_fill, 0, sizeof(int32_t) * L->G, s));
   }
   L->y_dirty = true;
+  L->rec0 = t0;
   if (ev[0]) CK(cudaEventRecord(ev[0], s));
   if (L->dtype == UNIF_MOE_BF16) {
     CK(unif::launch_router_tc(L, x, token_mask, T, shared_counts, residual_counts, s));
@@ -341,7 +359,33 @@ static int forward_core(unif_moe_t L, const void* x, void* out, int T, const uin
     CK(unif::launch_combine(L, out, T, s));
   L->y_dirty = false;
   if (ev[5]) CK(cudaEventRecord(ev[5], s));
+  return UNIF_MOE_OK;
+}
+
+// The forward after the argument checks (T > 0), in passes of at most
+// pass_tokens tokens; the stage events time the last pass.
+static int forward_core(unif_moe_t L, const void* x, void* out, int T, const uint8_t* token_mask,
+                        int32_t* shared_counts, int32_t* residual_counts, cudaStream_t s,
+                        const SublayerEpilogue* sub) {
+  const size_t row = elt_size(L) * (size_t)L->d;  // bytes per token row of x and out
+  const int P = L->pass_tokens;
+  for (int t0 = 0; t0 < T; t0 += P) {
+    const int n = T - t0 < P ? T - t0 : P;
+    const size_t off = (size_t)t0 * row;
+    SublayerEpilogue sp;
+    if (sub) {
+      sp = *sub;
+      sp.res = static_cast<const char*>(sub->res) + off;
+    }
+    const int rc = forward_pass(
+        L, static_cast<const char*>(x) + off, static_cast<char*>(out) + off, n, t0,
+        token_mask ? token_mask + t0 : nullptr, shared_counts ? shared_counts + t0 : nullptr,
+        residual_counts ? residual_counts + t0 : nullptr, s, sub ? &sp : nullptr, t0 + n >= T);
+    L->rec0 = 0;
+    if (rc != UNIF_MOE_OK) return rc;
+  }
   L->last_T = T;
+  L->last_pass_T = T - (T - 1) / P * P;
   return UNIF_MOE_OK;
 }
 
@@ -505,6 +549,9 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
     // (the combine copied the group sizes to grp_cnt; offsets pad each group
     // to whole 128-row tiles)
     std::vector<int32_t> cnt(L->G), off(L->G + 1);
+    // the table is that of the forward's last pass; its rows hold tokens
+    // relative to the pass's first token
+    const int tok_base = L->last_T - L->last_pass_T;
     CK(cudaMemcpyAsync(cnt.data(), L->ws.grp_cnt, sizeof(int32_t) * L->G, dh, s));
     CK(cudaStreamSynchronize(s));
     off[0] = 0;
@@ -530,7 +577,7 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
       for (size_t i = 0; i < n; ++i) ord[i] = i;
       std::sort(ord.begin(), ord.end(), [&](size_t a, size_t b) { return tok[a] < tok[b]; });
       for (size_t i = 0; i < n; ++i) {
-        if (row_token) row_token[off[g] + i] = tok[ord[i]];
+        if (row_token) row_token[off[g] + i] = tok_base + tok[ord[i]];
         if (row_weight) row_weight[off[g] + i] = wt[ord[i]];
       }
     }
@@ -549,6 +596,8 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
 }
 
 int64_t unif_moe_max_rows(unif_moe_t L) { return L ? L->max_rows : -1; }
+
+int unif_moe_pass_tokens(unif_moe_t L) { return L ? L->pass_tokens : -1; }
 
 int unif_moe_kernels_per_forward(unif_moe_t L) {
   if (!L) return -1;

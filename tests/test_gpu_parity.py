@@ -74,6 +74,27 @@ def test_stress_full_size():
     assert_parity(wl, g, rep)
 
 
+def test_forward_in_passes():
+    """d = 4096: the fp32 accumulator of 8,192 tokens fills the 128 MiB a pass
+    may use, so 8,969 tokens (text batch with padding, NaN-filled) run in two
+    passes, the second ragged. Decisions, counts and outputs of every token
+    match the oracle; the routing records cover both passes; the group table
+    is that of the last pass, with absolute token indices."""
+    s = workloads.spec("bert_base").with_(tokens=8969, d_model=4096, d_ff=1024, n_experts=2,
+                                          n_blocks=4)
+    wl = workloads.make_workload(s)
+    g = run_gpu(wl)
+    assert g.layer.pass_tokens() == 8192
+    m = wl.mask.numpy()
+    assert (g.y[m == 0] == 0).all() and np.isfinite(g.y).all()
+    assert_parity(wl, g, compare(wl, g, label="two passes"))
+    counts, offsets, tok, w = g.layer.groups()
+    real = tok.numpy()[tok.numpy() >= 0]
+    assert real.min() >= 8192 and real.max() < 8969
+    cb = g.b[8192:] + g.k[8192:] * (s.n_blocks - g.b[8192:])
+    assert int(counts.sum()) == int(cb[m[8192:] == 1].sum())
+
+
 # ------------------------------------------------------------- ragged sizes
 
 @pytest.mark.parametrize("T", [1, 7, 64, 129, 255, 257, 1000])
