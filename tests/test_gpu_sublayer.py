@@ -125,14 +125,14 @@ def test_sublayer_bert_padding(norm_first):
 
 @pytest.mark.parametrize("norm_first", [True, False])
 def test_sublayer_in_passes(norm_first):
-    """A sublayer forward that runs in two passes (d = 4096: 8,192 tokens per
+    """A sublayer forward that runs in two passes (d = 1024: 32,768 tokens per
     pass) adds the residual of each pass's own tokens."""
-    s = workloads.spec("bert_base").with_(tokens=8969, d_model=4096, d_ff=1024, n_experts=2,
+    s = workloads.spec("bert_base").with_(tokens=33468, d_model=1024, d_ff=1024, n_experts=2,
                                           n_blocks=4)
     wl = workloads.make_workload(s)
     gamma, beta = ln_params(s.d_model, torch.bfloat16, seed=10)
     g = run_sublayer(wl, gamma, beta, norm_first)
-    assert g.layer.pass_tokens() == 8192
+    assert g.layer.pass_tokens() == 32768
     check_sublayer(wl, g, gamma, beta, norm_first,
                    label="two passes, " + ("norm first" if norm_first else "norm after"))
 
