@@ -9,10 +9,13 @@ paper equation by equation (Eqs. 16-30); this module only compiles it, moves
 arrays in and out with ctypes, and chains the steps:
     prototypes (Eq. 20) -> route (Eqs. 17-27) -> forward (Eqs. 16, 28-30).
 `groups` lists the (expert, block) pairs the output sums over, grouped by
-pair (the bookkeeping behind Eq. 35). `upcycle` and `sublayer` place the
-layer the way the paper's backbones use it (Sec. III: experts initialised
-from one dense FFN; Appendix A, Architecture details: converted FFN layers of DeiT-S, normalised
-first, and of BERT, normalised after the residual sum).
+pair (the bookkeeping behind Eq. 35). `backward` and `diversity` are the
+training side (Sec. III-E): gradients through Eq. 30 with the discrete
+decisions held fixed, and the Gram regulariser of the router embeddings.
+`upcycle` and `sublayer` place the layer the way the paper's backbones use
+it (Sec. III: experts initialised from one dense FFN; Appendix A,
+Architecture details: converted FFN layers of DeiT-S, normalised first, and
+of BERT, normalised after the residual sum).
 """
 from __future__ import annotations
 
@@ -63,6 +66,9 @@ def _load():
             lib.oracle_groups.argtypes = [C.c_int] * 3 + [P] * 9 + [C.c_longlong]
             lib.oracle_groups.restype = C.c_longlong
             lib.oracle_layernorm.argtypes = [C.c_int, C.c_int, P, P, P, P, C.c_double, C.c_int, P]
+            lib.oracle_backward.argtypes = [C.c_int] * 5 + [P] * 15
+            lib.oracle_diversity.argtypes = [C.c_int, C.c_int, P, P]
+            lib.oracle_diversity.restype = C.c_double
             _lib = lib
     return _lib
 
@@ -283,3 +289,48 @@ def sublayer(x, w_router, w_up, w_down, B: int, gamma, beta, eps: float, norm_fi
     if mask is not None:
         out[_u8(mask) == 0] = 0.0
     return out, r
+
+
+@dataclass
+class Grads:
+    dx: np.ndarray         # [T][d]
+    dw_up: np.ndarray      # [K+1][H][d]
+    dw_down: np.ndarray    # [K+1][d][H]
+    dw_router: np.ndarray  # [d][K+1]
+    dbias: np.ndarray      # [K+1]
+
+
+def backward(x, w_router, w_up, w_down, shr_mask, expert_mask, B: int, dy,
+             th: Optional[Thresholds] = None, mask=None, bias=None) -> Grads:
+    """dL/d(inputs, parameters) given dL/dy, through Eq. 30 with the given
+    discrete decisions (shared block set and selected residual experts per
+    token) held fixed; alpha and s are recomputed from x and the router."""
+    xa = _f64(x)
+    T, d = xa.shape
+    wr = _f64(w_router)
+    wu = _f64(w_up)
+    wd = _f64(w_down)
+    g = _f64(dy)
+    K1, H = wu.shape[0], wu.shape[1]
+    th = th or Thresholds()
+    m = _u8(mask)
+    bias_a = None if bias is None else _f64(bias)
+    shr = np.ascontiguousarray(shr_mask, dtype=np.uint64)
+    em = np.ascontiguousarray(expert_mask, dtype=np.uint64)
+    out = Grads(dx=np.empty((T, d)), dw_up=np.empty((K1, H, d)), dw_down=np.empty((K1, d, H)),
+                dw_router=np.empty((d, K1)), dbias=np.empty(K1))
+    rc = _load().oracle_backward(T, d, H, K1 - 1, B, _p(xa), _p(m), _p(wr), _p(bias_a), _p(wu),
+                                 _p(wd), _p(th.array()), _p(shr), _p(em), _p(g), _p(out.dx),
+                                 _p(out.dw_up), _p(out.dw_down), _p(out.dw_router), _p(out.dbias))
+    if rc != 0:
+        raise ValueError("oracle_backward: bad arguments (%d)" % rc)
+    return out
+
+
+def diversity(w_router):
+    """Eq. diversity-loss: (L_div, dL_div/dW*) for W* = w_router [d][K+1]."""
+    wr = _f64(w_router)
+    d, K1 = wr.shape
+    grad = np.empty((d, K1))
+    L = _load().oracle_diversity(d, K1, _p(wr), _p(grad))
+    return float(L), grad

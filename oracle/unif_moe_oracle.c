@@ -362,3 +362,205 @@ int oracle_layernorm(int T, int d, const double* v, const uint8_t* mask, const d
   }
   return 0;
 }
+
+/* ------------------------------------------------------------------------
+ * Training (Sec. III-E): gradients of a loss through the layer output.
+ * ------------------------------------------------------------------------ */
+
+/* d GeLU / dv = Phi(v) + v phi(v), the derivative of the exact erf form. */
+static double gelu_grad(double v) {
+  return 0.5 * (1.0 + erf(v * M_SQRT1_2)) + v * exp(-0.5 * v * v) / sqrt(2.0 * M_PI);
+}
+
+/* Gradient of a scalar loss L given dL/dy (dy [T][d]) through the output of
+ * Eq. 30, with the discrete decisions held fixed: the shared block set
+ * (shr_mask, Eq. 22) and the set of selected residual experts (expert_mask,
+ * bit j = expert j, Eq. 27) are piecewise constant in the parameters (the
+ * rounding of Eq. 19, the TopK of Eq. 22 and the smallest prefix of Eq. 27
+ * move only at ties), so gradients flow through the pathway weights alpha
+ * (Eq. 18) and p_i = s_{q_i} (Eqs. 24-25), which are recomputed here from x
+ * and the router, and through the expert weights (Eq. 16). With alpha fixed
+ * (th[1] not NaN) it has no gradient; the prototypes mu_b only rank blocks
+ * and receive none.
+ *   y = alpha sum_{b in I_shr} E_shr^(b) + sum_{j selected} s_j sum_{b not in I_shr} E_j^(b)
+ * Per token and block channel h of expert e with weight w (alpha or s_j),
+ * a = x K_e[:, h]:
+ *   dL/dV_e[h, :] += w GeLU(a) dy,   dL/da = w (dy . V_e[h, :]) GeLU'(a),
+ *   dL/dK_e[:, h] += (dL/da) x,      dL/dx += (dL/da) K_e[:, h],
+ *   dL/dw += GeLU(a) (dy . V_e[h, :]);
+ * then alpha = tau + (1 - 2 tau) sigmoid(z_0) and s = softmax(z_1..z_K),
+ * z = x W* + bias, give dL/dz and dL/dW* = x^T dL/dz, dL/dbias = dL/dz,
+ * dL/dx += dL/dz W*^T.
+ * Outputs (overwritten): dx [T][d], dw_up [K+1][H][d], dw_down [K+1][d][H],
+ * dw_router [d][K+1], dbias [K+1] or NULL. Padding tokens (mask 0) add
+ * nothing and get dx = 0. */
+int oracle_backward(int T, int d, int H, int K, int B, const double* x, const uint8_t* mask,
+                    const double* w_router, const double* bias, const double* w_up,
+                    const double* w_down, const double* th, const uint64_t* shr_mask,
+                    const uint64_t* expert_mask, const double* dy, double* dx,
+                    double* dw_up, double* dw_down, double* dw_router, double* dbias) {
+  if (T < 0 || d <= 0 || H <= 0 || K <= 0 || K > ORACLE_MAX_K || B <= 0 || H % B ||
+      B > ORACLE_MAX_B)
+    return -1;
+  const int M = H / B;
+  const int K1 = K + 1;
+  const double tau = isnan(th[0]) ? (double)(B - 1) / ((double)B * B) : th[0];
+  const int adaptive = isnan(th[1]);
+  double* dz = (double*)calloc((size_t)T * K1, sizeof(double));
+  if (!dz) return -2;
+
+  /* The pathway weight of expert e for token t (0: not used by t). */
+#define PATH_WEIGHT(e, alpha_t, s_t, t)                                                 \
+  ((e) == 0 ? (shr_mask[t] != 0 ? (alpha_t) : 0.0)                                     \
+            : (((expert_mask[t] >> ((e) - 1)) & 1ull) ? (s_t)[(e) - 1] : 0.0))
+  /* Whether expert e runs block blk for token t (Eqs. 28-29). */
+#define RUNS_BLOCK(e, blk, t) \
+  ((e) == 0 ? (int)((shr_mask[t] >> (blk)) & 1ull) : !(int)((shr_mask[t] >> (blk)) & 1ull))
+
+  /* Router scores of token t: alpha (Eq. 18) and s (Eq. 24) from z = x W* + bias. */
+#define ROUTER_SCORES(t, z, alpha_t, s_t)                                               \
+  do {                                                                                  \
+    const double* xt_ = x + (size_t)(t) * d;                                            \
+    for (int c = 0; c < K1; ++c) {                                                      \
+      double acc = 0.0;                                                                 \
+      for (int i = 0; i < d; ++i) acc += xt_[i] * w_router[(size_t)i * K1 + c];         \
+      (z)[c] = acc + (bias ? bias[c] : 0.0);                                            \
+    }                                                                                   \
+    (alpha_t) = adaptive ? tau + (1.0 - 2.0 * tau) * sigmoid((z)[0]) : th[1];            \
+    double zm = (z)[1];                                                                 \
+    for (int j = 2; j <= K; ++j) zm = (z)[j] > zm ? (z)[j] : zm;                        \
+    double den = 0.0;                                                                   \
+    for (int j = 0; j < K; ++j) { (s_t)[j] = exp((z)[j + 1] - zm); den += (s_t)[j]; }  \
+    for (int j = 0; j < K; ++j) (s_t)[j] /= den;                                        \
+  } while (0)
+
+  /* Pass 1, per token: dL/dx through the experts, dL/dalpha and dL/ds, then
+   * dL/dz and its share of dL/dx. */
+#pragma omp parallel for schedule(dynamic, 16)
+  for (int t = 0; t < T; ++t) {
+    double* dxt = dx + (size_t)t * d;
+    for (int i = 0; i < d; ++i) dxt[i] = 0.0;
+    if (mask && !mask[t]) continue;
+    const double* xt = x + (size_t)t * d;
+    const double* gt = dy + (size_t)t * d;
+    double z[ORACLE_MAX_K + 1], s[ORACLE_MAX_K], dw[ORACLE_MAX_K + 1];
+    double alpha;
+    ROUTER_SCORES(t, z, alpha, s);
+    for (int e = 0; e < K1; ++e) {
+      dw[e] = 0.0;
+      const double w = PATH_WEIGHT(e, alpha, s, t);
+      if (e > 0 && !((expert_mask[t] >> (e - 1)) & 1ull)) continue;
+      if (e == 0 && shr_mask[t] == 0) continue;
+      for (int blk = 0; blk < B; ++blk) {
+        if (!RUNS_BLOCK(e, blk, t)) continue;
+        for (int h = blk * M; h < (blk + 1) * M; ++h) {
+          const double* key = w_up + ((size_t)e * H + h) * d;
+          double a = 0.0, gv = 0.0;
+          for (int i = 0; i < d; ++i) a += xt[i] * key[i];
+          for (int i = 0; i < d; ++i) gv += gt[i] * w_down[((size_t)e * d + i) * H + h];
+          dw[e] += gelu(a) * gv;
+          const double da = w * gv * gelu_grad(a);
+          for (int i = 0; i < d; ++i) dxt[i] += da * key[i];
+        }
+      }
+    }
+    /* Eq. 18: d alpha / d z_0 = (1 - 2 tau) sigma (1 - sigma). */
+    double* dzt = dz + (size_t)t * K1;
+    if (adaptive) {
+      const double sg = sigmoid(z[0]);
+      dzt[0] = dw[0] * (1.0 - 2.0 * tau) * sg * (1.0 - sg);
+    }
+    /* Eq. 24: softmax Jacobian, ds -> dz_j = s_j (ds_j - sum_l s_l ds_l). */
+    double dot = 0.0;
+    for (int j = 0; j < K; ++j) dot += s[j] * dw[1 + j];
+    for (int j = 0; j < K; ++j) dzt[1 + j] = s[j] * (dw[1 + j] - dot);
+    for (int c = 0; c < K1; ++c)
+      for (int i = 0; i < d; ++i) dxt[i] += dzt[c] * w_router[(size_t)i * K1 + c];
+  }
+
+  /* Pass 2, per expert channel (e, h): the weight gradients, summed over the
+   * tokens that run h's block of expert e. */
+#pragma omp parallel for schedule(dynamic, 4)
+  for (int eh = 0; eh < K1 * H; ++eh) {
+    const int e = eh / H, h = eh % H, blk = h / M;
+    double* gk = dw_up + ((size_t)e * H + h) * d;
+    for (int i = 0; i < d; ++i) {
+      gk[i] = 0.0;
+      dw_down[((size_t)e * d + i) * H + h] = 0.0;
+    }
+    const double* key = w_up + ((size_t)e * H + h) * d;
+    for (int t = 0; t < T; ++t) {
+      if (mask && !mask[t]) continue;
+      if (!RUNS_BLOCK(e, blk, t)) continue;
+      if (e > 0 && !((expert_mask[t] >> (e - 1)) & 1ull)) continue;
+      const double* xt = x + (size_t)t * d;
+      const double* gt = dy + (size_t)t * d;
+      double z[ORACLE_MAX_K + 1], s[ORACLE_MAX_K];
+      double alpha;
+      ROUTER_SCORES(t, z, alpha, s);
+      const double w = PATH_WEIGHT(e, alpha, s, t);
+      double a = 0.0, gv = 0.0;
+      for (int i = 0; i < d; ++i) a += xt[i] * key[i];
+      for (int i = 0; i < d; ++i) gv += gt[i] * w_down[((size_t)e * d + i) * H + h];
+      const double da = w * gv * gelu_grad(a);
+      const double wg = w * gelu(a);
+      for (int i = 0; i < d; ++i) {
+        gk[i] += da * xt[i];
+        dw_down[((size_t)e * d + i) * H + h] += wg * gt[i];
+      }
+    }
+  }
+
+  /* Pass 3: dL/dW* = x^T dL/dz (Eq. 17), dL/dbias = sum_t dL/dz. */
+#pragma omp parallel for schedule(static)
+  for (int i = 0; i < d; ++i) {
+    for (int c = 0; c < K1; ++c) {
+      double acc = 0.0;
+      for (int t = 0; t < T; ++t)
+        if (!mask || mask[t]) acc += x[(size_t)t * d + i] * dz[(size_t)t * K1 + c];
+      dw_router[(size_t)i * K1 + c] = acc;
+    }
+  }
+  if (dbias) {
+    for (int c = 0; c < K1; ++c) {
+      double acc = 0.0;
+      for (int t = 0; t < T; ++t)
+        if (!mask || mask[t]) acc += dz[(size_t)t * K1 + c];
+      dbias[c] = acc;
+    }
+  }
+#undef PATH_WEIGHT
+#undef RUNS_BLOCK
+#undef ROUTER_SCORES
+  free(dz);
+  return 0;
+}
+
+/* Gram regulariser of the router embeddings (Eq. diversity-loss):
+ *   L_div = || W*^T W* - I_{K+1} ||_F,  W* = w_router [d][K+1],
+ * and, with A = W*^T W* - I (symmetric), its gradient
+ *   dL_div / dW* = 2 W* A / L_div   (0 where L_div = 0).
+ * grad [d][K+1] may be NULL. Returns L_div. */
+double oracle_diversity(int d, int K1, const double* w_router, double* grad) {
+  double* A = (double*)malloc(sizeof(double) * (size_t)K1 * K1);
+  if (!A) return NAN;
+  double ss = 0.0;
+  for (int a = 0; a < K1; ++a)
+    for (int b = 0; b < K1; ++b) {
+      double g = 0.0;
+      for (int i = 0; i < d; ++i) g += w_router[(size_t)i * K1 + a] * w_router[(size_t)i * K1 + b];
+      A[a * K1 + b] = g - (a == b ? 1.0 : 0.0);
+      ss += A[a * K1 + b] * A[a * K1 + b];
+    }
+  const double L = sqrt(ss);
+  if (grad) {
+    for (int i = 0; i < d; ++i)
+      for (int b = 0; b < K1; ++b) {
+        double g = 0.0;
+        for (int a = 0; a < K1; ++a) g += w_router[(size_t)i * K1 + a] * A[a * K1 + b];
+        grad[(size_t)i * K1 + b] = L > 0.0 ? 2.0 * g / L : 0.0;
+      }
+  }
+  free(A);
+  return L;
+}

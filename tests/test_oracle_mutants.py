@@ -42,7 +42,8 @@ MUTANTS = {
     # round() replaced by truncation (Eq. 19)
     "b_truncated": ("int b = (int)nearbyint((double)B * alpha);", "int b = (int)((double)B * alpha);"),
     # GeLU without the 1/sqrt(2) scaling
-    "gelu_scale": ("erf(v * M_SQRT1_2)", "erf(v)"),
+    "gelu_scale": ("return 0.5 * v * (1.0 + erf(v * M_SQRT1_2));",
+                   "return 0.5 * v * (1.0 + erf(v));"),
     # layer normalisation with the unbiased (1/(d-1)) variance
     "ln_unbiased_variance": ("    var /= (double)d;", "    var /= (double)(d - 1);"),
     # eps added outside the square root
@@ -69,6 +70,27 @@ MUTANTS = {
                           "for (int i = 0; i < k; ++i) prev += p[i];"),
     # margin (iii) one-sided (only the distance above beta)
     "margin_iii_one_sided": ("mg[2] = fmin(P_k - beta, beta - prev);", "mg[2] = P_k - beta;"),
+    # training: GeLU derivative without the v phi(v) term
+    "gelu_grad_phi_only": ("return 0.5 * (1.0 + erf(v * M_SQRT1_2)) + v * exp(-0.5 * v * v) / sqrt(2.0 * M_PI);",
+                           "return 0.5 * (1.0 + erf(v * M_SQRT1_2));"),
+    # sigmoid derivative without the (1 - sigma) factor
+    "dalpha_sigmoid": ("dw[0] * (1.0 - 2.0 * tau) * sg * (1.0 - sg)", "dw[0] * (1.0 - 2.0 * tau) * sg"),
+    # the (1 - 2 tau) scale of Eq. 18 left out of the chain rule
+    "dalpha_scale": ("dw[0] * (1.0 - 2.0 * tau) * sg * (1.0 - sg)", "dw[0] * sg * (1.0 - sg)"),
+    # softmax Jacobian without the mean term
+    "softmax_jacobian": ("dzt[1 + j] = s[j] * (dw[1 + j] - dot);", "dzt[1 + j] = s[j] * dw[1 + j];"),
+    # value gradient with the pre-activation instead of GeLU of it
+    "dv_preactivation": ("const double wg = w * gelu(a);", "const double wg = w * a;"),
+    # key gradient without the pathway weight
+    "dk_unweighted": ("      const double da = w * gv * gelu_grad(a);\n      const double wg",
+                      "      const double da = gv * gelu_grad(a);\n      const double wg"),
+    # router gradient to x through the transposed router matrix
+    "dx_router_transposed": ("dxt[i] += dzt[c] * w_router[(size_t)i * K1 + c];",
+                             "dxt[i] += dzt[c] * w_router[(size_t)c * d + i];"),
+    # Gram regulariser gradient without the factor 2
+    "gram_grad_half": ("2.0 * g / L : 0.0", "g / L : 0.0"),
+    # Gram matrix without the identity subtracted
+    "gram_no_identity": ("A[a * K1 + b] = g - (a == b ? 1.0 : 0.0);", "A[a * K1 + b] = g;"),
 }
 
 # Mistakes planted in the Python side of the oracle (oracle/__init__.py).

@@ -651,3 +651,109 @@ def test_upcycled_experts_closed_form(oracle_mod):
         Pk = float(np.sum(r.p[t, :r.k[t]]))
         ref = sum(r.alpha[t] * Eb[t, blk] if shr[blk] else Pk * Eb[t, blk] for blk in range(B))
         np.testing.assert_allclose(y[t], ref, rtol=1e-12, atol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# Training (Sec. III-E): gradients through Eq. 30 and the Gram regulariser
+# --------------------------------------------------------------------------
+
+def fixed_decision_loss(x, w_router, w_up, w_down, bias, B, th, shr, em, dy, mask=None):
+    """<dy, y> with y the oracle's forward for the given discrete decisions
+    (shared block sets, selected experts) and alpha, s recomputed from the
+    perturbed parameters: a smooth function of every parameter."""
+    K = w_up.shape[0] - 1
+    mu = oracle.prototypes(w_up, B, oracle.ROUND_NONE)
+    r = oracle.route(x, w_router, mu, K, B, th, mask, bias)
+    y = oracle.forward(x, w_up, w_down, oracle.with_decisions(r, shr, em, B), B, mask)
+    return float(np.sum(dy * y))
+
+
+def central_differences(f, arrays, eps=1e-6):
+    """dL/da for every entry of every array by (f(a + eps) - f(a - eps)) / 2 eps."""
+    out = []
+    for a in arrays:
+        g = np.zeros_like(a)
+        flat, gf = a.reshape(-1), g.reshape(-1)
+        for i in range(flat.size):
+            keep = flat[i]
+            flat[i] = keep + eps
+            fp = f()
+            flat[i] = keep - eps
+            fm = f()
+            flat[i] = keep
+            gf[i] = (fp - fm) / (2 * eps)
+        out.append(g)
+    return out
+
+
+@pytest.mark.parametrize("th,masked", [(Thresholds(), False), (Thresholds(), True),
+                                       (Thresholds(alpha_fixed=0.4, topk_fixed=2), False),
+                                       (Thresholds(beta_fixed=0.8, prefix_blocks=1), True)])
+def test_backward_matches_finite_differences(oracle_mod, th, masked):
+    """Every gradient of the oracle's backward (x, keys, values, router
+    columns, router bias) against central differences of the pinned forward,
+    the discrete decisions held at the unperturbed ones."""
+    rng = np.random.default_rng(31)
+    T, d, H, K, B = 7, 4, 8, 3, 4
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, router_scale=3.0, T=T)
+    bias = rng.normal(0.0, 0.5, K + 1)
+    dy = rng.standard_normal((T, d))
+    mask = np.array([1, 0, 1, 1, 0, 1, 1], np.uint8) if masked else None
+    _, r = oracle.layer(x, w_router, w_up, w_down, B, th, mask=mask, bias=bias)
+    shr, em = r.shr_mask.copy(), r.expert_mask()
+    g = oracle.backward(x, w_router, w_up, w_down, shr, em, B, dy, th, mask, bias)
+    f = lambda: fixed_decision_loss(x, w_router, w_up, w_down, bias, B, th, shr, em, dy, mask)
+    num = central_differences(f, [x, w_up, w_down, w_router, bias])
+    for got, want in zip([g.dx, g.dw_up, g.dw_down, g.dw_router, g.dbias], num):
+        np.testing.assert_allclose(got, want, rtol=1e-6, atol=1e-8)
+    if masked:
+        assert (g.dx[mask == 0] == 0).all()
+    if not math.isnan(th.alpha_fixed):
+        assert (g.dw_router[:, 0] == 0).all()  # alpha fixed: no gradient to W_shr
+
+
+def test_backward_dense_ffn_closed_form(oracle_mod):
+    """alpha fixed at 1: y = GeLU(x K_shr) V_shr (every block shared), so
+    dV = dy^T GeLU(A), dA = (dy V) * GeLU'(A) with GeLU'(a) = Phi(a) + a phi(a)
+    (normal CDF and density from the library), dK = dA^T x, dx = dA K; the
+    router gets nothing (alpha fixed; the residual expert runs no block)."""
+    rng = np.random.default_rng(32)
+    T, d, H, K, B = 30, 12, 32, 3, 4
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, T=T)
+    dy = rng.standard_normal((T, d))
+    th = Thresholds(alpha_fixed=1.0)
+    _, r = oracle.layer(x, w_router, w_up, w_down, B, th)
+    g = oracle.backward(x, w_router, w_up, w_down, r.shr_mask, r.expert_mask(), B, dy, th)
+    A = x @ w_up[0].T
+    gA = (dy @ w_down[0]) * (norm.cdf(A) + A * norm.pdf(A))
+    np.testing.assert_allclose(g.dw_down[0], dy.T @ gelu_ref(A), rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(g.dw_up[0], gA.T @ x, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(g.dx, gA @ w_up[0], rtol=1e-12, atol=1e-12)
+    assert (g.dw_up[1:] == 0).all() and (g.dw_down[1:] == 0).all()
+    assert (g.dw_router == 0).all() and (g.dbias == 0).all()
+
+
+@pytest.mark.parametrize("c", [0.5, 1.0, 1.7])
+def test_diversity_closed_form(oracle_mod, c):
+    """W* = c Q with Q's K+1 columns orthonormal: W*^T W* - I = (c^2 - 1) I, so
+    L_div = |c^2 - 1| sqrt(K+1) and dL_div/dW* = 2 c sign(c^2 - 1) Q / sqrt(K+1)
+    (Eq. diversity-loss); orthonormal columns (c = 1) give 0."""
+    rng = np.random.default_rng(33)
+    d, K1 = 16, 5
+    Q, _ = np.linalg.qr(rng.standard_normal((d, K1)))
+    L, grad = oracle.diversity(c * Q)
+    np.testing.assert_allclose(L, abs(c * c - 1) * math.sqrt(K1), rtol=1e-12, atol=1e-13)
+    if c == 1.0:
+        return  # the norm has no gradient at 0 (L is rounding noise here)
+    want = 2 * c * np.sign(c * c - 1) * Q / math.sqrt(K1)
+    np.testing.assert_allclose(grad, want, rtol=1e-11, atol=1e-12)
+
+
+def test_diversity_finite_differences(oracle_mod):
+    rng = np.random.default_rng(34)
+    W = rng.standard_normal((6, 4)) * 0.7
+    L, grad = oracle.diversity(W)
+    G = np.linalg.norm(W.T @ W - np.eye(4))  # Frobenius norm, library routine
+    assert L == pytest.approx(G, rel=1e-13)
+    num, = central_differences(lambda: oracle.diversity(W)[0], [W])
+    np.testing.assert_allclose(grad, num, rtol=1e-7, atol=1e-9)
