@@ -81,7 +81,11 @@ enum {
                                       a [max_tokens][d] buffer for LN(x) */
   UNIF_MOE_FEATURE_HOST_IO = 2,    /* unif_moe_forward_host: device staging
                                       buffers for x, y, the mask and the counts */
-  UNIF_MOE_FEATURES_ALL = 3
+  UNIF_MOE_FEATURE_BACKWARD = 4,   /* unif_moe_backward: transposed copies of the
+                                      expert weights and per-row gradient buffers
+                                      (bf16 layers, d % 128 == 0) */
+  UNIF_MOE_FEATURES_DEFAULT = 3,   /* what unif_moe_create allocates */
+  UNIF_MOE_FEATURES_ALL = 7
 };
 /* Grouped GEMM kernels: the library picks the weight-stationary kernels
  * where a group's weight slice fits in shared memory, else the streaming
@@ -94,7 +98,8 @@ typedef struct {
   int gemm_kernels;      /* UNIF_MOE_GEMM_AUTO or UNIF_MOE_GEMM_STREAMING */
 } unif_moe_options;
 
-/* Fills *opts with the defaults of unif_moe_create: every feature, AUTO. */
+/* Fills *opts with the defaults of unif_moe_create: UNIF_MOE_FEATURES_DEFAULT
+ * (norm-first sublayer and host-buffer forward), AUTO. */
 UNIF_MOE_API void unif_moe_default_options(unif_moe_options* opts);
 
 /* Creates a layer (Sec. III-A): d_model = d, d_ff = H, n_experts = K residual
@@ -103,8 +108,8 @@ UNIF_MOE_API void unif_moe_default_options(unif_moe_options* opts);
  * Limits: 2 <= B <= 64, 1 <= K <= 64, H % B == 0, d % 8 == 0; for
  * UNIF_MOE_BF16 also d % 64 == 0 and M = H/B a multiple of 64.
  * Device workspace for max_tokens is allocated here, sized for the largest
- * possible C_B (Eq. 35) under th, with every optional feature's buffers
- * (UNIF_MOE_FEATURES_ALL); no later call allocates device memory.
+ * possible C_B (Eq. 35) under th, with the buffers of the default features
+ * (UNIF_MOE_FEATURES_DEFAULT); no later call allocates device memory.
  * Errors: ERR_ARG (out == NULL, bad values), ERR_SHAPE, ERR_CUDA (allocation). */
 UNIF_MOE_API int unif_moe_create(unif_moe_t* out, int d_model, int d_ff, int n_experts, int n_blocks,
                     const unif_moe_thresholds* th, unif_moe_dtype dtype, int max_tokens);
@@ -192,6 +197,36 @@ UNIF_MOE_API int unif_moe_sublayer_forward(unif_moe_t h, const void* x_dev, void
 UNIF_MOE_API int unif_moe_forward_host(unif_moe_t h, const void* x_host, void* out_host, int T,
                           const uint8_t* token_mask_host, int32_t* shared_counts_host,
                           int32_t* residual_counts_host, void* stream);
+
+/* Backward pass of the last forward for training (Sec. III-E): given
+ * dL/dy, the gradients of L with respect to x and to every parameter of
+ * the layer, with the discrete decisions of that forward held fixed (the
+ * rounding of Eq. 19, the TopK of Eq. 22 and the smallest prefix of Eq. 27
+ * are piecewise constant): gradients flow through the pathway weights alpha
+ * (Eq. 18) and s_j (Eq. 24) and through the experts (Eq. 16); the block
+ * prototypes mu_b only rank blocks and have none. With lambda_div != 0 the
+ * Gram regulariser L_div = ||W*^T W* - I_{K+1}||_F (Eq. diversity-loss) adds
+ * lambda_div dL_div/dW* to the router gradient (the total loss of Eq. loss).
+ *   x_dev  [T][d]   the input of that forward (layer dtype), unchanged
+ *   dy_dev [T][d]   dL/dy (layer dtype)
+ *   token_mask_dev  as given to that forward (padding gets dx = 0)
+ * Outputs (fp32, device, overwritten):
+ *   dx_dev        [T][d]        dL/dx
+ *   dw_up_dev     [K+1][H][d]   dL/dw_up (the layout of unif_moe_load_weights)
+ *   dw_down_dev   [K+1][d][H]   dL/dw_down
+ *   dw_router_dev [d][K+1]      dL/dw_router (+ lambda_div dL_div/dW*)
+ *   dbias_dev     [K+1] or NULL dL/d router bias
+ *   l_div_dev     [1] or NULL   L_div
+ * The weights are those last loaded. Needs a bf16 handle created with
+ * UNIF_MOE_FEATURE_BACKWARD (ERR_STATE otherwise) and a forward of the same
+ * T that ran in one pass (T <= unif_moe_pass_tokens; ERR_CAPACITY
+ * otherwise); enqueued on `stream` after that forward, no sync. Pointers
+ * 16-byte aligned. Errors: ERR_ARG, ERR_STATE, ERR_CAPACITY, ERR_CUDA. */
+UNIF_MOE_API int unif_moe_backward(unif_moe_t h, const void* x_dev, const void* dy_dev, int T,
+                                   const uint8_t* token_mask_dev, float* dx_dev,
+                                   float* dw_up_dev, float* dw_down_dev, float* dw_router_dev,
+                                   float* dbias_dev, float lambda_div, float* l_div_dev,
+                                   void* stream);
 
 /* Copies the decisions of the last forward (T tokens) to device buffers; any
  * pointer may be NULL:

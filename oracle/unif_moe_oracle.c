@@ -407,7 +407,26 @@ int oracle_backward(int T, int d, int H, int K, int B, const double* x, const ui
   const double tau = isnan(th[0]) ? (double)(B - 1) / ((double)B * B) : th[0];
   const int adaptive = isnan(th[1]);
   double* dz = (double*)calloc((size_t)T * K1, sizeof(double));
-  if (!dz) return -2;
+  /* alpha and s of every token, kept for the weight gradients of pass 2 */
+  double* alpha_all = (double*)calloc((size_t)T, sizeof(double));
+  double* s_all = (double*)calloc((size_t)T * K, sizeof(double));
+  /* Layout copies only: value rows V_e[h, :] contiguous, and their
+   * gradients accumulated in the same layout before the transposition into
+   * dw_down. */
+  double* V = (double*)malloc(sizeof(double) * (size_t)K1 * H * d);
+  double* dV = (double*)malloc(sizeof(double) * (size_t)K1 * H * d);
+  if (!dz || !alpha_all || !s_all || !V || !dV) {
+    free(dz);
+    free(alpha_all);
+    free(s_all);
+    free(V);
+    free(dV);
+    return -2;
+  }
+  for (int e = 0; e < K1; ++e)
+    for (int i = 0; i < d; ++i)
+      for (int h = 0; h < H; ++h)
+        V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * d + i) * H + h];
 
   /* The pathway weight of expert e for token t (0: not used by t). */
 #define PATH_WEIGHT(e, alpha_t, s_t, t)                                                 \
@@ -446,6 +465,8 @@ int oracle_backward(int T, int d, int H, int K, int B, const double* x, const ui
     double z[ORACLE_MAX_K + 1], s[ORACLE_MAX_K], dw[ORACLE_MAX_K + 1];
     double alpha;
     ROUTER_SCORES(t, z, alpha, s);
+    alpha_all[t] = alpha;
+    for (int j = 0; j < K; ++j) s_all[(size_t)t * K + j] = s[j];
     for (int e = 0; e < K1; ++e) {
       dw[e] = 0.0;
       const double w = PATH_WEIGHT(e, alpha, s, t);
@@ -455,9 +476,10 @@ int oracle_backward(int T, int d, int H, int K, int B, const double* x, const ui
         if (!RUNS_BLOCK(e, blk, t)) continue;
         for (int h = blk * M; h < (blk + 1) * M; ++h) {
           const double* key = w_up + ((size_t)e * H + h) * d;
+          const double* val = V + ((size_t)e * H + h) * d;
           double a = 0.0, gv = 0.0;
           for (int i = 0; i < d; ++i) a += xt[i] * key[i];
-          for (int i = 0; i < d; ++i) gv += gt[i] * w_down[((size_t)e * d + i) * H + h];
+          for (int i = 0; i < d; ++i) gv += gt[i] * val[i];
           dw[e] += gelu(a) * gv;
           const double da = w * gv * gelu_grad(a);
           for (int i = 0; i < d; ++i) dxt[i] += da * key[i];
@@ -484,32 +506,36 @@ int oracle_backward(int T, int d, int H, int K, int B, const double* x, const ui
   for (int eh = 0; eh < K1 * H; ++eh) {
     const int e = eh / H, h = eh % H, blk = h / M;
     double* gk = dw_up + ((size_t)e * H + h) * d;
+    double* gvr = dV + ((size_t)e * H + h) * d;
     for (int i = 0; i < d; ++i) {
       gk[i] = 0.0;
-      dw_down[((size_t)e * d + i) * H + h] = 0.0;
+      gvr[i] = 0.0;
     }
     const double* key = w_up + ((size_t)e * H + h) * d;
+    const double* val = V + ((size_t)e * H + h) * d;
     for (int t = 0; t < T; ++t) {
       if (mask && !mask[t]) continue;
       if (!RUNS_BLOCK(e, blk, t)) continue;
       if (e > 0 && !((expert_mask[t] >> (e - 1)) & 1ull)) continue;
       const double* xt = x + (size_t)t * d;
       const double* gt = dy + (size_t)t * d;
-      double z[ORACLE_MAX_K + 1], s[ORACLE_MAX_K];
-      double alpha;
-      ROUTER_SCORES(t, z, alpha, s);
-      const double w = PATH_WEIGHT(e, alpha, s, t);
+      const double* s = s_all + (size_t)t * K;
+      const double w = PATH_WEIGHT(e, alpha_all[t], s, t);
       double a = 0.0, gv = 0.0;
       for (int i = 0; i < d; ++i) a += xt[i] * key[i];
-      for (int i = 0; i < d; ++i) gv += gt[i] * w_down[((size_t)e * d + i) * H + h];
+      for (int i = 0; i < d; ++i) gv += gt[i] * val[i];
       const double da = w * gv * gelu_grad(a);
       const double wg = w * gelu(a);
       for (int i = 0; i < d; ++i) {
         gk[i] += da * xt[i];
-        dw_down[((size_t)e * d + i) * H + h] += wg * gt[i];
+        gvr[i] += wg * gt[i];
       }
     }
   }
+  for (int e = 0; e < K1; ++e)
+    for (int i = 0; i < d; ++i)
+      for (int h = 0; h < H; ++h)
+        dw_down[((size_t)e * d + i) * H + h] = dV[((size_t)e * H + h) * d + i];
 
   /* Pass 3: dL/dW* = x^T dL/dz (Eq. 17), dL/dbias = sum_t dL/dz. */
 #pragma omp parallel for schedule(static)
@@ -533,6 +559,10 @@ int oracle_backward(int T, int d, int H, int K, int B, const double* x, const ui
 #undef RUNS_BLOCK
 #undef ROUTER_SCORES
   free(dz);
+  free(alpha_all);
+  free(s_all);
+  free(V);
+  free(dV);
   return 0;
 }
 

@@ -20,7 +20,7 @@ from typing import Optional
 import torch
 
 __all__ = ["Layer", "lib", "UnifMoeError", "ERR", "EXPORTS", "Options", "FEATURE_NORM_FIRST",
-           "FEATURE_HOST_IO", "FEATURES_ALL"]
+           "FEATURE_HOST_IO", "FEATURE_BACKWARD", "FEATURES_DEFAULT", "FEATURES_ALL"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "lib", "libunif_moe.so")
@@ -32,6 +32,7 @@ ERR = {0: "OK", -1: "ERR_ARG", -2: "ERR_SHAPE", -3: "ERR_CAPACITY", -4: "ERR_CUD
 EXPORTS = ["unif_moe_default_thresholds", "unif_moe_default_options", "unif_moe_create",
            "unif_moe_create_ex", "unif_moe_load_weights",
            "unif_moe_load_upcycled", "unif_moe_forward", "unif_moe_sublayer_forward",
+           "unif_moe_backward",
            "unif_moe_forward_host", "unif_moe_get_routing",
            "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_pass_tokens",
            "unif_moe_kernels_per_forward",
@@ -55,7 +56,8 @@ class Options(C.Structure):
     _fields_ = [("features", C.c_uint), ("gemm_kernels", C.c_int)]
 
 
-FEATURE_NORM_FIRST, FEATURE_HOST_IO, FEATURES_ALL = 1, 2, 3
+FEATURE_NORM_FIRST, FEATURE_HOST_IO, FEATURE_BACKWARD = 1, 2, 4
+FEATURES_DEFAULT, FEATURES_ALL = 3, 7
 GEMM_KERNELS = {"auto": 0, "streaming": 1}
 
 
@@ -81,6 +83,7 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_forward.argtypes = [P, P, P, I, P, P, P, P]
         L.unif_moe_load_upcycled.argtypes = [P, P, P, P, P, P]
         L.unif_moe_sublayer_forward.argtypes = [P, P, P, I, P, P, P, P, P, C.c_float, I, P]
+        L.unif_moe_backward.argtypes = [P, P, P, I, P, P, P, P, P, P, C.c_float, P, P]
         L.unif_moe_forward_host.argtypes = [P, P, P, I, P, P, P, P]
         L.unif_moe_get_routing.argtypes = [P, P, P, P, P, P, P]
         L.unif_moe_get_groups.argtypes = [P, P, P, P, P, C.POINTER(C.c_int64), P]
@@ -129,7 +132,7 @@ class Layer:
     def __init__(self, d_model: int, d_ff: int, n_experts: int, n_blocks: int,
                  dtype: str = "bf16", max_tokens: int = 65536, tau: float = math.nan,
                  alpha_fixed: float = math.nan, beta_fixed: float = math.nan,
-                 topk_fixed: int = 0, prefix_blocks: int = 0, features: int = FEATURES_ALL,
+                 topk_fixed: int = 0, prefix_blocks: int = 0, features: int = FEATURES_DEFAULT,
                  gemm_kernels: str = "auto"):
         self.d, self.H, self.K, self.B = d_model, d_ff, n_experts, n_blocks
         self.dtype = dtype
@@ -206,6 +209,26 @@ class Layer:
                                       _stream(stream)))
         self.last_T = T
         return out
+
+    def backward(self, x: torch.Tensor, dy: torch.Tensor, mask: Optional[torch.Tensor] = None,
+                 lambda_div: float = 0.0, want_bias: bool = False, stream=None) -> dict:
+        """Gradients of the last forward (which must have run on x) given
+        dL/dy (Sec. III-E): dict of fp32 CUDA tensors dx, dw_up, dw_down,
+        dw_router (plus lambda_div dL_div/dW*), dbias (want_bias), l_div."""
+        T = x.shape[0]
+        dev = x.device
+        f32 = dict(dtype=torch.float32, device=dev)
+        g = dict(dx=torch.empty(T, self.d, **f32),
+                 dw_up=torch.empty(self.K + 1, self.H, self.d, **f32),
+                 dw_down=torch.empty(self.K + 1, self.d, self.H, **f32),
+                 dw_router=torch.empty(self.d, self.K + 1, **f32),
+                 dbias=torch.empty(self.K + 1, **f32) if want_bias else None,
+                 l_div=torch.empty(1, **f32))
+        _check(lib().unif_moe_backward(self._h, _ptr(x), _ptr(dy), T, _ptr(mask), _ptr(g["dx"]),
+                                       _ptr(g["dw_up"]), _ptr(g["dw_down"]),
+                                       _ptr(g["dw_router"]), _ptr(g["dbias"]),
+                                       float(lambda_div), _ptr(g["l_div"]), _stream(stream)))
+        return g
 
     def forward_host(self, x_host: torch.Tensor, out_host: torch.Tensor,
                      mask_host: Optional[torch.Tensor] = None,

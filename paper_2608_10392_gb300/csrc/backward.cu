@@ -1,0 +1,787 @@
+// Backward pass of the UniF-MoE layer (training, Sec. III-E) for bf16 layers,
+// on the tensor cores, over the group table of the forward that preceded it.
+//
+// The discrete decisions (b, I_shr, k and the selected experts) are
+// piecewise constant in the parameters, so gradients flow through the
+// pathway weights alpha (Eq. 18) and s_j (Eq. 24) and through the experts
+// (Eq. 16). For a group row (token t, expert e, block b) with weight w and
+// pre-activations a = x K_e[:, H_b]:
+//   g      = dy V_e[H_b, :]^T                 (the output gradient per channel)
+//   dL/da  = w g GeLU'(a)                     -> DA row
+//   w GeLU(a)                                 -> HW row
+//   dL/dw += sum_h GeLU(a_h) g_h              -> dwt[t][e] (alpha for e = 0, s_j for e = 1+j)
+// then, summed over rows:
+//   dL/dx[t]          += DA row K_e[H_b, :]   (the streaming down kernel on K^T)
+//   dL/dK_e[H_b, :]    = DA^T X[rows]         (weight-gradient kernel)
+//   dL/dV_e[:, H_b]    = DY[rows]^T HW        (same kernel)
+// and per token dL/dz from dL/dalpha and dL/ds (Eqs. 18, 24), dL/dW* = X^T dL/dz,
+// dL/dbias = sum dL/dz, dL/dx += dL/dz W*^T; the Gram regulariser (Eq.
+// diversity-loss) adds lambda_div dL_div/dW*.
+//
+// Kernels (in stream order): tile list from the forward's group sizes,
+// bwd_hidden_kernel (two tcgen05 accumulators: x K and dy V^T over the same
+// gathered rows), the down kernel for dL/dx, bwd_wgrad_kernel (tcgen05 with
+// MN-major operands: the token rows are the reduction dimension), the
+// router-gradient kernels and the Gram kernel. Every wait on an mbarrier is
+// bounded; a wait that runs out records kStatusTimeout and the CTA unwinds.
+#include <stdio.h>
+
+#include "decide.cuh"
+#include "internal.cuh"
+#include "tc_common.cuh"
+
+namespace unif {
+namespace tc {
+namespace bwd {
+
+// GeLU (exact erf form, Sec. II-A) and its derivative Phi(a) + a phi(a).
+__device__ __forceinline__ float gelu_f(float a) {
+  return 0.5f * a * (1.0f + erff(a * 0.70710678118654752f));
+}
+__device__ __forceinline__ float gelu_grad_f(float a) {
+  return 0.5f * (1.0f + erff(a * 0.70710678118654752f)) +
+         a * 0.39894228040143268f * expf(-0.5f * a * a);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Instruction descriptor of kind::f16 (bf16 in, fp32 accumulate) with both
+// operands MN-major (transpose bits 15 and 16).
+__device__ __forceinline__ uint32_t idesc_bf16_mn(int m, int n) {
+  return idesc_bf16(m, n) | (1u << 15) | (1u << 16);
+}
+
+// Shared-memory descriptor of an MN-major operand with the 128-byte swizzle:
+// each 128-byte row holds 64 consecutive MN elements of one K index, 8-row
+// (K) groups are 1024 bytes apart (stride-dimension offset), and blocks of
+// 64 MN elements are `lbo` bytes apart (leading-dimension offset).
+__device__ __forceinline__ uint64_t sw128_mn_desc(uint32_t saddr, uint32_t lbo) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+constexpr int kThreads = 416;     // 13 warps
+constexpr int kMmaWarp = 4;
+constexpr int kFirstEpiWarp = 5;  // warps 5-12
+constexpr int kEpiWarps = 8;
+constexpr int kStages = 2;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kAcc2 = 256;   // TMEM column of the second accumulator
+
+// ---------------------------------------------------------------------------
+// bwd_hidden_kernel: per (tile, N sub-tile) item, over the forward's tile
+// list, acc_a = X[rows] K_e[cols]^T and acc_g = DY[rows] V_e^T[cols]^T (both
+// reductions over d), then the epilogue of the header comment.
+// Roles: warps 0-3 fill the 2-deep stage ring (warp 2s gathers the x rows of
+// stage s and brings both weight tiles by TMA, warp 2s+1 gathers the dy
+// rows); warp 4 allocates TMEM and issues the MMAs; warps 5-12 run the
+// epilogue (warp w reads TMEM lane quarter w % 4, one half of the columns).
+// ---------------------------------------------------------------------------
+struct HiddenParams {
+  const int32_t* n_tiles;
+  const int32_t* tile_group;
+  const int32_t* tile_row0;
+  const int32_t* tile_rows;
+  const int32_t* row_tok;
+  const float* row_w;
+  const __nv_bfloat16* x;
+  const __nv_bfloat16* dy;
+  __nv_bfloat16* da;   // [rows][M]
+  __nv_bfloat16* hw;   // [rows][M]
+  float* dwt;          // [T][K+1]
+  int n_sub, bn, num_kb, B, M, H, d, K1;
+  int* status;
+  long long wait_limit;
+};
+
+__host__ __device__ constexpr uint32_t hidden_stage_bytes(int bn) {
+  return 2u * kStageA + 2u * (uint32_t)bn * kBK * 2u;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+bwd_hidden_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_constant__ CUtensorMap tm_wv,
+                  HiddenParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const uint32_t stage_bytes = hidden_stage_bytes(p.bn);
+  const uint32_t wtile = (uint32_t)p.bn * kBK * 2u;
+  const uint32_t s0 = smem_u32(smem);
+  // stage s: [x rows 16 KB][dy rows 16 KB][K tile][V tile]
+  auto sx = [&](int s) { return s0 + s * stage_bytes; };
+  auto sdy = [&](int s) { return s0 + s * stage_bytes + kStageA; };
+  auto swk = [&](int s) { return s0 + s * stage_bytes + 2 * kStageA; };
+  auto swv = [&](int s) { return s0 + s * stage_bytes + 2 * kStageA + wtile; };
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * stage_bytes);
+  const uint32_t bar0 = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
+  const uint32_t accf = bar0 + 8u * (2 * kStages);
+  const uint32_t acce = bar0 + 8u * (2 * kStages + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full_bar(s), 2);  // the x warp and the dy warp of the stage
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(accf, 1);
+    mbar_init(acce, kEpiWarps);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int n_items = p.n_tiles[0] * p.n_sub;
+
+  if (warp < 4) {
+    // ---- producers: warp 2s + kind owns stage s (kind 0: x rows and the
+    // weight tiles, kind 1: dy rows) ----
+    const int my_stage = warp >> 1, kind = warp & 1;
+    const __nv_bfloat16* src = kind == 0 ? p.x : p.dy;
+    const int j = lane & 7, rsub = lane >> 3;
+    bool ok = true;
+    int seq = 0;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      const int tile = item / p.n_sub, ns = item % p.n_sub;
+      const int g = p.tile_group[tile];
+      const int e = g / p.B, blk = g % p.B;
+      const int brow = e * p.H + blk * p.M + ns * p.bn;
+      const int r0 = p.tile_row0[tile], nrow = p.tile_rows[tile];
+      int tk[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        // padding rows gather token 0; their results are never kept
+        const int t = 32 * i + lane < nrow ? p.row_tok[r0 + 32 * i + lane] : 0;
+        tk[i] = t < 0 ? 0 : t;
+      }
+      for (int kb = 0; kb < p.num_kb; ++kb, ++seq) {
+        const int stage = seq % kStages;
+        if (stage != my_stage) continue;
+        const uint32_t phase = (uint32_t)(seq / kStages) & 1u;
+        ok = wait_warp(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
+        if (!ok) break;
+        if (kind == 0 && lane == 0) {
+          mbar_expect_tx_only(full_bar(stage), 2u * wtile);
+          tma_load_2d(swk(stage), &tm_wk, full_bar(stage), kb * kBK, brow);
+          tma_load_2d(swv(stage), &tm_wv, full_bar(stage), kb * kBK, brow);
+        }
+        const uint32_t dst = kind == 0 ? sx(stage) : sdy(stage);
+        const __nv_bfloat16* sj = src + j * 8 + kb * kBK;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int r = 4 * i + rsub;
+          const int t = __shfl_sync(0xffffffffu, tk[i >> 3], r & 31);
+          cp_async16(dst + r * 128u + ((j ^ (r & 7)) << 4), sj + (size_t)t * p.d);
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(full_bar(stage));
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---- MMA issuer ----
+    const uint32_t idesc = idesc_bf16(kBM, p.bn);
+    int seq = 0;
+    uint32_t acc_phase = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      ok = wait_warp(acce, acc_phase ^ 1u, abort_flag, p.status, p.wait_limit);
+      if (!ok) break;
+      tc_fence_after();
+      for (int kb = 0; kb < p.num_kb; ++kb, ++seq) {
+        const int stage = seq % kStages;
+        const uint32_t phase = (uint32_t)(seq / kStages) & 1u;
+        ok = wait_warp(full_bar(stage), phase, abort_flag, p.status, p.wait_limit);
+        if (!ok) break;
+        tc_fence_after();
+        if (elect_one()) {
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+            const uint32_t acc = (kb | k) != 0 ? 1u : 0u;
+            umma_bf16(tmem_base, sw128_desc(sx(stage) + k * 32), sw128_desc(swk(stage) + k * 32),
+                      idesc, acc);
+            umma_bf16(tmem_base + kAcc2, sw128_desc(sdy(stage) + k * 32),
+                      sw128_desc(swv(stage) + k * 32), idesc, acc);
+          }
+          umma_commit(empty_bar(stage));
+        }
+        __syncwarp();
+      }
+      if (!ok) break;
+      if (elect_one()) umma_commit(accf);
+      __syncwarp();
+      acc_phase ^= 1u;
+    }
+  } else if (warp >= kFirstEpiWarp) {
+    // ---- epilogue ----
+    const int q = warp & 3;
+    const int half = (warp - kFirstEpiWarp) >> 2;
+    const int cols = p.bn / 2;
+    const int c_begin = half * cols;
+    uint32_t acc_phase = 0;
+    for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
+      const int tile = item / p.n_sub, ns = item % p.n_sub;
+      const int g = p.tile_group[tile];
+      const int e = g / p.B;
+      const int r = q * 32 + lane;
+      const bool real = r < p.tile_rows[tile];
+      const int tok = real ? p.row_tok[p.tile_row0[tile] + r] : -1;
+      const float w = real ? p.row_w[p.tile_row0[tile] + r] : 0.f;
+      if (!wait_warp(accf, acc_phase, abort_flag, p.status, p.wait_limit)) break;
+      tc_fence_after();
+      const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16);
+      const size_t orow = ((size_t)tile * kBM + r) * p.M + ns * p.bn + c_begin;
+      float dot = 0.f;
+      for (int c = 0; c < cols; c += 16) {
+        float a[16], gv[16];
+        tmem_ld16(t_row + c_begin + c, a);
+        tmem_ld16(t_row + kAcc2 + c_begin + c, gv);
+        uint32_t od[8], oh[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float d0 = 0.f, d1 = 0.f, h0 = 0.f, h1 = 0.f;
+          if (tok >= 0) {
+            const float g0 = gelu_f(a[2 * i]), g1 = gelu_f(a[2 * i + 1]);
+            dot = fmaf(g0, gv[2 * i], dot);
+            dot = fmaf(g1, gv[2 * i + 1], dot);
+            d0 = w * gv[2 * i] * gelu_grad_f(a[2 * i]);
+            d1 = w * gv[2 * i + 1] * gelu_grad_f(a[2 * i + 1]);
+            h0 = w * g0;
+            h1 = w * g1;
+          }
+          od[i] = pack_bf16(d0, d1);
+          oh[i] = pack_bf16(h0, h1);
+        }
+        // padding rows are written as zeros: the weight-gradient kernel sums
+        // over whole tiles
+        uint4* pd = reinterpret_cast<uint4*>(p.da + orow + c);
+        uint4* ph = reinterpret_cast<uint4*>(p.hw + orow + c);
+        pd[0] = make_uint4(od[0], od[1], od[2], od[3]);
+        pd[1] = make_uint4(od[4], od[5], od[6], od[7]);
+        ph[0] = make_uint4(oh[0], oh[1], oh[2], oh[3]);
+        ph[1] = make_uint4(oh[4], oh[5], oh[6], oh[7]);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acce);
+      if (tok >= 0) atomicAdd(p.dwt + (size_t)tok * p.K1 + e, dot);
+      acc_phase ^= 1u;
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// bwd_wgrad_kernel: per item (group g, 128 features c of d, N chunk nc of the
+// block's M channels) two accumulators over all rows of the group, 64 rows
+// per stage:
+//   acc1[i][h] = sum_r X[tok_r][c*128 + i] DA[r][nc*N + h]   -> dK_e (transposed)
+//   acc2[i][h] = sum_r DY[tok_r][c*128 + i] HW[r][nc*N + h]  -> dV_e
+// The token rows are the reduction dimension, so both operands are MN-major:
+// the gathered rows (x, dy) and the TMA tiles (DA, HW) keep the 128-byte
+// swizzled row layout, read with MN-major descriptors. Each item owns its
+// output exactly (no atomics); groups without rows give zeros.
+// Roles: warps 0-3 fill the ring (warp 2s: x rows of stage s and the DA/HW
+// tiles by TMA; warp 2s+1: dy rows), warp 4 MMAs, warps 5-12 epilogue.
+// ---------------------------------------------------------------------------
+struct WgradParams {
+  const int32_t* counts;   // [G] group sizes (the forward's)
+  const int32_t* row_tok;  // per-group regions of `region` rows
+  const __nv_bfloat16* x;
+  const __nv_bfloat16* dy;
+  float* dw_up;    // [K+1][H][d]
+  float* dw_down;  // [K+1][d][H]
+  int G, region, B, M, H, d, N, n_nc, n_c;
+  int* status;
+  long long wait_limit;
+};
+
+constexpr uint32_t kRows = 64;                 // group rows per stage
+constexpr uint32_t kPBytes = 2u * kRows * 128u;  // 128 features x 64 rows (two 64-column blocks)
+
+__host__ __device__ constexpr uint32_t wgrad_stage_bytes(int N) {
+  return 2u * kPBytes + 2u * (uint32_t)(N / 64) * kRows * 128u;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constant__ CUtensorMap tm_hw,
+                 WgradParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const uint32_t stage_bytes = wgrad_stage_bytes(p.N);
+  const uint32_t qbytes = (uint32_t)(p.N / 64) * kRows * 128u;
+  const uint32_t s0 = smem_u32(smem);
+  // stage s: [x rows][dy rows][DA tile][HW tile]
+  auto spx = [&](int s) { return s0 + s * stage_bytes; };
+  auto spy = [&](int s) { return s0 + s * stage_bytes + kPBytes; };
+  auto sqa = [&](int s) { return s0 + s * stage_bytes + 2 * kPBytes; };
+  auto sqh = [&](int s) { return s0 + s * stage_bytes + 2 * kPBytes + qbytes; };
+  uint8_t* gen_base = smem;  // generic pointer for zero-filling padding rows
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * stage_bytes);
+  const uint32_t bar0 = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
+  const uint32_t accf = bar0 + 8u * (2 * kStages);
+  const uint32_t acce = bar0 + 8u * (2 * kStages + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int32_t* first_s = reinterpret_cast<int32_t*>(tmem_slot + 4);  // [G + 1] first tiles
+  int32_t* cnt_s = first_s + p.G + 1;                             // [G] sizes
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full_bar(s), 2);
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(accf, 1);
+    mbar_init(acce, kEpiWarps);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == kThreads / 32 - 1) tile_table(p.counts, p.G, p.region, lane, first_s, cnt_s);
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int n_items = p.G * p.n_c * p.n_nc;
+  // item -> (group, feature chunk, N chunk); tiles of the group: first_s
+  auto decode = [&](int item, int& g, int& c, int& nc) {
+    nc = item % p.n_nc;
+    c = (item / p.n_nc) % p.n_c;
+    g = item / (p.n_nc * p.n_c);
+  };
+
+  if (warp < 4) {
+    const int my_stage = warp >> 1, kind = warp & 1;
+    const __nv_bfloat16* src = kind == 0 ? p.x : p.dy;
+    const int j = lane & 7, rsub = lane >> 3;
+    bool ok = true;
+    int seq = 0;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      int g, c, nc;
+      decode(item, g, c, nc);
+      const int t_first = first_s[g], nt = first_s[g + 1] - t_first;
+      const int size = cnt_s[g];
+      for (int kt = 0; kt < nt * 2 && ok; ++kt, ++seq) {  // 64-row halves of the group's tiles
+        const int stage = seq % kStages;
+        if (stage != my_stage) continue;
+        const uint32_t phase = (uint32_t)(seq / kStages) & 1u;
+        ok = wait_warp(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
+        if (!ok) break;
+        const int row_in_group = kt * (int)kRows;  // first row of this half in the group
+        const int crow = (t_first + kt / 2) * kBM + (kt & 1) * (int)kRows;  // compact DA/HW row
+        if (kind == 0 && lane == 0) {
+          mbar_expect_tx_only(full_bar(stage), 2u * qbytes);
+          for (int b = 0; b < p.N / 64; ++b) {
+            tma_load_2d(sqa(stage) + b * kRows * 128u, &tm_da, full_bar(stage), nc * p.N + b * 64,
+                        crow);
+            tma_load_2d(sqh(stage) + b * kRows * 128u, &tm_hw, full_bar(stage), nc * p.N + b * 64,
+                        crow);
+          }
+        }
+        // this half's 64 row tokens: lane l holds rows l and l + 32 (-1: padding)
+        int tk[2];
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const int rg = row_in_group + 32 * i + lane;
+          tk[i] = rg < size ? p.row_tok[(size_t)g * p.region + rg] : -1;
+        }
+        const uint32_t dst = kind == 0 ? spx(stage) : spy(stage);
+        const __nv_bfloat16* sj = src + (size_t)c * 128 + j * 8;
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int r = 4 * i + rsub;
+            const int t = __shfl_sync(0xffffffffu, tk[r >> 5], r & 31);
+            const uint32_t off = b * kRows * 128u + r * 128u + ((j ^ (r & 7)) << 4);
+            if (t >= 0)
+              cp_async16(dst + off, sj + (size_t)t * p.d + b * 64);
+            else  // padding rows contribute zeros to the row sums
+              *reinterpret_cast<uint4*>(gen_base + (dst - s0) + off) = make_uint4(0u, 0u, 0u, 0u);
+          }
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(full_bar(stage));
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    const uint32_t idesc = idesc_bf16_mn(kBM, p.N);
+    const uint32_t lbo = kRows * 128u;  // 64-element MN blocks of 64 rows
+    int seq = 0;
+    uint32_t acc_phase = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      int g, c, nc;
+      decode(item, g, c, nc);
+      const int nt = first_s[g + 1] - first_s[g];
+      if (nt == 0) continue;  // no rows: the epilogue writes zeros
+      ok = wait_warp(acce, acc_phase ^ 1u, abort_flag, p.status, p.wait_limit);
+      if (!ok) break;
+      tc_fence_after();
+      for (int kt = 0; kt < nt * 2; ++kt, ++seq) {
+        const int stage = seq % kStages;
+        const uint32_t phase = (uint32_t)(seq / kStages) & 1u;
+        ok = wait_warp(full_bar(stage), phase, abort_flag, p.status, p.wait_limit);
+        if (!ok) break;
+        tc_fence_after();
+        if (elect_one()) {
+#pragma unroll
+          for (int k = 0; k < (int)kRows / 16; ++k) {  // 16 rows (two 8-row groups) per MMA
+            const uint32_t acc = (kt | k) != 0 ? 1u : 0u;
+            umma_bf16(tmem_base, sw128_mn_desc(spx(stage) + k * 2048u, lbo),
+                      sw128_mn_desc(sqa(stage) + k * 2048u, lbo), idesc, acc);
+            umma_bf16(tmem_base + kAcc2, sw128_mn_desc(spy(stage) + k * 2048u, lbo),
+                      sw128_mn_desc(sqh(stage) + k * 2048u, lbo), idesc, acc);
+          }
+          umma_commit(empty_bar(stage));
+        }
+        __syncwarp();
+      }
+      if (!ok) break;
+      if (elect_one()) umma_commit(accf);
+      __syncwarp();
+      acc_phase ^= 1u;
+    }
+  } else if (warp >= kFirstEpiWarp) {
+    const int q = warp & 3;
+    const int half = (warp - kFirstEpiWarp) >> 2;
+    const int cols = p.N / 2;
+    uint32_t acc_phase = 0;
+    for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
+      int g, c, nc;
+      decode(item, g, c, nc);
+      const int e = g / p.B, blk = g % p.B;
+      const int nt = first_s[g + 1] - first_s[g];
+      const int i = c * 128 + q * 32 + lane;  // this thread's feature
+      const int h0 = blk * p.M + nc * p.N + half * cols;  // first channel of its columns
+      float* up_col = p.dw_up + ((size_t)e * p.H + h0) * p.d + i;   // dK_e[h][i], stride d per h
+      float* dn_row = p.dw_down + ((size_t)e * p.d + i) * p.H + h0;  // dV_e[i][h], contiguous
+      if (nt == 0) {
+        for (int cc = 0; cc < cols; ++cc) {
+          up_col[(size_t)cc * p.d] = 0.f;
+          dn_row[cc] = 0.f;
+        }
+        continue;
+      }
+      if (!wait_warp(accf, acc_phase, abort_flag, p.status, p.wait_limit)) break;
+      tc_fence_after();
+      const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + half * cols;
+      for (int cc = 0; cc < cols; cc += 32) {
+        float v[32];
+        tmem_ld32(t_row + cc, v);
+#pragma unroll
+        for (int jj = 0; jj < 32; ++jj) up_col[(size_t)(cc + jj) * p.d] = v[jj];
+        tmem_ld32(t_row + kAcc2 + cc, v);
+#pragma unroll
+        for (int jj = 0; jj < 32; jj += 4)
+          *reinterpret_cast<float4*>(dn_row + cc + jj) = make_float4(v[jj], v[jj + 1], v[jj + 2], v[jj + 3]);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acce);
+      acc_phase ^= 1u;
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Router gradients (Eqs. 17, 18, 24)
+// ---------------------------------------------------------------------------
+// One warp per token: dL/dz_0 = dL/dalpha (1 - 2 tau) sigma(z_0)(1 - sigma(z_0))
+// (adaptive alpha; sigma(z_0) = (alpha - tau) / (1 - 2 tau) from the stored
+// alpha), dL/dz_{1+j} = s_j (dL/ds_j - sum_l s_l dL/ds_l); then dx[t] +=
+// dL/dz W*^T (W* = the router matrix's first K+1 columns, fp32 [d][Cp]).
+__global__ void router_grad_kernel(int T, int K, int Cp, int d, float tau, int adaptive,
+                                   const uint8_t* __restrict__ mask,
+                                   const float* __restrict__ alpha, const float* __restrict__ s,
+                                   const float* __restrict__ dwt, const float* __restrict__ wr,
+                                   float* __restrict__ dz, float* __restrict__ dx) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (warp >= T) return;
+  const int t = warp;
+  const int K1 = K + 1;
+  float* dzt = dz + (size_t)t * K1;
+  if (mask && !mask[t]) {
+    for (int c = lane; c < K1; c += 32) dzt[c] = 0.f;
+    return;
+  }
+  const float* st = s + (size_t)t * K;
+  const float* gt = dwt + (size_t)t * K1;
+  float part = 0.f;
+  for (int j = lane; j < K; j += 32) part += st[j] * gt[1 + j];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+  for (int j = lane; j < K; j += 32) dzt[1 + j] = st[j] * (gt[1 + j] - part);
+  if (lane == 0) {
+    float dz0 = 0.f;
+    if (adaptive && tau < 0.5f) {
+      const float sg = (alpha[t] - tau) / (1.0f - 2.0f * tau);
+      dz0 = gt[0] * (1.0f - 2.0f * tau) * sg * (1.0f - sg);
+    }
+    dzt[0] = dz0;
+  }
+  __syncwarp();
+  float* dxt = dx + (size_t)t * d;
+  for (int i = lane; i < d; i += 32) {
+    float acc = 0.f;
+    for (int c = 0; c < K1; ++c) acc = fmaf(dzt[c], wr[(size_t)i * Cp + c], acc);
+    dxt[i] += acc;
+  }
+}
+
+// dL/dW*[i][c] = sum_t x[t][i] dL/dz[t][c] and dL/dbias[c] = sum_t dL/dz[t][c]:
+// block (i-block of 256 features, 128-token chunk); partial sums added
+// atomically (the outputs start at zero).
+constexpr int kRgTokens = 128;
+__global__ void __launch_bounds__(256)
+router_wgrad_kernel(int T, int K1, int d, const uint8_t* __restrict__ mask,
+                    const __nv_bfloat16* __restrict__ x, const float* __restrict__ dz,
+                    float* __restrict__ dw_router, float* __restrict__ dbias) {
+  extern __shared__ float dz_s[];  // [kRgTokens][K1]
+  const int t0 = blockIdx.y * kRgTokens;
+  const int nt = min(kRgTokens, T - t0);
+  for (int k = threadIdx.x; k < nt * K1; k += blockDim.x) {
+    const int t = t0 + k / K1;
+    dz_s[k] = (mask && !mask[t]) ? 0.f : dz[(size_t)t0 * K1 + k];
+  }
+  __syncthreads();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < d) {
+    for (int c0 = 0; c0 < K1; c0 += 16) {
+      float acc[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) acc[u] = 0.f;
+      for (int tt = 0; tt < nt; ++tt) {
+        const int t = t0 + tt;
+        const float xv = (mask && !mask[t]) ? 0.f : __bfloat162float(x[(size_t)t * d + i]);
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+          if (c0 + u < K1) acc[u] = fmaf(xv, dz_s[tt * K1 + c0 + u], acc[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+        if (c0 + u < K1) atomicAdd(dw_router + (size_t)i * K1 + c0 + u, acc[u]);
+    }
+  }
+  if (dbias && blockIdx.x == 0) {
+    for (int c = threadIdx.x; c < K1; c += blockDim.x) {
+      float acc = 0.f;
+      for (int tt = 0; tt < nt; ++tt) acc += dz_s[tt * K1 + c];
+      atomicAdd(dbias + c, acc);
+    }
+  }
+}
+
+// Gram regulariser (Eq. diversity-loss): A = W*^T W* - I over the K+1 router
+// columns, L_div = ||A||_F; dW* += lambda 2 W* A / L_div (nothing where
+// L_div = 0). One block; A in shared memory ([K1][K1] fp32).
+__global__ void __launch_bounds__(256)
+diversity_kernel(int K1, int d, int Cp, const float* __restrict__ wr, float lambda,
+                 float* __restrict__ dw_router, float* __restrict__ l_out) {
+  extern __shared__ float A_s[];  // [K1][K1], then one reduction slot per warp
+  float* red = A_s + K1 * K1;
+  float ss = 0.f;
+  for (int k = threadIdx.x; k < K1 * K1; k += blockDim.x) {
+    const int a = k / K1, b = k % K1;
+    float g = 0.f;
+    for (int i = 0; i < d; ++i) g = fmaf(wr[(size_t)i * Cp + a], wr[(size_t)i * Cp + b], g);
+    g -= (a == b) ? 1.f : 0.f;
+    A_s[k] = g;
+    ss += g * g;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float tot = 0.f;
+  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
+  const float L = sqrtf(tot);
+  if (threadIdx.x == 0 && l_out) *l_out = L;
+  if (L > 0.f && lambda != 0.f && dw_router) {
+    const float scale = 2.f * lambda / L;
+    for (int k = threadIdx.x; k < d * K1; k += blockDim.x) {
+      const int i = k / K1, b = k % K1;
+      float g = 0.f;
+      for (int a = 0; a < K1; ++a) g = fmaf(wr[(size_t)i * Cp + a], A_s[a * K1 + b], g);
+      dw_router[k] += scale * g;
+    }
+  }
+}
+
+// out[e][c][r] = in[e][r][c] for bf16 [E][R][C] (32 x 32 tiles through shared
+// memory).
+__global__ void transpose_bf16_kernel(const __nv_bfloat16* __restrict__ in,
+                                      __nv_bfloat16* __restrict__ out, int R, int C) {
+  __shared__ __nv_bfloat16 tile[32][33];
+  const size_t base = (size_t)blockIdx.z * R * C;
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  for (int k = threadIdx.y; k < 32; k += blockDim.y) {
+    const int r = r0 + k, c = c0 + threadIdx.x;
+    if (r < R && c < C) tile[k][threadIdx.x] = in[base + (size_t)r * C + c];
+  }
+  __syncthreads();
+  for (int k = threadIdx.y; k < 32; k += blockDim.y) {
+    const int c = c0 + k, r = r0 + threadIdx.x;
+    if (r < R && c < C) out[base + (size_t)c * R + r] = tile[threadIdx.x][k];
+  }
+}
+
+}  // namespace bwd
+}  // namespace tc
+
+// ---- host side ----
+
+int backward_setup(unif_moe_layer* L) {
+  using namespace tc::bwd;
+  const uint64_t E = (uint64_t)L->K + 1;
+  Workspace& w = L->ws;
+  if (!encode_bf16_map(&L->tm_wdownT, w.w_downT, L->d, E * L->H, tc::kBK, L->up_bn, 128) ||
+      !encode_bf16_map(&L->tm_wupT, w.w_upT, L->H, E * L->d, tc::kBK, L->down_bn, 128) ||
+      !encode_bf16_map(&L->tm_da, w.da, L->M, (uint64_t)L->max_rows, tc::kBK, tc::kBM, 128) ||
+      !encode_bf16_map(&L->tm_da64, w.da, L->M, (uint64_t)L->max_rows, tc::kBK, kRows, 128) ||
+      !encode_bf16_map(&L->tm_hw64, w.hw, L->M, (uint64_t)L->max_rows, tc::kBK, kRows, 128)) {
+    set_error("cuTensorMapEncodeTiled failed for the backward maps");
+    return UNIF_MOE_ERR_CUDA;
+  }
+  L->bwd_hidden_smem = 1024 + kStages * hidden_stage_bytes(L->up_bn) + 256;
+  L->bwd_wgrad_smem =
+      1024 + kStages * wgrad_stage_bytes(L->up_bn) + 64 + 4 * (2 * (uint32_t)L->G + 1) + 16;
+  if (L->bwd_hidden_smem > 232448 || L->bwd_wgrad_smem > 232448) {
+    set_error("backward: shared memory for block width %d and %d groups exceeds 227 KB", L->M,
+              L->G);
+    return UNIF_MOE_ERR_SHAPE;
+  }
+  if (cudaFuncSetAttribute(bwd_hidden_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)L->bwd_hidden_smem) != cudaSuccess ||
+      cudaFuncSetAttribute(bwd_wgrad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)L->bwd_wgrad_smem) != cudaSuccess) {
+    set_error("cudaFuncSetAttribute failed for the backward kernels");
+    return UNIF_MOE_ERR_CUDA;
+  }
+  return UNIF_MOE_OK;
+}
+
+cudaError_t launch_transpose_weights(unif_moe_layer* L, cudaStream_t s) {
+  using namespace tc::bwd;
+  const int E = L->K + 1;
+  dim3 blk(32, 8);
+  // w_up [E][H][d] -> w_upT [E][d][H]; w_down [E][d][H] -> w_downT [E][H][d]
+  transpose_bf16_kernel<<<dim3((L->d + 31) / 32, (L->H + 31) / 32, E), blk, 0, s>>>(
+      static_cast<const __nv_bfloat16*>(L->w_up), static_cast<__nv_bfloat16*>(L->ws.w_upT), L->H,
+      L->d);
+  transpose_bf16_kernel<<<dim3((L->H + 31) / 32, (L->d + 31) / 32, E), blk, 0, s>>>(
+      static_cast<const __nv_bfloat16*>(L->w_down), static_cast<__nv_bfloat16*>(L->ws.w_downT),
+      L->d, L->H);
+  return cudaGetLastError();
+}
+
+int backward_run(unif_moe_layer* L, const void* x, const void* dy, int T, const uint8_t* mask,
+                 float* dx, float* dw_up, float* dw_down, float* dw_router, float* dbias,
+                 float lambda_div, float* l_div, cudaStream_t s) {
+  using namespace tc::bwd;
+  Workspace& w = L->ws;
+  const int K1 = L->K + 1;
+#define CKB(call)                                                               \
+  do {                                                                          \
+    cudaError_t e_ = (call);                                                    \
+    if (e_ != cudaSuccess) {                                                    \
+      set_error("%s failed: %s", #call, cudaGetErrorString(e_));                \
+      return UNIF_MOE_ERR_CUDA;                                                 \
+    }                                                                           \
+  } while (0)
+  CKB(cudaMemsetAsync(dx, 0, sizeof(float) * (size_t)T * L->d, s));
+  CKB(cudaMemsetAsync(w.dwt, 0, sizeof(float) * (size_t)T * K1, s));
+  CKB(cudaMemsetAsync(dw_router, 0, sizeof(float) * (size_t)L->d * K1, s));
+  if (dbias) CKB(cudaMemsetAsync(dbias, 0, sizeof(float) * K1, s));
+  // tile list of the forward's groups (sizes in grp_cnt, rows in the regions)
+  CKB(launch_tile_list_from(L, w.grp_cnt, s));
+  // hidden gradients
+  {
+    HiddenParams p;
+    p.n_tiles = w.n_tiles; p.tile_group = w.tile_group; p.tile_row0 = w.tile_row0;
+    p.tile_rows = w.tile_rows; p.row_tok = w.row_tok; p.row_w = w.row_w;
+    p.x = static_cast<const __nv_bfloat16*>(x);
+    p.dy = static_cast<const __nv_bfloat16*>(dy);
+    p.da = static_cast<__nv_bfloat16*>(w.da);
+    p.hw = static_cast<__nv_bfloat16*>(w.hw);
+    p.dwt = w.dwt;
+    p.n_sub = L->up_nsub; p.bn = L->up_bn; p.num_kb = L->d / tc::kBK;
+    p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d; p.K1 = K1;
+    p.status = w.status;
+    p.wait_limit = gemm_wait_limit();
+    bwd_hidden_kernel<<<L->n_sm, kThreads, L->bwd_hidden_smem, s>>>(L->tm_wup, L->tm_wdownT, p);
+    CKB(cudaGetLastError());
+  }
+  // dL/dx from the experts: DA K_e (the down kernel on the transposed keys)
+  CKB(launch_down_streaming(L, L->tm_da, L->tm_wupT, nullptr, dx, s));
+  // dL/dK_e and dL/dV_e
+  {
+    WgradParams p;
+    p.counts = w.grp_cnt; p.row_tok = w.row_tok;
+    p.x = static_cast<const __nv_bfloat16*>(x);
+    p.dy = static_cast<const __nv_bfloat16*>(dy);
+    p.dw_up = dw_up; p.dw_down = dw_down;
+    p.G = L->G; p.region = L->region_rows; p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;
+    p.N = L->up_bn; p.n_nc = L->up_nsub; p.n_c = L->d / 128;
+    p.status = w.status;
+    p.wait_limit = gemm_wait_limit();
+    bwd_wgrad_kernel<<<L->n_sm, kThreads, L->bwd_wgrad_smem, s>>>(L->tm_da64, L->tm_hw64, p);
+    CKB(cudaGetLastError());
+  }
+  // router: dL/dz, its share of dL/dx, dL/dW*, dL/dbias
+  const int adaptive = isnan(L->th.alpha_fixed) ? 1 : 0;
+  router_grad_kernel<<<(T * 32 + 255) / 256, 256, 0, s>>>(
+      T, L->K, L->router_cols_pad, L->d, L->tau, adaptive, mask, w.alpha, w.s, w.dwt, L->wr, w.dz,
+      dx);
+  CKB(cudaGetLastError());
+  router_wgrad_kernel<<<dim3((L->d + 255) / 256, (T + kRgTokens - 1) / kRgTokens), 256,
+                        sizeof(float) * kRgTokens * K1, s>>>(
+      T, K1, L->d, mask, static_cast<const __nv_bfloat16*>(x), w.dz, dw_router, dbias);
+  CKB(cudaGetLastError());
+  if (lambda_div != 0.f || l_div) {
+    diversity_kernel<<<1, 256, sizeof(float) * (K1 * K1 + 8), s>>>(
+        K1, L->d, L->router_cols_pad, L->wr, lambda_div, dw_router, l_div);
+    CKB(cudaGetLastError());
+  }
+#undef CKB
+  return UNIF_MOE_OK;
+}
+
+}  // namespace unif

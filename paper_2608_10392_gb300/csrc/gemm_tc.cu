@@ -255,11 +255,12 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     // down: this thread's row token and weight, fetched one tile ahead
     int t_nxt = -1;
     float w_nxt = 0.f;
+    // (row_w == nullptr: every row's weight is 1)
     if (MODE == 1 && blockIdx.x < n_items &&
         q * 32 + lane < p.tile_rows[blockIdx.x / p.n_sub]) {
       const int r = p.tile_row0[blockIdx.x / p.n_sub] + q * 32 + lane;
       t_nxt = p.row_tok[r];
-      w_nxt = p.row_w[r];
+      w_nxt = p.row_w ? p.row_w[r] : 1.f;
     }
     for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
       const int tile = item / p.n_sub, ns = item % p.n_sub;
@@ -271,7 +272,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         const int r = p.tile_row0[nt] + q * 32 + lane;
         const bool real = q * 32 + lane < p.tile_rows[nt];
         t_nxt = real ? p.row_tok[r] : -1;
-        w_nxt = real ? p.row_w[r] : 0.f;
+        w_nxt = real ? (p.row_w ? p.row_w[r] : 1.f) : 0.f;
       }
       if (!wait_warp(accf_bar(acc), acc_phase, abort_flag, p.status, p.wait_limit)) break;
       tc_fence_after();
@@ -658,6 +659,28 @@ cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t
   p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
   tc::grouped_gemm_kernel<1><<<L->n_sm, tc::kThreads, tc::Cfg<1>::kSmem, s>>>(L->tm_h, L->tm_wdown,
                                                                              p);
+  return cudaGetLastError();
+}
+
+// The streaming down-projection kernel on other operands: out[tok] +=
+// w(row) * A[row] B_e[H_b, :] over the tile list, A an [rows][M] bf16 map
+// like h's and B a [(K+1) d][H] bf16 map like w_down's; row_w == nullptr
+// gives every row weight 1 (the backward's dL/dx = dL/da K_e^T).
+cudaError_t launch_down_streaming(unif_moe_layer* L, const CUtensorMap& tmA,
+                                  const CUtensorMap& tmB, const float* row_w, float* out,
+                                  cudaStream_t s) {
+  tc::Params p;
+  p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group; p.tile_row0 = L->ws.tile_row0;
+  p.tile_rows = L->ws.tile_rows;
+  p.row_tok = L->ws.row_tok; p.row_w = row_w;
+  p.B = L->B; p.M = L->M; p.H = L->H; p.d = L->d;
+  p.x = nullptr;
+  p.h = nullptr;
+  p.y32 = out;
+  p.status = L->ws.status;
+  p.wait_limit = tc::g_wait_limit;
+  p.n_sub = L->down_nsub; p.bn = L->down_bn; p.num_kb = L->M / tc::kBK;
+  tc::grouped_gemm_kernel<1><<<L->n_sm, tc::kThreads, tc::Cfg<1>::kSmem, s>>>(tmA, tmB, p);
   return cudaGetLastError();
 }
 

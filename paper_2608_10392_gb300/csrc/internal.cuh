@@ -82,6 +82,13 @@ struct Workspace {
   int32_t* b_stage = nullptr;
   int32_t* k_stage = nullptr;
   int* status = nullptr;         // device status word
+  // Backward pass (UNIF_MOE_FEATURE_BACKWARD).
+  void* w_upT = nullptr;         // [K+1][d][H] keys transposed (layer dtype)
+  void* w_downT = nullptr;       // [K+1][H][d] values transposed
+  void* da = nullptr;            // [max_rows][M] dL/da per group row (rows as h)
+  void* hw = nullptr;            // [max_rows][M] w GeLU(a) per group row
+  float* dwt = nullptr;          // [max_tokens][K+1] dL/dalpha, dL/ds_j per token
+  float* dz = nullptr;           // [max_tokens][K+1] dL/dz (router logits)
 };
 
 }  // namespace unif
@@ -139,6 +146,13 @@ struct unif_moe_layer {
   // number of output column slices run as separate work items
   int ws_down_bn = 0, ws_down_nsub = 0, down_slices = 1;
   CUtensorMap tm_wdown_ws;  // w_down slabs of ws_down_bn rows
+  // backward: transposed weights and the per-row gradient buffers
+  CUtensorMap tm_wdownT;    // w_downT [(K+1) H][d], boxes of 64 x up_bn
+  CUtensorMap tm_wupT;      // w_upT [(K+1) d][H], boxes of 64 x down_bn
+  CUtensorMap tm_da;        // da [max_rows][M], boxes of 64 x 128 (dx GEMM A operand)
+  CUtensorMap tm_da64;      // da, boxes of 64 x 64 (weight-gradient operand)
+  CUtensorMap tm_hw64;      // hw, boxes of 64 x 64
+  uint32_t bwd_hidden_smem = 0, bwd_wgrad_smem = 0;
   // Optional caller-owned timing events recorded at the stage boundaries.
   cudaEvent_t stage_ev[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
 };
@@ -163,6 +177,8 @@ cudaError_t launch_combine_residual(unif_moe_layer* L, const void* x, void* out,
                                     float eps, bool norm, int T, cudaStream_t s);
 // Tile list from the router's group sizes, for streaming grouped GEMMs.
 cudaError_t launch_tile_list(unif_moe_layer* L, cudaStream_t s);
+// The same from group sizes at `sizes` (the forward's, for the backward).
+cudaError_t launch_tile_list_from(unif_moe_layer* L, const int32_t* sizes, cudaStream_t s);
 cudaError_t launch_sort_affinities(unif_moe_layer* L, int T, int32_t* q, float* p,
                                    cudaStream_t s);
 int forward_chunks(int T);
@@ -186,5 +202,14 @@ int router_tc_setup(unif_moe_layer* L);
 bool router_can_group(int Cp, int K, int G);
 cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
                              int32_t* b_out, int32_t* k_out, cudaStream_t s);
+cudaError_t launch_down_streaming(unif_moe_layer* L, const CUtensorMap& tmA,
+                                  const CUtensorMap& tmB, const float* row_w, float* out,
+                                  cudaStream_t s);
+// Backward pass (backward.cu).
+int backward_setup(unif_moe_layer* L);  // workspace maps and kernel attributes
+cudaError_t launch_transpose_weights(unif_moe_layer* L, cudaStream_t s);
+int backward_run(unif_moe_layer* L, const void* x, const void* dy, int T, const uint8_t* mask,
+                 float* dx, float* dw_up, float* dw_down, float* dw_router, float* dbias,
+                 float lambda_div, float* l_div, cudaStream_t s);
 
 }  // namespace unif

@@ -816,9 +816,13 @@ cudaError_t launch_sort_affinities(unif_moe_layer* L, int T, int32_t* q, float* 
 }
 
 cudaError_t launch_tile_list(unif_moe_layer* L, cudaStream_t s) {
+  return launch_tile_list_from(L, L->ws.grp_fill, s);
+}
+
+cudaError_t launch_tile_list_from(unif_moe_layer* L, const int32_t* sizes, cudaStream_t s) {
   Workspace& w = L->ws;
   tile_list_kernel<<<1, 256, sizeof(int32_t) * (2 * (size_t)L->G + 1), s>>>(
-      w.grp_fill, L->G, L->region_rows, w.n_tiles, w.tile_group, w.tile_row0, w.tile_rows);
+      sizes, L->G, L->region_rows, w.n_tiles, w.tile_group, w.tile_row0, w.tile_rows);
   return cudaGetLastError();
 }
 

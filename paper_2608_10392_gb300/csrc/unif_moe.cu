@@ -70,7 +70,8 @@ void free_all(unif_moe_layer* L) {
                   L->ws.tile_row0, L->ws.row_tok, L->ws.row_w, L->ws.hbuf, L->ws.y32,
                   L->ws.xn, L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
                   L->ws.k_stage, L->ws.status, L->ws.grp_fill,
-                  L->ws.tile_rows};
+                  L->ws.tile_rows, L->ws.w_upT, L->ws.w_downT, L->ws.da, L->ws.hw,
+                  L->ws.dwt, L->ws.dz};
   for (void* q : ptrs)
     if (q) cudaFree(q);
 }
@@ -96,7 +97,7 @@ const char* unif_moe_last_error(void) { return unif::g_err; }
 
 void unif_moe_default_options(unif_moe_options* opts) {
   if (!opts) return;
-  opts->features = UNIF_MOE_FEATURES_ALL;
+  opts->features = UNIF_MOE_FEATURES_DEFAULT;
   opts->gemm_kernels = UNIF_MOE_GEMM_AUTO;
 }
 
@@ -243,6 +244,18 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
     if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.out_stage), es * T * d_model);
     ALLOC(w.mask_stage, T); ALLOC(w.b_stage, T); ALLOC(w.k_stage, T);
   }
+  if (o.features & UNIF_MOE_FEATURE_BACKWARD) {
+    if (rc == UNIF_MOE_OK && (dtype != UNIF_MOE_BF16 || !L->fused_group || d_model % 128 != 0)) {
+      set_error("the backward pass needs a bf16 layer with d %% 128 == 0 (d=%d)", d_model);
+      rc = UNIF_MOE_ERR_SHAPE;
+    }
+    const size_t wbytes = es * E * d_ff * d_model;
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.w_upT), wbytes);
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.w_downT), wbytes);
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.da), es * (size_t)L->max_rows * M);
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.hw), es * (size_t)L->max_rows * M);
+    ALLOC(w.dwt, T * E); ALLOC(w.dz, T * E);
+  }
 #undef ALLOC
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
                             cudaMemset(w.y32, 0, sizeof(float) * L->pass_tokens * d_model) !=
@@ -261,6 +274,7 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   }
   if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::gemm_tc_setup(L);
   if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::router_tc_setup(L);
+  if (rc == UNIF_MOE_OK && (o.features & UNIF_MOE_FEATURE_BACKWARD)) rc = unif::backward_setup(L);
   if (rc != UNIF_MOE_OK) {
     free_all(L);
     delete L;
@@ -280,6 +294,7 @@ int unif_moe_load_weights(unif_moe_t L, const void* w_router, const void* w_up,
   CK(cudaMemcpyAsync(L->w_up, w_up, bytes, cudaMemcpyDeviceToDevice, s));
   CK(cudaMemcpyAsync(L->w_down, w_down, bytes, cudaMemcpyDeviceToDevice, s));
   CK(unif::launch_prototypes(L, w_router, router_bias, s));
+  if (L->features & UNIF_MOE_FEATURE_BACKWARD) CK(unif::launch_transpose_weights(L, s));
   L->loaded = true;
   return UNIF_MOE_OK;
 }
@@ -408,8 +423,42 @@ int unif_moe_load_upcycled(unif_moe_t L, const void* w_router, const void* w_up_
                        cudaMemcpyDeviceToDevice, s));
   }
   CK(unif::launch_prototypes(L, w_router, router_bias, s));
+  if (L->features & UNIF_MOE_FEATURE_BACKWARD) CK(unif::launch_transpose_weights(L, s));
   L->loaded = true;
   return UNIF_MOE_OK;
+}
+
+int unif_moe_backward(unif_moe_t L, const void* x, const void* dy, int T, const uint8_t* mask,
+                      float* dx, float* dw_up, float* dw_down, float* dw_router, float* dbias,
+                      float lambda_div, float* l_div, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (!(L->features & UNIF_MOE_FEATURE_BACKWARD)) {
+    set_error("backward on a handle created without UNIF_MOE_FEATURE_BACKWARD");
+    return UNIF_MOE_ERR_STATE;
+  }
+  if (L->last_T < 0 || T != L->last_T) {
+    set_error("backward needs the forward of the same T before it (T=%d, last forward %d)", T,
+              L->last_T);
+    return UNIF_MOE_ERR_STATE;
+  }
+  if (T > L->pass_tokens) {
+    set_error("backward of %d tokens: the forward ran in passes of %d", T, L->pass_tokens);
+    return UNIF_MOE_ERR_CAPACITY;
+  }
+  if (!x || !dy || !dx || !dw_up || !dw_down || !dw_router) {
+    set_error("NULL input or output");
+    return UNIF_MOE_ERR_ARG;
+  }
+  if (!aligned16(x) || !aligned16(dy) || !aligned16(dx) || !aligned16(dw_up) ||
+      !aligned16(dw_down) || !aligned16(dw_router)) {
+    set_error("backward buffers must be 16-byte aligned");
+    return UNIF_MOE_ERR_ARG;
+  }
+  if (T == 0) return UNIF_MOE_OK;
+  DeviceGuard dg(L->device);
+  return unif::backward_run(L, x, dy, T, mask, dx, dw_up, dw_down, dw_router, dbias, lambda_div,
+                            l_div, static_cast<cudaStream_t>(stream));
 }
 
 int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_t* token_mask,

@@ -65,7 +65,7 @@ def test_argument_errors_without_gpu(lib):
     assert lib.unif_moe_create(C.byref(h), 64, 256, 4, 4, C.byref(bad), 1, 16) == -1
     opts = pkg.Options()
     lib.unif_moe_default_options(C.byref(opts))
-    assert opts.features == pkg.FEATURES_ALL and opts.gemm_kernels == 0
+    assert opts.features == pkg.FEATURES_DEFAULT and opts.gemm_kernels == 0
     for o in (pkg.Options(8, 0), pkg.Options(3, 2), pkg.Options(3, -1)):  # unknown bit / kind
         assert lib.unif_moe_create_ex(C.byref(h), 64, 256, 4, 4, None, 1, 16, C.byref(o)) == -1
     assert b"options" in lib.unif_moe_last_error()
@@ -74,6 +74,8 @@ def test_argument_errors_without_gpu(lib):
     assert lib.unif_moe_load_upcycled(None, None, None, None, None, None) == -1
     assert lib.unif_moe_sublayer_forward(None, None, None, 4, None, None, None, None, None,
                                          1e-5, 1, None) == -1
+    assert lib.unif_moe_backward(None, None, None, 4, None, None, None, None, None, None, 0.0,
+                                 None, None) == -1
     assert lib.unif_moe_sync_status(None, None) == -1
     assert lib.unif_moe_max_rows(None) == -1
     assert lib.unif_moe_kernels_per_forward(None) == -1
