@@ -25,8 +25,19 @@ MUTANTS = {
     # priorities pin sees it)
     "prototype_sum": ("round_to(sum / (double)M, round_mode)", "round_to(sum, round_mode)"),
     # transposed value matrix
-    "value_transposed": ("V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * d + i) * H + h];",
-                         "V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * H + h) * d + i];"),
+    "value_transposed": ("  for (int e = 0; e <= K; ++e)\n    for (int i = 0; i < d; ++i)\n"
+                         "      for (int h = 0; h < H; ++h)\n"
+                         "        V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * d + i) * H + h];",
+                         "  for (int e = 0; e <= K; ++e)\n    for (int i = 0; i < d; ++i)\n"
+                         "      for (int h = 0; h < H; ++h)\n"
+                         "        V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * H + h) * d + i];"),
+    # the backward's value rows read transposed
+    "bwd_value_transposed": ("  for (int e = 0; e < K1; ++e)\n    for (int i = 0; i < d; ++i)\n"
+                             "      for (int h = 0; h < H; ++h)\n"
+                             "        V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * d + i) * H + h];",
+                             "  for (int e = 0; e < K1; ++e)\n    for (int i = 0; i < d; ++i)\n"
+                             "      for (int h = 0; h < H; ++h)\n"
+                             "        V[((size_t)e * H + h) * d + i] = w_down[((size_t)e * H + h) * d + i];"),
     # residual experts run the shared blocks instead of the complement (Eq. 23)
     "residual_blocks": ("EXPERT_BLOCKS(1 + j, 0);", "EXPERT_BLOCKS(1 + j, 1);"),
     # shared pathway weighted by beta instead of alpha (Eq. 30)
