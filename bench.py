@@ -191,10 +191,14 @@ class OracleRunner:
     """The CPU oracle, as it stands, on the first `tokens` token slots of a
     workload (inputs converted to fp64 once, outside the timing)."""
 
-    def __init__(self, wl):
+    def __init__(self, wl, train=False):
         import oracle
         s = wl.spec
         self.o, self.wl, self.s = oracle, wl, s
+        self.train = train
+        if train:  # a training step: the backward too, for a seeded dL/dy
+            import numpy as np
+            self.dy = np.random.default_rng(17).standard_normal((s.tokens, s.d_model))
         self.rm = oracle.ROUND_BF16 if s.dtype == "bf16" else oracle.ROUND_F32
         self.th = oracle.Thresholds(s.tau, s.alpha_fixed, s.beta_fixed, s.topk_fixed,
                                     s.prefix_blocks)
@@ -206,8 +210,13 @@ class OracleRunner:
         x = self.xa[:tokens]
         t0 = time.perf_counter()
         for _ in range(repeat):
-            self.o.layer(x, self.wr, self.wu, self.wd, self.s.n_blocks, self.th, m,
-                         self.wl.router_bias, self.rm)
+            _, r = self.o.layer(x, self.wr, self.wu, self.wd, self.s.n_blocks, self.th, m,
+                                self.wl.router_bias, self.rm)
+            if self.train:
+                self.o.backward(x, self.wr, self.wu, self.wd, r.shr_mask, r.expert_mask(),
+                                self.s.n_blocks, self.dy[:tokens], self.th, m,
+                                self.wl.router_bias)
+                self.o.diversity(self.wr)
         dt = time.perf_counter() - t0
         valid = tokens if m is None else int(m.sum())
         return valid * repeat / dt, dt, valid * repeat
@@ -268,6 +277,9 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=50)
     ap.add_argument("--routing", default="adaptive", choices=sorted(ROUTINGS),
                     help="routing variant (Table IV ablations, fixed thresholds)")
+    ap.add_argument("--train", action="store_true",
+                    help="time a training step: the forward, then the backward pass with the "
+                         "Gram regulariser (Sec. III-E, lambda_div 0.01)")
     ap.add_argument("--sublayer", default="none", choices=["none", "pre", "post"],
                     help="time the layer inside a Transformer sublayer: x + F(LN(x)) (pre) or "
                          "LN(x + F(x)) (post), seeded LayerNorm parameters")
@@ -291,7 +303,9 @@ def main():
 
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2608_10392_gb300 import Layer
+    from paper_2608_10392_gb300 import FEATURE_BACKWARD, FEATURES_DEFAULT, Layer
+    if args.train and args.sublayer != "none":
+        raise SystemExit("--train times the layer alone")
 
     dist = None
     if world > 1:
@@ -308,7 +322,8 @@ def main():
     T_valid = T if mask is None else int(mask.sum())
     layer = Layer(s.d_model, s.d_ff, s.n_experts, s.n_blocks, dtype=s.dtype, max_tokens=T,
                   tau=s.tau, alpha_fixed=s.alpha_fixed, beta_fixed=s.beta_fixed,
-                  topk_fixed=s.topk_fixed, prefix_blocks=s.prefix_blocks)
+                  topk_fixed=s.topk_fixed, prefix_blocks=s.prefix_blocks,
+                  features=FEATURES_DEFAULT | (FEATURE_BACKWARD if args.train else 0))
     layer.load_weights(w_router.to(dev), w_up.to(dev), w_down.to(dev),
                        None if bias is None else bias.to(dev))
     xd = x.to(dev)
@@ -323,7 +338,21 @@ def main():
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
     flush_r = torch.zeros(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
 
-    if args.sublayer == "none":
+    bwd_ev = None
+    if args.train:
+        gen = torch.Generator().manual_seed(rank + 17)
+        dy = torch.randn(T, s.d_model, generator=gen).to(xd.dtype).to(dev)
+        grads = {}
+
+        def step():
+            layer.forward(xd, out=out, mask=md, shared_counts=bcnt, residual_counts=kcnt)
+            if bwd_ev is not None:
+                bwd_ev[0].record(stream)
+            grads.update(layer.backward(xd, dy, mask=md, lambda_div=0.01, want_bias=True,
+                                        out=grads or None))
+            if bwd_ev is not None:
+                bwd_ev[1].record(stream)
+    elif args.sublayer == "none":
         def step():
             layer.forward(xd, out=out, mask=md, shared_counts=bcnt, residual_counts=kcnt)
     else:
@@ -390,13 +419,19 @@ def main():
     # consecutive kernels. Those events serialise the kernels (no dependent
     # launch overlaps its predecessor), so each duration is the kernel's own
     # launch; the timed steps above run without them.
+    bwd_pairs = [(mk(), mk()) for _ in range(K)] if args.train else None
     for i in range(K):
         flush.zero_()
         flush_r.max()
         layer.set_stage_events(stage_ev[i])
+        if args.train:
+            bwd_ev = bwd_pairs[i]
         step()
     torch.cuda.synchronize(dev)
     layer.set_stage_events(None)
+    bwd_ev = None
+    if layer.sync_status() != 0:
+        raise RuntimeError("device status word set during the per-kernel pass")
 
     step_ms = [starts[i].elapsed_time(ends[i]) for i in range(K)]
     total_ms = sum(step_ms)
@@ -417,7 +452,7 @@ def main():
     e2e_ms = []
     # (the host-buffer entry point runs the layer alone: no end-to-end line
     # for a sublayer run)
-    for _ in range(args.e2e_steps if args.sublayer == "none" else 0):
+    for _ in range(args.e2e_steps if args.sublayer == "none" and not args.train else 0):
         a, b = mk(), mk()
         a.record(stream)
         layer.forward_host(xh, oh, mh, bh, kh)
@@ -513,12 +548,26 @@ def main():
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": statistics.fmean(e2e_ms)},
         # (a norm-first sublayer adds its layer-normalisation kernel)
-        "gpu_launches": (layer.kernels_per_forward() * n_pass + (args.sublayer == "pre")) * K,
+        # (a norm-first sublayer adds its layer-normalisation kernel; a
+        # training step the backward's seven kernels)
+        "gpu_launches": (layer.kernels_per_forward() * n_pass + (args.sublayer == "pre") +
+                         (7 if args.train else 0)) * K,
         "clocks": clocks,
     }
+    if args.train:
+        bwd_ms = statistics.fmean(a.elapsed_time(b) for a, b in bwd_pairs)
+        # backward GEMM work: the hidden kernel's two products, dL/dx and the
+        # two weight gradients, each 2 d M flops per (token, pair)
+        line["config"]["step"] = ("training: forward, then backward with the Gram regulariser "
+                                  "(Sec. III-E, lambda_div 0.01)")
+        line["train"] = {"backward_ms": bwd_ms,
+                         "backward_TFLOP/s": 5.0 * gemm_flops / bwd_ms / 1e9,
+                         "step_activated_TFLOP/s": 7.0 * gemm_flops / ms / 1e9,
+                         "backward_kind": "timed in the per-kernel pass (events around the "
+                                          "backward call)"}
     if not args.no_cpu_baseline and world >= 1:
         wl = workloads.Workload(s, w_router, w_up, w_down, bias, x, mask)
-        v, dt, n, tokens, repeat = OracleRunner(wl).sample()
+        v, dt, n, tokens, repeat = OracleRunner(wl, train=args.train).sample()
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": oracle_cores(), "kind": "oracle",
                                 "sample": "first %d of the workload's %d token slots, %d passes "
                                           "(%d valid tokens in all, %.1f s)"

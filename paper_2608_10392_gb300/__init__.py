@@ -211,19 +211,22 @@ class Layer:
         return out
 
     def backward(self, x: torch.Tensor, dy: torch.Tensor, mask: Optional[torch.Tensor] = None,
-                 lambda_div: float = 0.0, want_bias: bool = False, stream=None) -> dict:
+                 lambda_div: float = 0.0, want_bias: bool = False, out: Optional[dict] = None,
+                 stream=None) -> dict:
         """Gradients of the last forward (which must have run on x) given
         dL/dy (Sec. III-E): dict of fp32 CUDA tensors dx, dw_up, dw_down,
-        dw_router (plus lambda_div dL_div/dW*), dbias (want_bias), l_div."""
+        dw_router (plus lambda_div dL_div/dW*), dbias (want_bias), l_div;
+        `out`, such a dict from an earlier call, is filled again."""
         T = x.shape[0]
         dev = x.device
         f32 = dict(dtype=torch.float32, device=dev)
-        g = dict(dx=torch.empty(T, self.d, **f32),
-                 dw_up=torch.empty(self.K + 1, self.H, self.d, **f32),
-                 dw_down=torch.empty(self.K + 1, self.d, self.H, **f32),
-                 dw_router=torch.empty(self.d, self.K + 1, **f32),
-                 dbias=torch.empty(self.K + 1, **f32) if want_bias else None,
-                 l_div=torch.empty(1, **f32))
+        g = out if out is not None else dict(
+            dx=torch.empty(T, self.d, **f32),
+            dw_up=torch.empty(self.K + 1, self.H, self.d, **f32),
+            dw_down=torch.empty(self.K + 1, self.d, self.H, **f32),
+            dw_router=torch.empty(self.d, self.K + 1, **f32),
+            dbias=torch.empty(self.K + 1, **f32) if want_bias else None,
+            l_div=torch.empty(1, **f32))
         _check(lib().unif_moe_backward(self._h, _ptr(x), _ptr(dy), T, _ptr(mask), _ptr(g["dx"]),
                                        _ptr(g["dw_up"]), _ptr(g["dw_down"]),
                                        _ptr(g["dw_router"]), _ptr(g["dbias"]),
