@@ -34,13 +34,12 @@ namespace unif {
 namespace tc {
 namespace bwd {
 
-// GeLU (exact erf form, Sec. II-A) and its derivative Phi(a) + a phi(a).
-__device__ __forceinline__ float gelu_f(float a) {
-  return 0.5f * a * (1.0f + erff(a * 0.70710678118654752f));
-}
-__device__ __forceinline__ float gelu_grad_f(float a) {
-  return 0.5f * (1.0f + erff(a * 0.70710678118654752f)) +
-         a * 0.39894228040143268f * expf(-0.5f * a * a);
+// GeLU (exact erf form, Sec. II-A) and its derivative Phi(a) + a phi(a),
+// from one evaluation of Phi.
+__device__ __forceinline__ void gelu_and_grad(float a, float& g, float& dg) {
+  const float cdf = 0.5f * (1.0f + erff(a * 0.70710678118654752f));
+  g = a * cdf;
+  dg = cdf + a * 0.39894228040143268f * __expf(-0.5f * a * a);
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -255,11 +254,13 @@ bwd_hidden_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_consta
         for (int i = 0; i < 8; ++i) {
           float d0 = 0.f, d1 = 0.f, h0 = 0.f, h1 = 0.f;
           if (tok >= 0) {
-            const float g0 = gelu_f(a[2 * i]), g1 = gelu_f(a[2 * i + 1]);
+            float g0, g1, dg0, dg1;
+            gelu_and_grad(a[2 * i], g0, dg0);
+            gelu_and_grad(a[2 * i + 1], g1, dg1);
             dot = fmaf(g0, gv[2 * i], dot);
             dot = fmaf(g1, gv[2 * i + 1], dot);
-            d0 = w * gv[2 * i] * gelu_grad_f(a[2 * i]);
-            d1 = w * gv[2 * i + 1] * gelu_grad_f(a[2 * i + 1]);
+            d0 = w * gv[2 * i] * dg0;
+            d1 = w * gv[2 * i + 1] * dg1;
             h0 = w * g0;
             h1 = w * g1;
           }
@@ -301,8 +302,8 @@ bwd_hidden_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_consta
 // the gathered rows (x, dy) and the TMA tiles (DA, HW) keep the 128-byte
 // swizzled row layout, read with MN-major descriptors. Each item owns its
 // output exactly (no atomics); groups without rows give zeros.
-// Roles: warps 0-3 fill the ring (warp 2s: x rows of stage s and the DA/HW
-// tiles by TMA; warp 2s+1: dy rows), warp 4 MMAs, warps 5-12 epilogue.
+// Roles: warps 0-3 fill the 4-deep ring (warp s: the x and dy rows of stage
+// s, and the DA/HW tiles by TMA), warp 4 MMAs, warps 5-12 epilogue.
 // ---------------------------------------------------------------------------
 struct WgradParams {
   const int32_t* counts;   // [G] group sizes (the forward's)
@@ -316,8 +317,10 @@ struct WgradParams {
   long long wait_limit;
 };
 
-constexpr uint32_t kRows = 64;                 // group rows per stage
-constexpr uint32_t kPBytes = 2u * kRows * 128u;  // 128 features x 64 rows (two 64-column blocks)
+constexpr uint32_t kRows = 32;                 // group rows per stage
+constexpr uint32_t kPBytes = 2u * kRows * 128u;  // 128 features x 32 rows (two 64-column blocks)
+constexpr int kWStages = 4;                      // one stage per producer warp
+constexpr int kQuarters = kBM / (int)kRows;      // stages per 128-row tile
 
 __host__ __device__ constexpr uint32_t wgrad_stage_bytes(int N) {
   return 2u * kPBytes + 2u * (uint32_t)(N / 64) * kRows * 128u;
@@ -337,21 +340,21 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
   auto sqa = [&](int s) { return s0 + s * stage_bytes + 2 * kPBytes; };
   auto sqh = [&](int s) { return s0 + s * stage_bytes + 2 * kPBytes + qbytes; };
   uint8_t* gen_base = smem;  // generic pointer for zero-filling padding rows
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * stage_bytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWStages * stage_bytes);
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
-  const uint32_t accf = bar0 + 8u * (2 * kStages);
-  const uint32_t acce = bar0 + 8u * (2 * kStages + 1);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 2);
+  auto empty_bar = [&](int s) { return bar0 + 8u * (kWStages + s); };
+  const uint32_t accf = bar0 + 8u * (2 * kWStages);
+  const uint32_t acce = bar0 + 8u * (2 * kWStages + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kWStages + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int32_t* first_s = reinterpret_cast<int32_t*>(tmem_slot + 4);  // [G + 1] first tiles
   int32_t* cnt_s = first_s + p.G + 1;                             // [G] sizes
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(full_bar(s), 2);
+    for (int s = 0; s < kWStages; ++s) {
+      mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
     mbar_init(accf, 1);
@@ -377,9 +380,10 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
     g = item / (p.n_nc * p.n_c);
   };
 
-  if (warp < 4) {
-    const int my_stage = warp >> 1, kind = warp & 1;
-    const __nv_bfloat16* src = kind == 0 ? p.x : p.dy;
+  if (warp < kWStages) {
+    // ---- producers: warp w owns stage w: the x and dy rows of its 32 group
+    // rows, and lane 0 brings the DA and HW tiles by TMA ----
+    const int my_stage = warp;
     const int j = lane & 7, rsub = lane >> 3;
     bool ok = true;
     int seq = 0;
@@ -388,15 +392,15 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
       decode(item, g, c, nc);
       const int t_first = first_s[g], nt = first_s[g + 1] - t_first;
       const int size = cnt_s[g];
-      for (int kt = 0; kt < nt * 2 && ok; ++kt, ++seq) {  // 64-row halves of the group's tiles
-        const int stage = seq % kStages;
+      for (int kt = 0; kt < nt * kQuarters && ok; ++kt, ++seq) {  // 32-row quarters of the tiles
+        const int stage = seq % kWStages;
         if (stage != my_stage) continue;
-        const uint32_t phase = (uint32_t)(seq / kStages) & 1u;
+        const uint32_t phase = (uint32_t)(seq / kWStages) & 1u;
         ok = wait_warp(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
         if (!ok) break;
-        const int row_in_group = kt * (int)kRows;  // first row of this half in the group
-        const int crow = (t_first + kt / 2) * kBM + (kt & 1) * (int)kRows;  // compact DA/HW row
-        if (kind == 0 && lane == 0) {
+        const int row_in_group = kt * (int)kRows;  // first row of this quarter in the group
+        const int crow = (t_first + kt / kQuarters) * kBM + (kt % kQuarters) * (int)kRows;
+        if (lane == 0) {
           mbar_expect_tx_only(full_bar(stage), 2u * qbytes);
           for (int b = 0; b < p.N / 64; ++b) {
             tma_load_2d(sqa(stage) + b * kRows * 128u, &tm_da, full_bar(stage), nc * p.N + b * 64,
@@ -405,26 +409,25 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
                         crow);
           }
         }
-        // this half's 64 row tokens: lane l holds rows l and l + 32 (-1: padding)
-        int tk[2];
+        // this quarter's row tokens: lane l holds row l (-1: padding)
+        const int rg = row_in_group + lane;
+        const int tk = rg < size ? p.row_tok[(size_t)g * p.region + rg] : -1;
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
-          const int rg = row_in_group + 32 * i + lane;
-          tk[i] = rg < size ? p.row_tok[(size_t)g * p.region + rg] : -1;
-        }
-        const uint32_t dst = kind == 0 ? spx(stage) : spy(stage);
-        const __nv_bfloat16* sj = src + (size_t)c * 128 + j * 8;
+        for (int kind = 0; kind < 2; ++kind) {
+          const uint32_t dst = kind == 0 ? spx(stage) : spy(stage);
+          const __nv_bfloat16* sj = (kind == 0 ? p.x : p.dy) + (size_t)c * 128 + j * 8;
 #pragma unroll
-        for (int b = 0; b < 2; ++b) {
+          for (int b = 0; b < 2; ++b) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int r = 4 * i + rsub;
-            const int t = __shfl_sync(0xffffffffu, tk[r >> 5], r & 31);
-            const uint32_t off = b * kRows * 128u + r * 128u + ((j ^ (r & 7)) << 4);
-            if (t >= 0)
-              cp_async16(dst + off, sj + (size_t)t * p.d + b * 64);
-            else  // padding rows contribute zeros to the row sums
-              *reinterpret_cast<uint4*>(gen_base + (dst - s0) + off) = make_uint4(0u, 0u, 0u, 0u);
+            for (int i = 0; i < (int)kRows / 4; ++i) {
+              const int r = 4 * i + rsub;
+              const int t = __shfl_sync(0xffffffffu, tk, r);
+              const uint32_t off = b * kRows * 128u + r * 128u + ((j ^ (r & 7)) << 4);
+              if (t >= 0)
+                cp_async16(dst + off, sj + (size_t)t * p.d + b * 64);
+              else  // padding rows contribute zeros to the row sums
+                *reinterpret_cast<uint4*>(gen_base + (dst - s0) + off) = make_uint4(0u, 0u, 0u, 0u);
+            }
           }
         }
         cp_async_commit();
@@ -436,7 +439,7 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
     }
   } else if (warp == kMmaWarp) {
     const uint32_t idesc = idesc_bf16_mn(kBM, p.N);
-    const uint32_t lbo = kRows * 128u;  // 64-element MN blocks of 64 rows
+    const uint32_t lbo = kRows * 128u;  // 64-element MN blocks of kRows rows
     int seq = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
@@ -448,9 +451,9 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
       ok = wait_warp(acce, acc_phase ^ 1u, abort_flag, p.status, p.wait_limit);
       if (!ok) break;
       tc_fence_after();
-      for (int kt = 0; kt < nt * 2; ++kt, ++seq) {
-        const int stage = seq % kStages;
-        const uint32_t phase = (uint32_t)(seq / kStages) & 1u;
+      for (int kt = 0; kt < nt * kQuarters; ++kt, ++seq) {
+        const int stage = seq % kWStages;
+        const uint32_t phase = (uint32_t)(seq / kWStages) & 1u;
         ok = wait_warp(full_bar(stage), phase, abort_flag, p.status, p.wait_limit);
         if (!ok) break;
         tc_fence_after();
@@ -527,12 +530,15 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
 // One warp per token: dL/dz_0 = dL/dalpha (1 - 2 tau) sigma(z_0)(1 - sigma(z_0))
 // (adaptive alpha; sigma(z_0) = (alpha - tau) / (1 - 2 tau) from the stored
 // alpha), dL/dz_{1+j} = s_j (dL/ds_j - sum_l s_l dL/ds_l); then dx[t] +=
-// dL/dz W*^T (W* = the router matrix's first K+1 columns, fp32 [d][Cp]).
-__global__ void router_grad_kernel(int T, int K, int Cp, int d, float tau, int adaptive,
-                                   const uint8_t* __restrict__ mask,
-                                   const float* __restrict__ alpha, const float* __restrict__ s,
-                                   const float* __restrict__ dwt, const float* __restrict__ wr,
-                                   float* __restrict__ dz, float* __restrict__ dx) {
+// dL/dz W*^T, with W*^T the router's first K+1 columns transposed (fp32
+// [K+1][d], so that the lanes read consecutive features). Lane l keeps
+// dL/dz_c for c = l, l + 32, l + 64 in registers.
+__global__ void __launch_bounds__(256)
+router_grad_kernel(int T, int K, int d, float tau, int adaptive,
+                   const uint8_t* __restrict__ mask, const float* __restrict__ alpha,
+                   const float* __restrict__ s, const float* __restrict__ dwt,
+                   const float* __restrict__ wrT, float* __restrict__ dz,
+                   float* __restrict__ dx) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (warp >= T) return;
   const int t = warp;
@@ -548,101 +554,139 @@ __global__ void router_grad_kernel(int T, int K, int Cp, int d, float tau, int a
   for (int j = lane; j < K; j += 32) part += st[j] * gt[1 + j];
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-  for (int j = lane; j < K; j += 32) dzt[1 + j] = st[j] * (gt[1 + j] - part);
-  if (lane == 0) {
-    float dz0 = 0.f;
-    if (adaptive && tau < 0.5f) {
-      const float sg = (alpha[t] - tau) / (1.0f - 2.0f * tau);
-      dz0 = gt[0] * (1.0f - 2.0f * tau) * sg * (1.0f - sg);
+  float zc[3];  // dL/dz_c for c = lane + 32 u
+#pragma unroll
+  for (int u = 0; u < 3; ++u) {
+    const int c = lane + 32 * u;
+    float v = 0.f;
+    if (c == 0) {
+      if (adaptive && tau < 0.5f) {
+        const float sg = (alpha[t] - tau) / (1.0f - 2.0f * tau);
+        v = gt[0] * (1.0f - 2.0f * tau) * sg * (1.0f - sg);
+      }
+    } else if (c < K1) {
+      v = st[c - 1] * (gt[c] - part);
     }
-    dzt[0] = dz0;
+    zc[u] = v;
+    if (c < K1) dzt[c] = v;
   }
-  __syncwarp();
   float* dxt = dx + (size_t)t * d;
-  for (int i = lane; i < d; i += 32) {
+  for (int i0 = 0; i0 < d; i0 += 32) {
+    const int i = i0 + lane;
     float acc = 0.f;
-    for (int c = 0; c < K1; ++c) acc = fmaf(dzt[c], wr[(size_t)i * Cp + c], acc);
-    dxt[i] += acc;
+    for (int c = 0; c < K1; ++c) {
+      const float zv = __shfl_sync(0xffffffffu, zc[c >> 5], c & 31);
+      if (i < d) acc = fmaf(zv, wrT[(size_t)c * d + i], acc);
+    }
+    if (i < d) dxt[i] += acc;
+  }
+}
+
+// W*^T: the router's first K+1 columns (fp32 [d][Cp]) as [K+1][d].
+__global__ void router_transpose_kernel(int K1, int d, int Cp, const float* __restrict__ wr,
+                                        float* __restrict__ wrT) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k < K1 * d) {
+    const int c = k / d, i = k % d;
+    wrT[k] = wr[(size_t)i * Cp + c];
   }
 }
 
 // dL/dW*[i][c] = sum_t x[t][i] dL/dz[t][c] and dL/dbias[c] = sum_t dL/dz[t][c]:
-// block (i-block of 256 features, 128-token chunk); partial sums added
-// atomically (the outputs start at zero).
-constexpr int kRgTokens = 128;
+// block (32 features x 8 token lanes) of one token slice; the 8 lanes'
+// partial sums are added in shared memory, then once per block into the
+// outputs (which start at zero).
+constexpr int kRgSlices = 16;
 __global__ void __launch_bounds__(256)
 router_wgrad_kernel(int T, int K1, int d, const uint8_t* __restrict__ mask,
                     const __nv_bfloat16* __restrict__ x, const float* __restrict__ dz,
                     float* __restrict__ dw_router, float* __restrict__ dbias) {
-  extern __shared__ float dz_s[];  // [kRgTokens][K1]
-  const int t0 = blockIdx.y * kRgTokens;
-  const int nt = min(kRgTokens, T - t0);
-  for (int k = threadIdx.x; k < nt * K1; k += blockDim.x) {
-    const int t = t0 + k / K1;
-    dz_s[k] = (mask && !mask[t]) ? 0.f : dz[(size_t)t0 * K1 + k];
-  }
-  __syncthreads();
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < d) {
-    for (int c0 = 0; c0 < K1; c0 += 16) {
-      float acc[16];
+  __shared__ float red[8][32][17];
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const int i = blockIdx.x * 32 + tx;
+  const int per = (T + gridDim.y - 1) / gridDim.y;
+  const int t_begin = blockIdx.y * per, t_end = min(T, t_begin + per);
+  for (int c0 = 0; c0 < K1; c0 += 16) {
+    float acc[16], bacc[16];
 #pragma unroll
-      for (int u = 0; u < 16; ++u) acc[u] = 0.f;
-      for (int tt = 0; tt < nt; ++tt) {
-        const int t = t0 + tt;
-        const float xv = (mask && !mask[t]) ? 0.f : __bfloat162float(x[(size_t)t * d + i]);
-#pragma unroll
-        for (int u = 0; u < 16; ++u)
-          if (c0 + u < K1) acc[u] = fmaf(xv, dz_s[tt * K1 + c0 + u], acc[u]);
-      }
+    for (int u = 0; u < 16; ++u) acc[u] = bacc[u] = 0.f;
+    for (int t = t_begin + ty; t < t_end; t += 8) {
+      if (mask && !mask[t]) continue;
+      const float xv = i < d ? __bfloat162float(x[(size_t)t * d + i]) : 0.f;
+      const float* zt = dz + (size_t)t * K1 + c0;
 #pragma unroll
       for (int u = 0; u < 16; ++u)
-        if (c0 + u < K1) atomicAdd(dw_router + (size_t)i * K1 + c0 + u, acc[u]);
+        if (c0 + u < K1) {
+          const float zv = zt[u];
+          acc[u] = fmaf(xv, zv, acc[u]);
+          bacc[u] += zv;
+        }
     }
-  }
-  if (dbias && blockIdx.x == 0) {
-    for (int c = threadIdx.x; c < K1; c += blockDim.x) {
-      float acc = 0.f;
-      for (int tt = 0; tt < nt; ++tt) acc += dz_s[tt * K1 + c];
-      atomicAdd(dbias + c, acc);
+#pragma unroll
+    for (int u = 0; u < 16; ++u) red[ty][tx][u] = acc[u];
+    __syncthreads();
+    if (ty == 0 && i < d) {
+      for (int u = 0; u < 16 && c0 + u < K1; ++u) {
+        float v = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) v += red[w][tx][u];
+        atomicAdd(dw_router + (size_t)i * K1 + c0 + u, v);
+      }
+    }
+    __syncthreads();
+    if (dbias && blockIdx.x == 0) {  // the bias sums, from lane 0 of each token lane
+#pragma unroll
+      for (int u = 0; u < 16; ++u) red[ty][tx][u] = tx == 0 ? bacc[u] : 0.f;
+      __syncthreads();
+      if (threadIdx.x < 16 && c0 + (int)threadIdx.x < K1) {
+        float v = 0.f;
+        for (int w = 0; w < 8; ++w) v += red[w][0][threadIdx.x];
+        atomicAdd(dbias + c0 + threadIdx.x, v);
+      }
+      __syncthreads();
     }
   }
 }
 
-// Gram regulariser (Eq. diversity-loss): A = W*^T W* - I over the K+1 router
-// columns, L_div = ||A||_F; dW* += lambda 2 W* A / L_div (nothing where
-// L_div = 0). One block; A in shared memory ([K1][K1] fp32).
+// Gram regulariser (Eq. diversity-loss): A = W*^T W* - I over the K+1
+// router columns (one block per entry, reduced over d), then L_div = ||A||_F
+// and dW* += lambda 2 W* A / L_div (nothing where L_div = 0), W*^T as
+// [K+1][d] fp32.
+__global__ void __launch_bounds__(128)
+gram_kernel(int K1, int d, const float* __restrict__ wrT, float* __restrict__ A) {
+  __shared__ float red[4];
+  const int a = blockIdx.x / K1, b = blockIdx.x % K1;
+  float g = 0.f;
+  for (int i = threadIdx.x; i < d; i += blockDim.x)
+    g = fmaf(wrT[(size_t)a * d + i], wrT[(size_t)b * d + i], g);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = g;
+  __syncthreads();
+  if (threadIdx.x == 0) A[blockIdx.x] = red[0] + red[1] + red[2] + red[3] - (a == b ? 1.f : 0.f);
+}
+
 __global__ void __launch_bounds__(256)
-diversity_kernel(int K1, int d, int Cp, const float* __restrict__ wr, float lambda,
-                 float* __restrict__ dw_router, float* __restrict__ l_out) {
-  extern __shared__ float A_s[];  // [K1][K1], then one reduction slot per warp
-  float* red = A_s + K1 * K1;
+diversity_grad_kernel(int K1, int d, const float* __restrict__ wrT, const float* __restrict__ A,
+                      float lambda, float* __restrict__ dw_router, float* __restrict__ l_out) {
+  __shared__ float red[8];
   float ss = 0.f;
-  for (int k = threadIdx.x; k < K1 * K1; k += blockDim.x) {
-    const int a = k / K1, b = k % K1;
-    float g = 0.f;
-    for (int i = 0; i < d; ++i) g = fmaf(wr[(size_t)i * Cp + a], wr[(size_t)i * Cp + b], g);
-    g -= (a == b) ? 1.f : 0.f;
-    A_s[k] = g;
-    ss += g * g;
-  }
+  for (int k = threadIdx.x; k < K1 * K1; k += blockDim.x) ss = fmaf(A[k], A[k], ss);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
   float tot = 0.f;
-  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
+#pragma unroll
+  for (int w = 0; w < 8; ++w) tot += red[w];
   const float L = sqrtf(tot);
-  if (threadIdx.x == 0 && l_out) *l_out = L;
-  if (L > 0.f && lambda != 0.f && dw_router) {
-    const float scale = 2.f * lambda / L;
-    for (int k = threadIdx.x; k < d * K1; k += blockDim.x) {
-      const int i = k / K1, b = k % K1;
-      float g = 0.f;
-      for (int a = 0; a < K1; ++a) g = fmaf(wr[(size_t)i * Cp + a], A_s[a * K1 + b], g);
-      dw_router[k] += scale * g;
-    }
-  }
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k == 0 && l_out) *l_out = L;
+  if (k >= d * K1 || !(L > 0.f) || lambda == 0.f || !dw_router) return;
+  const int i = k / K1, b = k % K1;
+  float g = 0.f;
+  for (int a = 0; a < K1; ++a) g = fmaf(wrT[(size_t)a * d + i], A[a * K1 + b], g);
+  dw_router[k] += 2.f * lambda / L * g;
 }
 
 // out[e][c][r] = in[e][r][c] for bf16 [E][R][C] (32 x 32 tiles through shared
@@ -675,14 +719,14 @@ int backward_setup(unif_moe_layer* L) {
   if (!encode_bf16_map(&L->tm_wdownT, w.w_downT, L->d, E * L->H, tc::kBK, L->up_bn, 128) ||
       !encode_bf16_map(&L->tm_wupT, w.w_upT, L->H, E * L->d, tc::kBK, L->down_bn, 128) ||
       !encode_bf16_map(&L->tm_da, w.da, L->M, (uint64_t)L->max_rows, tc::kBK, tc::kBM, 128) ||
-      !encode_bf16_map(&L->tm_da64, w.da, L->M, (uint64_t)L->max_rows, tc::kBK, kRows, 128) ||
-      !encode_bf16_map(&L->tm_hw64, w.hw, L->M, (uint64_t)L->max_rows, tc::kBK, kRows, 128)) {
+      !encode_bf16_map(&L->tm_da_q, w.da, L->M, (uint64_t)L->max_rows, tc::kBK, kRows, 128) ||
+      !encode_bf16_map(&L->tm_hw_q, w.hw, L->M, (uint64_t)L->max_rows, tc::kBK, kRows, 128)) {
     set_error("cuTensorMapEncodeTiled failed for the backward maps");
     return UNIF_MOE_ERR_CUDA;
   }
   L->bwd_hidden_smem = 1024 + kStages * hidden_stage_bytes(L->up_bn) + 256;
   L->bwd_wgrad_smem =
-      1024 + kStages * wgrad_stage_bytes(L->up_bn) + 64 + 4 * (2 * (uint32_t)L->G + 1) + 16;
+      1024 + kWStages * wgrad_stage_bytes(L->up_bn) + 96 + 4 * (2 * (uint32_t)L->G + 1) + 16;
   if (L->bwd_hidden_smem > 232448 || L->bwd_wgrad_smem > 232448) {
     set_error("backward: shared memory for block width %d and %d groups exceeds 227 KB", L->M,
               L->G);
@@ -762,22 +806,25 @@ int backward_run(unif_moe_layer* L, const void* x, const void* dy, int T, const 
     p.N = L->up_bn; p.n_nc = L->up_nsub; p.n_c = L->d / 128;
     p.status = w.status;
     p.wait_limit = gemm_wait_limit();
-    bwd_wgrad_kernel<<<L->n_sm, kThreads, L->bwd_wgrad_smem, s>>>(L->tm_da64, L->tm_hw64, p);
+    bwd_wgrad_kernel<<<L->n_sm, kThreads, L->bwd_wgrad_smem, s>>>(L->tm_da_q, L->tm_hw_q, p);
     CKB(cudaGetLastError());
   }
-  // router: dL/dz, its share of dL/dx, dL/dW*, dL/dbias
-  const int adaptive = isnan(L->th.alpha_fixed) ? 1 : 0;
-  router_grad_kernel<<<(T * 32 + 255) / 256, 256, 0, s>>>(
-      T, L->K, L->router_cols_pad, L->d, L->tau, adaptive, mask, w.alpha, w.s, w.dwt, L->wr, w.dz,
-      dx);
+  // router: W*^T, dL/dz, its share of dL/dx, dL/dW*, dL/dbias
+  router_transpose_kernel<<<(K1 * L->d + 255) / 256, 256, 0, s>>>(K1, L->d, L->router_cols_pad,
+                                                                   L->wr, w.wrT);
   CKB(cudaGetLastError());
-  router_wgrad_kernel<<<dim3((L->d + 255) / 256, (T + kRgTokens - 1) / kRgTokens), 256,
-                        sizeof(float) * kRgTokens * K1, s>>>(
+  const int adaptive = isnan(L->th.alpha_fixed) ? 1 : 0;
+  router_grad_kernel<<<(T * 32 + 255) / 256, 256, 0, s>>>(T, L->K, L->d, L->tau, adaptive, mask,
+                                                         w.alpha, w.s, w.dwt, w.wrT, w.dz, dx);
+  CKB(cudaGetLastError());
+  router_wgrad_kernel<<<dim3((L->d + 31) / 32, kRgSlices), 256, 0, s>>>(
       T, K1, L->d, mask, static_cast<const __nv_bfloat16*>(x), w.dz, dw_router, dbias);
   CKB(cudaGetLastError());
   if (lambda_div != 0.f || l_div) {
-    diversity_kernel<<<1, 256, sizeof(float) * (K1 * K1 + 8), s>>>(
-        K1, L->d, L->router_cols_pad, L->wr, lambda_div, dw_router, l_div);
+    gram_kernel<<<K1 * K1, 128, 0, s>>>(K1, L->d, w.wrT, w.gram);
+    CKB(cudaGetLastError());
+    diversity_grad_kernel<<<(L->d * K1 + 255) / 256, 256, 0, s>>>(K1, L->d, w.wrT, w.gram,
+                                                                  lambda_div, dw_router, l_div);
     CKB(cudaGetLastError());
   }
 #undef CKB

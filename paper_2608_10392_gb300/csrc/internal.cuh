@@ -89,6 +89,8 @@ struct Workspace {
   void* hw = nullptr;            // [max_rows][M] w GeLU(a) per group row
   float* dwt = nullptr;          // [max_tokens][K+1] dL/dalpha, dL/ds_j per token
   float* dz = nullptr;           // [max_tokens][K+1] dL/dz (router logits)
+  float* wrT = nullptr;          // [K+1][d] the router's W* transposed (fp32)
+  float* gram = nullptr;         // [K+1][K+1] W*^T W* - I
 };
 
 }  // namespace unif
@@ -150,8 +152,8 @@ struct unif_moe_layer {
   CUtensorMap tm_wdownT;    // w_downT [(K+1) H][d], boxes of 64 x up_bn
   CUtensorMap tm_wupT;      // w_upT [(K+1) d][H], boxes of 64 x down_bn
   CUtensorMap tm_da;        // da [max_rows][M], boxes of 64 x 128 (dx GEMM A operand)
-  CUtensorMap tm_da64;      // da, boxes of 64 x 64 (weight-gradient operand)
-  CUtensorMap tm_hw64;      // hw, boxes of 64 x 64
+  CUtensorMap tm_da_q;      // da, boxes of 64 x 32 (weight-gradient operand)
+  CUtensorMap tm_hw_q;      // hw, boxes of 64 x 32
   uint32_t bwd_hidden_smem = 0, bwd_wgrad_smem = 0;
   // Optional caller-owned timing events recorded at the stage boundaries.
   cudaEvent_t stage_ev[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};

@@ -71,7 +71,7 @@ void free_all(unif_moe_layer* L) {
                   L->ws.xn, L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
                   L->ws.k_stage, L->ws.status, L->ws.grp_fill,
                   L->ws.tile_rows, L->ws.w_upT, L->ws.w_downT, L->ws.da, L->ws.hw,
-                  L->ws.dwt, L->ws.dz};
+                  L->ws.dwt, L->ws.dz, L->ws.wrT, L->ws.gram};
   for (void* q : ptrs)
     if (q) cudaFree(q);
 }
@@ -255,6 +255,7 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
     if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.da), es * (size_t)L->max_rows * M);
     if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.hw), es * (size_t)L->max_rows * M);
     ALLOC(w.dwt, T * E); ALLOC(w.dz, T * E);
+    ALLOC(w.wrT, E * d_model); ALLOC(w.gram, E * E);
   }
 #undef ALLOC
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
