@@ -66,7 +66,6 @@ constexpr int kThreads = 416;     // 13 warps
 constexpr int kMmaWarp = 4;
 constexpr int kFirstEpiWarp = 5;  // warps 5-12
 constexpr int kEpiWarps = 8;
-constexpr int kStages = 2;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAcc2 = 256;   // TMEM column of the second accumulator
 
@@ -74,10 +73,12 @@ constexpr uint32_t kAcc2 = 256;   // TMEM column of the second accumulator
 // bwd_hidden_kernel: per (tile, N sub-tile) item, over the forward's tile
 // list, acc_a = X[rows] K_e[cols]^T and acc_g = DY[rows] V_e^T[cols]^T (both
 // reductions over d), then the epilogue of the header comment.
-// Roles: warps 0-3 fill the 2-deep stage ring (warp 2s gathers the x rows of
-// stage s and brings both weight tiles by TMA, warp 2s+1 gathers the dy
-// rows); warp 4 allocates TMEM and issues the MMAs; warps 5-12 run the
-// epilogue (warp w reads TMEM lane quarter w % 4, one half of the columns).
+// Roles: warps 0-3 fill a 4-deep ring of single-operand stages (even
+// stages: 128 gathered x rows and the key tile; odd stages: dy rows and the
+// value tile, so that each 64-deep k-block takes one stage of each; warp s
+// owns stage s and its lane 0 brings the stage's weight tile by TMA); warp 4
+// allocates TMEM and issues the MMAs; warps 5-12 run the epilogue (warp w
+// reads TMEM lane quarter w % 4, one half of the columns).
 // ---------------------------------------------------------------------------
 struct HiddenParams {
   const int32_t* n_tiles;
@@ -96,8 +97,10 @@ struct HiddenParams {
   long long wait_limit;
 };
 
+constexpr int kHStages = 4;
+
 __host__ __device__ constexpr uint32_t hidden_stage_bytes(int bn) {
-  return 2u * kStageA + 2u * (uint32_t)bn * kBK * 2u;
+  return kStageA + (uint32_t)bn * kBK * 2u;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -108,24 +111,22 @@ bwd_hidden_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_consta
   const uint32_t stage_bytes = hidden_stage_bytes(p.bn);
   const uint32_t wtile = (uint32_t)p.bn * kBK * 2u;
   const uint32_t s0 = smem_u32(smem);
-  // stage s: [x rows 16 KB][dy rows 16 KB][K tile][V tile]
-  auto sx = [&](int s) { return s0 + s * stage_bytes; };
-  auto sdy = [&](int s) { return s0 + s * stage_bytes + kStageA; };
-  auto swk = [&](int s) { return s0 + s * stage_bytes + 2 * kStageA; };
-  auto swv = [&](int s) { return s0 + s * stage_bytes + 2 * kStageA + wtile; };
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * stage_bytes);
+  // stage s: [128 rows x 64 (16 KB)][weight tile bn x 64]
+  auto sa = [&](int s) { return s0 + s * stage_bytes; };
+  auto sw = [&](int s) { return s0 + s * stage_bytes + kStageA; };
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kHStages * stage_bytes);
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
-  const uint32_t accf = bar0 + 8u * (2 * kStages);
-  const uint32_t acce = bar0 + 8u * (2 * kStages + 1);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 2);
+  auto empty_bar = [&](int s) { return bar0 + 8u * (kHStages + s); };
+  const uint32_t accf = bar0 + 8u * (2 * kHStages);
+  const uint32_t acce = bar0 + 8u * (2 * kHStages + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kHStages + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(full_bar(s), 2);  // the x warp and the dy warp of the stage
+    for (int s = 0; s < kHStages; ++s) {
+      mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
     mbar_init(accf, 1);
@@ -144,11 +145,12 @@ bwd_hidden_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_consta
   const uint32_t tmem_base = *tmem_slot;
   const int n_items = p.n_tiles[0] * p.n_sub;
 
-  if (warp < 4) {
-    // ---- producers: warp 2s + kind owns stage s (kind 0: x rows and the
-    // weight tiles, kind 1: dy rows) ----
-    const int my_stage = warp >> 1, kind = warp & 1;
+  if (warp < kHStages) {
+    // ---- producers: warp s owns stage s (s even: x rows and key tiles, s
+    // odd: dy rows and value tiles) ----
+    const int my_stage = warp, kind = warp & 1;
     const __nv_bfloat16* src = kind == 0 ? p.x : p.dy;
+    const CUtensorMap* tmw = kind == 0 ? &tm_wk : &tm_wv;
     const int j = lane & 7, rsub = lane >> 3;
     bool ok = true;
     int seq = 0;
@@ -165,18 +167,19 @@ bwd_hidden_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_consta
         const int t = 32 * i + lane < nrow ? p.row_tok[r0 + 32 * i + lane] : 0;
         tk[i] = t < 0 ? 0 : t;
       }
-      for (int kb = 0; kb < p.num_kb; ++kb, ++seq) {
-        const int stage = seq % kStages;
+      // stage sequence: seq = 2 kb + kind over the item's k-blocks
+      for (int ks = 0; ks < 2 * p.num_kb; ++ks, ++seq) {
+        const int stage = seq % kHStages;
         if (stage != my_stage) continue;
-        const uint32_t phase = (uint32_t)(seq / kStages) & 1u;
+        const int kb = ks >> 1;
+        const uint32_t phase = (uint32_t)(seq / kHStages) & 1u;
         ok = wait_warp(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
         if (!ok) break;
-        if (kind == 0 && lane == 0) {
-          mbar_expect_tx_only(full_bar(stage), 2u * wtile);
-          tma_load_2d(swk(stage), &tm_wk, full_bar(stage), kb * kBK, brow);
-          tma_load_2d(swv(stage), &tm_wv, full_bar(stage), kb * kBK, brow);
+        if (lane == 0) {
+          mbar_expect_tx_only(full_bar(stage), wtile);
+          tma_load_2d(sw(stage), tmw, full_bar(stage), kb * kBK, brow);
         }
-        const uint32_t dst = kind == 0 ? sx(stage) : sdy(stage);
+        const uint32_t dst = sa(stage);
         const __nv_bfloat16* sj = src + j * 8 + kb * kBK;
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
@@ -201,21 +204,19 @@ bwd_hidden_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_consta
       ok = wait_warp(acce, acc_phase ^ 1u, abort_flag, p.status, p.wait_limit);
       if (!ok) break;
       tc_fence_after();
-      for (int kb = 0; kb < p.num_kb; ++kb, ++seq) {
-        const int stage = seq % kStages;
-        const uint32_t phase = (uint32_t)(seq / kStages) & 1u;
+      for (int ks = 0; ks < 2 * p.num_kb; ++ks, ++seq) {
+        const int stage = seq % kHStages;
+        const uint32_t phase = (uint32_t)(seq / kHStages) & 1u;
         ok = wait_warp(full_bar(stage), phase, abort_flag, p.status, p.wait_limit);
         if (!ok) break;
         tc_fence_after();
+        // even stages feed x K (acc_a), odd ones dy V^T (acc_g)
+        const uint32_t d_tmem = tmem_base + ((ks & 1) ? kAcc2 : 0u);
         if (elect_one()) {
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k) {
-            const uint32_t acc = (kb | k) != 0 ? 1u : 0u;
-            umma_bf16(tmem_base, sw128_desc(sx(stage) + k * 32), sw128_desc(swk(stage) + k * 32),
-                      idesc, acc);
-            umma_bf16(tmem_base + kAcc2, sw128_desc(sdy(stage) + k * 32),
-                      sw128_desc(swv(stage) + k * 32), idesc, acc);
-          }
+          for (int k = 0; k < kBK / 16; ++k)
+            umma_bf16(d_tmem, sw128_desc(sa(stage) + k * 32), sw128_desc(sw(stage) + k * 32),
+                      idesc, ((ks >> 1) | k) != 0 ? 1u : 0u);
           umma_commit(empty_bar(stage));
         }
         __syncwarp();
@@ -300,8 +301,9 @@ bwd_hidden_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_consta
 //   acc2[i][h] = sum_r DY[tok_r][c*128 + i] HW[r][nc*N + h]  -> dV_e
 // The token rows are the reduction dimension, so both operands are MN-major:
 // the gathered rows (x, dy) and the TMA tiles (DA, HW) keep the 128-byte
-// swizzled row layout, read with MN-major descriptors. Each item owns its
-// output exactly (no atomics); groups without rows give zeros.
+// swizzled row layout, read with MN-major descriptors. A group's rows are
+// split into chunks of kChunkTiles tiles, one work item each, whose partial
+// sums are added into the (zeroed) outputs.
 // Roles: warps 0-3 fill the 4-deep ring (warp s: the x and dy rows of stage
 // s, and the DA/HW tiles by TMA), warp 4 MMAs, warps 5-12 epilogue.
 // ---------------------------------------------------------------------------
@@ -321,6 +323,7 @@ constexpr uint32_t kRows = 32;                 // group rows per stage
 constexpr uint32_t kPBytes = 2u * kRows * 128u;  // 128 features x 32 rows (two 64-column blocks)
 constexpr int kWStages = 4;                      // one stage per producer warp
 constexpr int kQuarters = kBM / (int)kRows;      // stages per 128-row tile
+constexpr int kChunkTiles = 8;                   // tiles of a group per work item
 
 __host__ __device__ constexpr uint32_t wgrad_stage_bytes(int N) {
   return 2u * kPBytes + 2u * (uint32_t)(N / 64) * kRows * 128u;
@@ -350,6 +353,7 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int32_t* first_s = reinterpret_cast<int32_t*>(tmem_slot + 4);  // [G + 1] first tiles
   int32_t* cnt_s = first_s + p.G + 1;                             // [G] sizes
+  int32_t* chunk_s = cnt_s + p.G;                                 // [G + 1] first chunks
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -366,18 +370,47 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
   }
-  if (warp == kThreads / 32 - 1) tile_table(p.counts, p.G, p.region, lane, first_s, cnt_s);
+  if (warp == kThreads / 32 - 1) {
+    tile_table(p.counts, p.G, p.region, lane, first_s, cnt_s);
+    __syncwarp();
+    // each group's tiles in chunks of kChunkTiles: the first chunk of every
+    // group (chunk_s[G] = all chunks)
+    int carry = 0;
+    for (int g0 = 0; g0 < p.G; g0 += 32) {
+      const int g = g0 + lane;
+      const int nch = g < p.G ? (first_s[g + 1] - first_s[g] + kChunkTiles - 1) / kChunkTiles : 0;
+      int inc = nch;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += v;
+      }
+      if (g < p.G) chunk_s[g] = carry + inc - nch;
+      carry += __shfl_sync(0xffffffffu, inc, 31);
+    }
+    if (lane == 0) chunk_s[p.G] = carry;
+  }
   __syncwarp();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int n_items = p.G * p.n_c * p.n_nc;
-  // item -> (group, feature chunk, N chunk); tiles of the group: first_s
-  auto decode = [&](int item, int& g, int& c, int& nc) {
+  const int n_items = chunk_s[p.G] * p.n_c * p.n_nc;
+  // item -> (group g, its tiles [t0, t0 + nt) of one chunk, feature chunk c,
+  // N chunk nc); rows of the chunk start at row r0 of the group
+  auto decode = [&](int item, int& g, int& t0, int& nt, int& r0, int& c, int& nc) {
     nc = item % p.n_nc;
     c = (item / p.n_nc) % p.n_c;
-    g = item / (p.n_nc * p.n_c);
+    const int q = item / (p.n_nc * p.n_c);
+    int lo = 0, hi = p.G - 1;  // the last group whose first chunk is <= q
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (chunk_s[mid] <= q) lo = mid; else hi = mid - 1;
+    }
+    g = lo;
+    const int k = q - chunk_s[g];
+    t0 = first_s[g] + k * kChunkTiles;
+    nt = min(kChunkTiles, first_s[g + 1] - t0);
+    r0 = k * kChunkTiles * kBM;
   };
 
   if (warp < kWStages) {
@@ -388,9 +421,8 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
     bool ok = true;
     int seq = 0;
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-      int g, c, nc;
-      decode(item, g, c, nc);
-      const int t_first = first_s[g], nt = first_s[g + 1] - t_first;
+      int g, t_first, nt, r0, c, nc;
+      decode(item, g, t_first, nt, r0, c, nc);
       const int size = cnt_s[g];
       for (int kt = 0; kt < nt * kQuarters && ok; ++kt, ++seq) {  // 32-row quarters of the tiles
         const int stage = seq % kWStages;
@@ -398,7 +430,7 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
         const uint32_t phase = (uint32_t)(seq / kWStages) & 1u;
         ok = wait_warp(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit);
         if (!ok) break;
-        const int row_in_group = kt * (int)kRows;  // first row of this quarter in the group
+        const int row_in_group = r0 + kt * (int)kRows;  // first row of this quarter in the group
         const int crow = (t_first + kt / kQuarters) * kBM + (kt % kQuarters) * (int)kRows;
         if (lane == 0) {
           mbar_expect_tx_only(full_bar(stage), 2u * qbytes);
@@ -444,10 +476,8 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
     uint32_t acc_phase = 0;
     bool ok = true;
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-      int g, c, nc;
-      decode(item, g, c, nc);
-      const int nt = first_s[g + 1] - first_s[g];
-      if (nt == 0) continue;  // no rows: the epilogue writes zeros
+      int g, t_first, nt, r0, c, nc;
+      decode(item, g, t_first, nt, r0, c, nc);
       ok = wait_warp(acce, acc_phase ^ 1u, abort_flag, p.status, p.wait_limit);
       if (!ok) break;
       tc_fence_after();
@@ -481,33 +511,27 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
     const int cols = p.N / 2;
     uint32_t acc_phase = 0;
     for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
-      int g, c, nc;
-      decode(item, g, c, nc);
+      int g, t_first, nt, r0, c, nc;
+      decode(item, g, t_first, nt, r0, c, nc);
       const int e = g / p.B, blk = g % p.B;
-      const int nt = first_s[g + 1] - first_s[g];
       const int i = c * 128 + q * 32 + lane;  // this thread's feature
       const int h0 = blk * p.M + nc * p.N + half * cols;  // first channel of its columns
       float* up_col = p.dw_up + ((size_t)e * p.H + h0) * p.d + i;   // dK_e[h][i], stride d per h
       float* dn_row = p.dw_down + ((size_t)e * p.d + i) * p.H + h0;  // dV_e[i][h], contiguous
-      if (nt == 0) {
-        for (int cc = 0; cc < cols; ++cc) {
-          up_col[(size_t)cc * p.d] = 0.f;
-          dn_row[cc] = 0.f;
-        }
-        continue;
-      }
       if (!wait_warp(accf, acc_phase, abort_flag, p.status, p.wait_limit)) break;
       tc_fence_after();
       const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + half * cols;
+      // the chunks of a group add their partial sums (the outputs start at zero)
       for (int cc = 0; cc < cols; cc += 32) {
         float v[32];
         tmem_ld32(t_row + cc, v);
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) up_col[(size_t)(cc + jj) * p.d] = v[jj];
+        for (int jj = 0; jj < 32; ++jj) atomicAdd(up_col + (size_t)(cc + jj) * p.d, v[jj]);
         tmem_ld32(t_row + kAcc2 + cc, v);
 #pragma unroll
         for (int jj = 0; jj < 32; jj += 4)
-          *reinterpret_cast<float4*>(dn_row + cc + jj) = make_float4(v[jj], v[jj + 1], v[jj + 2], v[jj + 3]);
+          atomicAdd(reinterpret_cast<float4*>(dn_row + cc + jj),
+                    make_float4(v[jj], v[jj + 1], v[jj + 2], v[jj + 3]));
       }
       tc_fence_before();
       __syncwarp();
@@ -724,9 +748,9 @@ int backward_setup(unif_moe_layer* L) {
     set_error("cuTensorMapEncodeTiled failed for the backward maps");
     return UNIF_MOE_ERR_CUDA;
   }
-  L->bwd_hidden_smem = 1024 + kStages * hidden_stage_bytes(L->up_bn) + 256;
+  L->bwd_hidden_smem = 1024 + kHStages * hidden_stage_bytes(L->up_bn) + 256;
   L->bwd_wgrad_smem =
-      1024 + kWStages * wgrad_stage_bytes(L->up_bn) + 96 + 4 * (2 * (uint32_t)L->G + 1) + 16;
+      1024 + kWStages * wgrad_stage_bytes(L->up_bn) + 96 + 4 * (3 * (uint32_t)L->G + 2) + 16;
   if (L->bwd_hidden_smem > 232448 || L->bwd_wgrad_smem > 232448) {
     set_error("backward: shared memory for block width %d and %d groups exceeds 227 KB", L->M,
               L->G);
@@ -795,7 +819,9 @@ int backward_run(unif_moe_layer* L, const void* x, const void* dy, int T, const 
   }
   // dL/dx from the experts: DA K_e (the down kernel on the transposed keys)
   CKB(launch_down_streaming(L, L->tm_da, L->tm_wupT, nullptr, dx, s));
-  // dL/dK_e and dL/dV_e
+  // dL/dK_e and dL/dV_e (chunks of each group's rows add their parts)
+  CKB(cudaMemsetAsync(dw_up, 0, sizeof(float) * (size_t)K1 * L->H * L->d, s));
+  CKB(cudaMemsetAsync(dw_down, 0, sizeof(float) * (size_t)K1 * L->H * L->d, s));
   {
     WgradParams p;
     p.counts = w.grp_cnt; p.row_tok = w.row_tok;
