@@ -557,15 +557,15 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
 // dL/dz W*^T, with W*^T the router's first K+1 columns transposed (fp32
 // [K+1][d], so that the lanes read consecutive features). Lane l keeps
 // dL/dz_c for c = l, l + 32, l + 64 in registers.
-__global__ void __launch_bounds__(256)
-router_grad_kernel(int T, int K, int d, float tau, int adaptive,
-                   const uint8_t* __restrict__ mask, const float* __restrict__ alpha,
-                   const float* __restrict__ s, const float* __restrict__ dwt,
-                   const float* __restrict__ wrT, float* __restrict__ dz,
-                   float* __restrict__ dx) {
-  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (warp >= T) return;
-  const int t = warp;
+// dL/dz of token t and its share of dL/dx (one warp, `lane` its lane).
+__device__ __forceinline__ void router_grad_token(int t, int K, int d, float tau, int adaptive,
+                                                  const uint8_t* __restrict__ mask,
+                                                  const float* __restrict__ alpha,
+                                                  const float* __restrict__ s,
+                                                  const float* __restrict__ dwt,
+                                                  const float* __restrict__ wrT,
+                                                  float* __restrict__ dz,
+                                                  float* __restrict__ dx, int lane) {
   const int K1 = K + 1;
   float* dzt = dz + (size_t)t * K1;
   if (mask && !mask[t]) {
@@ -606,6 +606,28 @@ router_grad_kernel(int T, int K, int d, float tau, int adaptive,
   }
 }
 
+
+// The block's warps take tokens in turn; W*^T is staged in shared memory
+// when it fits (wrT_smem), else read from global memory.
+__global__ void __launch_bounds__(256)
+router_grad_kernel(int T, int K, int d, float tau, int adaptive,
+                   const uint8_t* __restrict__ mask, const float* __restrict__ alpha,
+                   const float* __restrict__ s, const float* __restrict__ dwt,
+                   const float* __restrict__ wrT_g, float* __restrict__ dz,
+                   float* __restrict__ dx, int wrT_smem) {
+  extern __shared__ float wrT_s[];
+  const int K1 = K + 1;
+  if (wrT_smem) {
+    for (int k = threadIdx.x; k < K1 * d; k += blockDim.x) wrT_s[k] = wrT_g[k];
+    __syncthreads();
+  }
+  const float* wrT = wrT_smem ? wrT_s : wrT_g;
+  const int lane = threadIdx.x & 31;
+  const int warps = gridDim.x * (blockDim.x >> 5);
+  for (int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); t < T; t += warps)
+    router_grad_token(t, K, d, tau, adaptive, mask, alpha, s, dwt, wrT, dz, dx, lane);
+}
+
 // W*^T: the router's first K+1 columns (fp32 [d][Cp]) as [K+1][d].
 __global__ void router_transpose_kernel(int K1, int d, int Cp, const float* __restrict__ wr,
                                         float* __restrict__ wrT) {
@@ -620,7 +642,7 @@ __global__ void router_transpose_kernel(int K1, int d, int Cp, const float* __re
 // block (32 features x 8 token lanes) of one token slice; the 8 lanes'
 // partial sums are added in shared memory, then once per block into the
 // outputs (which start at zero).
-constexpr int kRgSlices = 16;
+constexpr int kRgSlices = 128;
 __global__ void __launch_bounds__(256)
 router_wgrad_kernel(int T, int K1, int d, const uint8_t* __restrict__ mask,
                     const __nv_bfloat16* __restrict__ x, const float* __restrict__ dz,
@@ -840,8 +862,11 @@ int backward_run(unif_moe_layer* L, const void* x, const void* dy, int T, const 
                                                                    L->wr, w.wrT);
   CKB(cudaGetLastError());
   const int adaptive = isnan(L->th.alpha_fixed) ? 1 : 0;
-  router_grad_kernel<<<(T * 32 + 255) / 256, 256, 0, s>>>(T, L->K, L->d, L->tau, adaptive, mask,
-                                                         w.alpha, w.s, w.dwt, w.wrT, w.dz, dx);
+  const size_t wrT_bytes = sizeof(float) * (size_t)K1 * L->d;
+  const int wrT_smem = wrT_bytes <= 48 * 1024 ? 1 : 0;
+  const int rg_blocks = min((T + 7) / 8, L->n_sm * 8);
+  router_grad_kernel<<<rg_blocks, 256, wrT_smem ? wrT_bytes : 0, s>>>(
+      T, L->K, L->d, L->tau, adaptive, mask, w.alpha, w.s, w.dwt, w.wrT, w.dz, dx, wrT_smem);
   CKB(cudaGetLastError());
   router_wgrad_kernel<<<dim3((L->d + 31) / 32, kRgSlices), 256, 0, s>>>(
       T, K1, L->d, mask, static_cast<const __nv_bfloat16*>(x), w.dz, dw_router, dbias);
