@@ -124,7 +124,7 @@ def measured_traffic(workload, kernel):
     rec = json.load(open(path)).get(workload, {})
     csrc = os.path.join(ROOT, "paper_2608_10392_gb300", "csrc")
     h = hashlib.sha1()
-    for f in ("gemm_ws.cu", "tc_common.cuh"):
+    for f in rec.get("sources", []):
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(fh.read())
     if rec.get("kernel_source_sha1") != h.hexdigest():
