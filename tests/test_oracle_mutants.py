@@ -104,15 +104,27 @@ MUTANTS = {
     "gram_no_identity": ("A[a * K1 + b] = g - (a == b ? 1.0 : 0.0);", "A[a * K1 + b] = g;"),
 }
 
-# Mistakes planted in the Python side of the oracle (oracle/__init__.py).
+# Mistakes planted in the Python side of the oracle: (file, old, new).
 PY_MUTANTS = {
     # given experts listed by increasing affinity
-    "with_decisions_ascending": ("sel.sort(key=lambda j: (-r.s[t, j], j))",
+    "with_decisions_ascending": ("__init__.py", "sel.sort(key=lambda j: (-r.s[t, j], j))",
                                  "sel.sort(key=lambda j: (r.s[t, j], j))"),
     # the unselected experts placed first, so the first k are the wrong ones
-    "with_decisions_rest_first": ("order = sel + rest", "order = rest + sel"),
+    "with_decisions_rest_first": ("__init__.py", "order = sel + rest", "order = rest + sel"),
     # affinities left in expert order instead of following q
-    "with_decisions_p_unsorted": ("p[t] = r.s[t, order]", "p[t] = r.s[t]"),
+    "with_decisions_p_unsorted": ("__init__.py", "p[t] = r.s[t, order]", "p[t] = r.s[t]"),
+    # the shared set with a strict threshold
+    "diag_strict_threshold": ("diagnostics.py", "S[i, j] = c >= delta", "S[i, j] = c > delta"),
+    # residual order by increasing score
+    "diag_order_ascending": ("diagnostics.py", "np.argsort(-(xa @ _f64(w_res))",
+                             "np.argsort((xa @ _f64(w_res))"),
+    # residual outputs taken from the shared positions
+    "diag_residual_rows": ("diagnostics.py", "ER = E - ES", "ER = ES"),
+    # error relative to the residual target instead of the original output
+    "diag_error_scale": ("diagnostics.py", "ynorm = max(np.linalg.norm(y[t]), 1e-12)",
+                         "ynorm = max(np.linalg.norm(r[t]), 1e-12)"),
+    # ridge weight without the 1/m
+    "diag_gamma_scale": ("diagnostics.py", "1e-6 * tr / m * np.eye(m)", "1e-6 * tr * np.eye(m)"),
 }
 
 
@@ -133,14 +145,16 @@ def test_pins_catch_mutant(name, tmp_path):
     assert res.returncode != 0, "no pin caught mutant %s:\n%s" % (name, res.stdout[-2000:])
 
 
-def run_pins_in_copy(tmp_path, old, new):
+def run_pins_in_copy(tmp_path, fname, old, new):
     """Runs the pins in a tree of their own holding a copy of the oracle
-    package whose Python source has `old` replaced by `new`."""
-    src = open(os.path.join(ROOT, "oracle", "__init__.py")).read()
-    assert src.count(old) == 1, "mutation anchor not found: " + old
+    package whose Python file `fname` has `old` replaced by `new`."""
     (tmp_path / "oracle").mkdir()
-    (tmp_path / "oracle" / "__init__.py").write_text(src.replace(old, new))
-    shutil.copy(SRC, tmp_path / "oracle" / "unif_moe_oracle.c")
+    for f in os.listdir(os.path.join(ROOT, "oracle")):
+        if f.endswith((".py", ".c")):
+            shutil.copy(os.path.join(ROOT, "oracle", f), tmp_path / "oracle" / f)
+    src = open(os.path.join(ROOT, "oracle", fname)).read()
+    assert src.count(old) == 1, "mutation anchor not found: " + old
+    (tmp_path / "oracle" / fname).write_text(src.replace(old, new))
     (tmp_path / "tests").mkdir()
     for f in ("conftest.py", "test_oracle_pins.py"):
         shutil.copy(os.path.join(ROOT, "tests", f), tmp_path / "tests" / f)
@@ -155,7 +169,7 @@ def run_pins_in_copy(tmp_path, old, new):
 def test_unmutated_copy_passes(tmp_path):
     """Control for the Python mutants: the copied tree itself passes, so a
     mutant's failure comes from its planted mistake."""
-    res = run_pins_in_copy(tmp_path, "order = sel + rest", "order = sel + rest")
+    res = run_pins_in_copy(tmp_path, "__init__.py", "order = sel + rest", "order = sel + rest")
     assert res.returncode == 0, res.stdout[-2000:]
 
 
@@ -163,6 +177,6 @@ def test_unmutated_copy_passes(tmp_path):
 def test_pins_catch_python_mutant(name, tmp_path):
     """The same check for the Python wrapper: a copy of the oracle package
     with one planted mistake, next to copies of the pins."""
-    old, new = PY_MUTANTS[name]
-    res = run_pins_in_copy(tmp_path, old, new)
+    fname, old, new = PY_MUTANTS[name]
+    res = run_pins_in_copy(tmp_path, fname, old, new)
     assert res.returncode != 0, "no pin caught mutant %s:\n%s" % (name, res.stdout[-2000:])

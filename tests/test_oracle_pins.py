@@ -757,3 +757,127 @@ def test_diversity_finite_differences(oracle_mod):
     assert L == pytest.approx(G, rel=1e-13)
     num, = central_differences(lambda: oracle.diversity(W)[0], [W])
     np.testing.assert_allclose(grad, num, rtol=1e-7, atol=1e-9)
+
+
+# --------------------------------------------------------------------------
+# Diagnostics of Sec. II-B: value alignment and functional demand
+# --------------------------------------------------------------------------
+
+def test_value_alignment_closed_forms(oracle_mod):
+    """Eq. shared-set on constructed value rows (d = 2): identical rows have
+    c = 1, opposite rows c = -1, rows (3, 4) and (4, 3) have c = 24/25
+    exactly (an exact cosine counts at delta = 0.96, the set uses >=), and a
+    zero row is aligned with nothing."""
+    from oracle import diagnostics as dg
+    d, H, K = 2, 8, 3
+    wd = np.zeros((K + 1, d, H))
+    v1 = np.array([[3.0, 4.0], [1.0, 0.0], [0.0, 2.0], [5.0, 1.0],
+                   [1.0, 1.0], [2.0, -1.0], [0.0, 0.0], [1.0, 3.0]])  # [H][d]
+    v2 = v1.copy()
+    v2[0] = [4.0, 3.0]          # c = 24/25
+    v2[1] = [-1.0, 0.0]         # c = -1
+    v2[2] = [0.0, 7.0]          # c = 1 (positive scale)
+    v2[3] = [-1.0, 5.0]         # orthogonal: c = 0
+    v3 = -v1                    # every row opposite
+    for e, v in ((1, v1), (2, v2), (3, v3)):
+        wd[e] = v.T
+    rho, S = dg.value_alignment(wd, 0.96)
+    # expert 1 vs 2: rows 0 (24/25), 2, 4, 5, 7 aligned; 1 (opposite), 3 (orthogonal), 6 (zero) not
+    assert S[0, 1].tolist() == [True, False, True, False, True, True, False, True]
+    assert rho[0, 1] == pytest.approx(5 / 8) and rho[1, 0] == pytest.approx(5 / 8)
+    assert rho[0, 2] == 0.0
+    assert rho[0, 0] == pytest.approx(7 / 8)  # every nonzero row with itself
+    _, S2 = dg.value_alignment(wd, 0.96 + 1e-12)
+    assert not S2[0, 1, 0] and S2[0, 1, 2]
+
+
+def test_expert_outputs_match_layer_oracle(oracle_mod):
+    """E_e(x) of the diagnostic equals the layer oracle's dense FFN of that
+    expert (alpha fixed at 1 with expert e as the shared one); E^S with every
+    channel is E, with none is 0."""
+    from oracle import diagnostics as dg
+    rng = np.random.default_rng(41)
+    T, d, H, K, B = 20, 8, 16, 3, 4
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, T=T)
+    E, ES = dg.expert_outputs(x, w_up, w_down, np.ones((T, H), bool))
+    _, ES0 = dg.expert_outputs(x, w_up, w_down, np.zeros((T, H), bool))
+    np.testing.assert_array_equal(ES, E)
+    assert (ES0 == 0).all()
+    for e in range(1, K + 1):
+        wu = w_up.copy()
+        wd = w_down.copy()
+        wu[0], wd[0] = w_up[e], w_down[e]
+        y, _ = oracle.layer(x, w_router, wu, wd, B, Thresholds(alpha_fixed=1.0))
+        np.testing.assert_allclose(E[:, e - 1], y, rtol=1e-12, atol=1e-13)
+
+
+def test_functional_demand_identical_experts(oracle_mod):
+    """Experts copied from one FFN align at every channel (rho = 1), so the
+    shared response is the whole output, r = 0 and k_eps = 1 for every token."""
+    from oracle import diagnostics as dg
+    rng = np.random.default_rng(42)
+    T, d, H, K, B = 16, 8, 16, 4, 4
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, router_scale=3.0, T=T)
+    w_up[:] = w_up[0]
+    w_down[:] = w_down[0]
+    rho, _ = dg.value_alignment(w_down, 0.98)
+    assert (rho == 1).all()
+    k, err, _ = dg.functional_demand(x, w_router, w_up, w_down, rng.standard_normal((d, K)),
+                                     0.98, 0.05)
+    assert (k == 1).all() and np.abs(err).max() < 1e-12
+
+
+def test_functional_demand_nothing_shared(oracle_mod):
+    """delta above 1 shares nothing: r = y_orig. With the residual order of
+    the original router the first two residual rows are E_i and E_j, which
+    span r: e_2 is the ridge's own (1e-6-relative) residual; e_1 is the
+    distance of r from the line of E_i, from the normal equations by hand."""
+    from oracle import diagnostics as dg
+    rng = np.random.default_rng(43)
+    T, d, H, K, B = 12, 10, 16, 4, 4
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, router_scale=3.0, T=T)
+    k, err, pair = dg.functional_demand(x, w_router, w_up, w_down, w_router[:, 1:], 2.0, 1e-3)
+    E, _ = dg.expert_outputs(x, w_up, w_down, np.zeros((T, H), bool))
+    i, j, ti, tj = dg.top2_pairs(x, w_router)
+    assert (pair[:, 0] == i).all() and (pair[:, 1] == j).all()
+    for t in range(T):
+        r = ti[t] * E[t, i[t]] + tj[t] * E[t, j[t]]
+        Ei = E[t, i[t]]
+        g = Ei @ Ei
+        a = (Ei @ r) / (g * (1 + 1e-6))
+        assert err[t, 0] == pytest.approx(np.linalg.norm(r - a * Ei) / np.linalg.norm(r),
+                                          rel=1e-9, abs=1e-12)
+        assert err[t, 1] < 1e-5
+    assert (k <= 2).all()
+    k0, _, _ = dg.functional_demand(x, w_router, w_up, w_down, w_router[:, 1:], 2.0, -1.0)
+    assert (k0 == K + 1).all()  # no prefix reaches a negative tolerance: the sentinel
+
+
+def test_functional_demand_ridge_by_augmented_least_squares(oracle_mod):
+    """Every e_m against the ridge solved another way: least squares on the
+    stacked system [R^T; sqrt(gamma) I] a = [r; 0] (scipy.linalg.lstsq)."""
+    import scipy.linalg
+    from oracle import diagnostics as dg
+    rng = np.random.default_rng(44)
+    T, d, H, K, B, delta = 10, 12, 32, 5, 4, 0.8
+    x, w_router, w_up, w_down = rand_layer(rng, d, H, K, B, router_scale=3.0, T=T)
+    w_down[2:] = w_down[1] + 0.8 * rng.standard_normal(w_down[2:].shape) / math.sqrt(H)
+    w_res = rng.standard_normal((d, K))
+    k, err, pair = dg.functional_demand(x, w_router, w_up, w_down, w_res, delta, 0.1)
+    _, S = dg.value_alignment(w_down, delta)
+    i, j, ti, tj = dg.top2_pairs(x, w_router)
+    E, ES = dg.expert_outputs(x, w_up, w_down, S[i, j])
+    q = np.argsort(-(x @ w_res), axis=1, kind="stable")
+    assert 0 < S[i, j].sum() < T * H  # some channels shared, some not
+    for t in range(T):
+        y = ti[t] * E[t, i[t]] + tj[t] * E[t, j[t]]
+        sb = ti[t] * ES[t, i[t]] + tj[t] * ES[t, j[t]]
+        for m in range(1, K + 1):
+            R = (E - ES)[t, q[t, :m]]
+            gam = 1e-6 * np.sum(R * R) / m
+            A = np.vstack([R.T, math.sqrt(gam) * np.eye(m)])
+            a = scipy.linalg.lstsq(A, np.concatenate([y - sb, np.zeros(m)]))[0]
+            want = np.linalg.norm(sb + a @ R - y) / np.linalg.norm(y)
+            assert err[t, m - 1] == pytest.approx(want, rel=1e-7, abs=1e-12)
+        hit = np.nonzero(err[t] <= 0.1)[0]
+        assert k[t] == (hit[0] + 1 if len(hit) else K + 1)
