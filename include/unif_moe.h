@@ -84,8 +84,11 @@ enum {
   UNIF_MOE_FEATURE_BACKWARD = 4,   /* unif_moe_backward: transposed copies of the
                                       expert weights and per-row gradient buffers
                                       (bf16 layers, d % 128 == 0) */
+  UNIF_MOE_FEATURE_DIAGNOSTICS = 8, /* unif_moe_value_alignment and
+                                      unif_moe_functional_demand: per-token
+                                      expert outputs, 2 * max_tokens * K * d fp32 */
   UNIF_MOE_FEATURES_DEFAULT = 3,   /* what unif_moe_create allocates */
-  UNIF_MOE_FEATURES_ALL = 7
+  UNIF_MOE_FEATURES_ALL = 15
 };
 /* Grouped GEMM kernels: the library picks the weight-stationary kernels
  * where a group's weight slice fits in shared memory, else the streaming
@@ -227,6 +230,38 @@ UNIF_MOE_API int unif_moe_backward(unif_moe_t h, const void* x_dev, const void* 
                                    float* dw_up_dev, float* dw_down_dev, float* dw_router_dev,
                                    float* dbias_dev, float lambda_div, float* l_div_dev,
                                    void* stream);
+
+/* Diagnostics of Sec. II-B, on the layer's K residual experts (experts 1..K
+ * of the loaded weights) and their router columns: analysis tools, not part
+ * of the forward. Handles created with UNIF_MOE_FEATURE_DIAGNOSTICS
+ * (ERR_STATE otherwise), after a weight load. fp32 arithmetic.
+ *
+ * Value alignment (Eq. shared-set): for experts i, j (0-based among the
+ * residual experts) and channel h, c_ijh = V_i[h,:] . V_j[h,:] /
+ * (|V_i[h,:]| |V_j[h,:]|) (0 for a zero row), S_ij(delta) = {h : c_ijh >=
+ * delta}; rho_dev [K][K] fp32 receives rho_ij = |S_ij| / H.
+ * Errors: ERR_ARG (NULL rho, delta not finite), ERR_STATE, ERR_CUDA. */
+UNIF_MOE_API int unif_moe_value_alignment(unif_moe_t h, float delta, float* rho_dev,
+                                          void* stream);
+
+/* Functional demand (Eqs. diagnostic-original .. functional-demand): for each
+ * token of x_dev [T][d] (layer dtype), its top-2 pair (i, j) of
+ * s = softmax(x W_g + bias) (the layer's router; ties to the lower index),
+ * s~ = s / (s_i + s_j), y_orig = sum_{e in {i,j}} s~_e E_e(x), S_bar = the
+ * same over the channels S_ij(delta), r = y_orig - S_bar, the residual order
+ * q of x W_r (w_res_dev [d][K], layer dtype: the residual router, e.g. one
+ * trained on the residual positions), R_m = E_{q_1..q_m} over the channels
+ * outside S_ij, the ridge fit a* = (R_m R_m^T + gamma_m I)^{-1} R_m r with
+ * gamma_m = 1e-6 tr(R_m R_m^T) / m (fp64; a = 0 when R_m = 0), and
+ *   e_m = |a*^T R_m - r| / max(|y_orig|, 1e-12),  k_eps = min{m : e_m <= eps}
+ * or the sentinel K + 1. Outputs (device): k_eps_dev [T] int32, err_dev
+ * [T][K] fp32 (e_1..e_K) or NULL, pair_dev [T][2] int32 (i, j) or NULL.
+ * Needs 2 <= K <= 32 (ERR_SHAPE) and T <= max_tokens (ERR_CAPACITY).
+ * Errors also ERR_ARG, ERR_STATE, ERR_CUDA. */
+UNIF_MOE_API int unif_moe_functional_demand(unif_moe_t h, const void* x_dev, int T,
+                                            const void* w_res_dev, float delta, float eps,
+                                            int32_t* k_eps_dev, float* err_dev,
+                                            int32_t* pair_dev, void* stream);
 
 /* Copies the decisions of the last forward (T tokens) to device buffers; any
  * pointer may be NULL:

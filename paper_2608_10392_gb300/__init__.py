@@ -20,7 +20,8 @@ from typing import Optional
 import torch
 
 __all__ = ["Layer", "lib", "UnifMoeError", "ERR", "EXPORTS", "Options", "FEATURE_NORM_FIRST",
-           "FEATURE_HOST_IO", "FEATURE_BACKWARD", "FEATURES_DEFAULT", "FEATURES_ALL"]
+           "FEATURE_HOST_IO", "FEATURE_BACKWARD", "FEATURE_DIAGNOSTICS", "FEATURES_DEFAULT",
+           "FEATURES_ALL"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "lib", "libunif_moe.so")
@@ -32,7 +33,7 @@ ERR = {0: "OK", -1: "ERR_ARG", -2: "ERR_SHAPE", -3: "ERR_CAPACITY", -4: "ERR_CUD
 EXPORTS = ["unif_moe_default_thresholds", "unif_moe_default_options", "unif_moe_create",
            "unif_moe_create_ex", "unif_moe_load_weights",
            "unif_moe_load_upcycled", "unif_moe_forward", "unif_moe_sublayer_forward",
-           "unif_moe_backward",
+           "unif_moe_backward", "unif_moe_value_alignment", "unif_moe_functional_demand",
            "unif_moe_forward_host", "unif_moe_get_routing",
            "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_pass_tokens",
            "unif_moe_kernels_per_forward",
@@ -56,8 +57,8 @@ class Options(C.Structure):
     _fields_ = [("features", C.c_uint), ("gemm_kernels", C.c_int)]
 
 
-FEATURE_NORM_FIRST, FEATURE_HOST_IO, FEATURE_BACKWARD = 1, 2, 4
-FEATURES_DEFAULT, FEATURES_ALL = 3, 7
+FEATURE_NORM_FIRST, FEATURE_HOST_IO, FEATURE_BACKWARD, FEATURE_DIAGNOSTICS = 1, 2, 4, 8
+FEATURES_DEFAULT, FEATURES_ALL = 3, 15
 GEMM_KERNELS = {"auto": 0, "streaming": 1}
 
 
@@ -84,6 +85,8 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_load_upcycled.argtypes = [P, P, P, P, P, P]
         L.unif_moe_sublayer_forward.argtypes = [P, P, P, I, P, P, P, P, P, C.c_float, I, P]
         L.unif_moe_backward.argtypes = [P, P, P, I, P, P, P, P, P, P, C.c_float, P, P]
+        L.unif_moe_value_alignment.argtypes = [P, C.c_float, P, P]
+        L.unif_moe_functional_demand.argtypes = [P, P, I, P, C.c_float, C.c_float, P, P, P, P]
         L.unif_moe_forward_host.argtypes = [P, P, P, I, P, P, P, P]
         L.unif_moe_get_routing.argtypes = [P, P, P, P, P, P, P]
         L.unif_moe_get_groups.argtypes = [P, P, P, P, P, C.POINTER(C.c_int64), P]
@@ -232,6 +235,26 @@ class Layer:
                                        _ptr(g["dw_router"]), _ptr(g["dbias"]),
                                        float(lambda_div), _ptr(g["l_div"]), _stream(stream)))
         return g
+
+    def value_alignment(self, delta: float, stream=None) -> torch.Tensor:
+        """rho [K][K] of the residual experts (Sec. II-B, Eq. shared-set)."""
+        rho = torch.empty(self.K, self.K, dtype=torch.float32, device=torch.device("cuda"))
+        _check(lib().unif_moe_value_alignment(self._h, float(delta), _ptr(rho), _stream(stream)))
+        return rho
+
+    def functional_demand(self, x: torch.Tensor, w_res: torch.Tensor, delta: float, eps: float,
+                          stream=None) -> dict:
+        """k_eps [T], e [T][K] and the top-2 pair [T][2] of every token (Sec.
+        II-B); w_res [d][K] the residual router (layer dtype)."""
+        T = x.shape[0]
+        dev = x.device
+        out = dict(k_eps=torch.empty(T, dtype=torch.int32, device=dev),
+                   err=torch.empty(T, self.K, dtype=torch.float32, device=dev),
+                   pair=torch.empty(T, 2, dtype=torch.int32, device=dev))
+        _check(lib().unif_moe_functional_demand(self._h, _ptr(x), T, _ptr(w_res), float(delta),
+                                                float(eps), _ptr(out["k_eps"]), _ptr(out["err"]),
+                                                _ptr(out["pair"]), _stream(stream)))
+        return out
 
     def forward_host(self, x_host: torch.Tensor, out_host: torch.Tensor,
                      mask_host: Optional[torch.Tensor] = None,

@@ -91,6 +91,14 @@ struct Workspace {
   float* dz = nullptr;           // [max_tokens][K+1] dL/dz (router logits)
   float* wrT = nullptr;          // [K+1][d] the router's W* transposed (fp32)
   float* gram = nullptr;         // [K+1][K+1] W*^T W* - I
+  // Diagnostics of Sec. II-B (UNIF_MOE_FEATURE_DIAGNOSTICS).
+  uint32_t* diag_sets = nullptr; // [K][K][ceil(H/32)] aligned channel sets S_ij
+  int* diag_counts = nullptr;    // [K][K] |S_ij|
+  int32_t* diag_pair = nullptr;  // [max_tokens][2] top-2 pair
+  float* diag_wts = nullptr;     // [max_tokens][2] its normalised weights
+  int32_t* diag_q = nullptr;     // [max_tokens][K] residual order
+  float* diag_E = nullptr;       // [max_tokens][K][d] E_e(x)
+  float* diag_ES = nullptr;      // [max_tokens][K][d] E_e^{S_ij}(x)
 };
 
 }  // namespace unif
@@ -213,5 +221,9 @@ cudaError_t launch_transpose_weights(unif_moe_layer* L, cudaStream_t s);
 int backward_run(unif_moe_layer* L, const void* x, const void* dy, int T, const uint8_t* mask,
                  float* dx, float* dw_up, float* dw_down, float* dw_router, float* dbias,
                  float lambda_div, float* l_div, cudaStream_t s);
+// Diagnostics (diagnostics.cu); 0 or -1 (CUDA failure).
+int diag_alignment(unif_moe_layer* L, float delta, float* rho, cudaStream_t s);
+int diag_demand(unif_moe_layer* L, const void* x, int T, const void* w_res, float delta,
+                float eps, int32_t* k_eps, float* err, int32_t* pair_out, cudaStream_t s);
 
 }  // namespace unif

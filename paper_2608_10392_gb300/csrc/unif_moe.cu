@@ -71,7 +71,9 @@ void free_all(unif_moe_layer* L) {
                   L->ws.xn, L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
                   L->ws.k_stage, L->ws.status, L->ws.grp_fill,
                   L->ws.tile_rows, L->ws.w_upT, L->ws.w_downT, L->ws.da, L->ws.hw,
-                  L->ws.dwt, L->ws.dz, L->ws.wrT, L->ws.gram};
+                  L->ws.dwt, L->ws.dz, L->ws.wrT, L->ws.gram, L->ws.diag_sets,
+                  L->ws.diag_counts, L->ws.diag_pair, L->ws.diag_wts, L->ws.diag_q,
+                  L->ws.diag_E, L->ws.diag_ES};
   for (void* q : ptrs)
     if (q) cudaFree(q);
 }
@@ -256,6 +258,12 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
     if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.hw), es * (size_t)L->max_rows * M);
     ALLOC(w.dwt, T * E); ALLOC(w.dz, T * E);
     ALLOC(w.wrT, E * d_model); ALLOC(w.gram, E * E);
+  }
+  if (o.features & UNIF_MOE_FEATURE_DIAGNOSTICS) {
+    const size_t H32 = ((size_t)d_ff + 31) / 32;
+    ALLOC(w.diag_sets, K * K * H32); ALLOC(w.diag_counts, K * K);
+    ALLOC(w.diag_pair, 2 * T); ALLOC(w.diag_wts, 2 * T); ALLOC(w.diag_q, T * K);
+    ALLOC(w.diag_E, T * K * d_model); ALLOC(w.diag_ES, T * K * d_model);
   }
 #undef ALLOC
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
@@ -460,6 +468,55 @@ int unif_moe_backward(unif_moe_t L, const void* x, const void* dy, int T, const 
   DeviceGuard dg(L->device);
   return unif::backward_run(L, x, dy, T, mask, dx, dw_up, dw_down, dw_router, dbias, lambda_div,
                             l_div, static_cast<cudaStream_t>(stream));
+}
+
+int unif_moe_value_alignment(unif_moe_t L, float delta, float* rho, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (!(L->features & UNIF_MOE_FEATURE_DIAGNOSTICS)) {
+    set_error("diagnostics on a handle created without UNIF_MOE_FEATURE_DIAGNOSTICS");
+    return UNIF_MOE_ERR_STATE;
+  }
+  if (!L->loaded) { set_error("no weights loaded"); return UNIF_MOE_ERR_STATE; }
+  if (!rho || !isfinite(delta)) { set_error("rho is NULL or delta not finite"); return UNIF_MOE_ERR_ARG; }
+  DeviceGuard dg(L->device);
+  if (unif::diag_alignment(L, delta, rho, static_cast<cudaStream_t>(stream)) != 0) {
+    set_error("value alignment launch failed");
+    return UNIF_MOE_ERR_CUDA;
+  }
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_functional_demand(unif_moe_t L, const void* x, int T, const void* w_res,
+                               float delta, float eps, int32_t* k_eps, float* err,
+                               int32_t* pair, void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (!(L->features & UNIF_MOE_FEATURE_DIAGNOSTICS)) {
+    set_error("diagnostics on a handle created without UNIF_MOE_FEATURE_DIAGNOSTICS");
+    return UNIF_MOE_ERR_STATE;
+  }
+  if (!L->loaded) { set_error("no weights loaded"); return UNIF_MOE_ERR_STATE; }
+  if (L->K < 2 || L->K > 32) {
+    set_error("functional demand needs 2 <= K <= 32 (K=%d)", L->K);
+    return UNIF_MOE_ERR_SHAPE;
+  }
+  if (T < 0 || T > L->max_tokens) {
+    set_error("T=%d outside [0, max_tokens=%d]", T, L->max_tokens);
+    return T < 0 ? UNIF_MOE_ERR_ARG : UNIF_MOE_ERR_CAPACITY;
+  }
+  if (T == 0) return UNIF_MOE_OK;
+  if (!x || !w_res || !k_eps || !isfinite(delta) || !isfinite(eps)) {
+    set_error("NULL x, w_res or k_eps, or delta / eps not finite");
+    return UNIF_MOE_ERR_ARG;
+  }
+  DeviceGuard dg(L->device);
+  if (unif::diag_demand(L, x, T, w_res, delta, eps, k_eps, err, pair,
+                        static_cast<cudaStream_t>(stream)) != 0) {
+    set_error("functional demand launch failed");
+    return UNIF_MOE_ERR_CUDA;
+  }
+  return UNIF_MOE_OK;
 }
 
 int unif_moe_forward(unif_moe_t L, const void* x, void* out, int T, const uint8_t* token_mask,

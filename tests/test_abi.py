@@ -66,7 +66,7 @@ def test_argument_errors_without_gpu(lib):
     opts = pkg.Options()
     lib.unif_moe_default_options(C.byref(opts))
     assert opts.features == pkg.FEATURES_DEFAULT and opts.gemm_kernels == 0
-    for o in (pkg.Options(8, 0), pkg.Options(3, 2), pkg.Options(3, -1)):  # unknown bit / kind
+    for o in (pkg.Options(16, 0), pkg.Options(3, 2), pkg.Options(3, -1)):  # unknown bit / kind
         assert lib.unif_moe_create_ex(C.byref(h), 64, 256, 4, 4, None, 1, 16, C.byref(o)) == -1
     assert b"options" in lib.unif_moe_last_error()
     assert lib.unif_moe_forward(None, None, None, 4, None, None, None, None) == -1
@@ -76,6 +76,9 @@ def test_argument_errors_without_gpu(lib):
                                          1e-5, 1, None) == -1
     assert lib.unif_moe_backward(None, None, None, 4, None, None, None, None, None, None, 0.0,
                                  None, None) == -1
+    assert lib.unif_moe_value_alignment(None, 0.98, None, None) == -1
+    assert lib.unif_moe_functional_demand(None, None, 4, None, 0.98, 0.05, None, None, None,
+                                          None) == -1
     assert lib.unif_moe_sync_status(None, None) == -1
     assert lib.unif_moe_max_rows(None) == -1
     assert lib.unif_moe_kernels_per_forward(None) == -1
