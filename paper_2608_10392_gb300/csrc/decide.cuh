@@ -353,34 +353,36 @@ __device__ __forceinline__ void named_bar(uint32_t id, uint32_t n) {
 
 // Shared-memory ints group_rows needs.
 __host__ __device__ constexpr int group_rows_smem_ints(int NW, int G) {
-  return NW * G + G + 8;  // chunk counts, bases, misc
+  return NW * G + 8;  // per-chunk counts (then first rows), misc
 }
 
 // Runs in the NW decision warps of a router CTA (threads tid = 0 .. NW*32-1,
-// named barrier `bar`; thread tid holds token t0 + tid), after warp w's
-// count_chunk_pairs wrote its 32-token chunk's per-group pair counts to
-// sm[w * G + g] and its lane masks to masks[w * 128 ...] (masks[blk] = lanes
-// sharing block blk, masks[64 + j] = lanes selecting residual expert j).
-// Token i of the CTA has alpha at dec_s[i * dec_stride + 2K] and its
-// affinities s_1..s_K at dec_s[i * dec_stride + j]. `sm` has
-// group_rows_smem_ints(NW, G) ints.
+// named barrier `bar`; thread tid holds token t0 + tid, with shared block set
+// `shr` and residual expert set `em`), after warp w's count_chunk_pairs
+// wrote its 32-token chunk's per-group pair counts to sm[w * G + g] and its
+// lane masks to masks[w * 128 ...] (masks[blk] = lanes sharing block blk,
+// masks[64 + j] = lanes selecting residual expert j). Token i of the CTA has
+// alpha at dec_s[i * dec_stride + 2K] and its affinities s_1..s_K at
+// dec_s[i * dec_stride + j]. `sm` has group_rows_smem_ints(NW, G) ints.
 //
-// With one warp per scheduler, per-row work must be short and free of
-// shared-memory round trips: a thread takes one (group, chunk) pair, walks
-// the chunk's member bits of the group (token order) and writes those rows
-// one after another.
+// Each thread writes its own token's rows: with one warp per scheduler the
+// phase is bound by the length of each thread's chain of index arithmetic,
+// and a token's rows (b + k (B - b) of them) make a shorter chain than the
+// rows of one (group, chunk) pair walked by one thread.
 template <int NW>
-__device__ void group_rows(const GroupArgs& a, int tid, int t0, const uint32_t* masks,
-                           const float* dec_s, int dec_stride, int32_t* sm, uint32_t bar) {
+__device__ void group_rows(const GroupArgs& a, int tid, int t0, uint64_t shr, uint64_t em,
+                           const uint32_t* masks, const float* dec_s, int dec_stride,
+                           int32_t* sm, uint32_t bar) {
   constexpr int NT = NW * 32;
   const int G = a.G, B = a.B;
-  int32_t* cnt_s = sm;                    // [NW][G] chunk counts
-  int32_t* base_s = cnt_s + NW * G;       // [G] first reserved row, or -1
-  // 1. this CTA's rows of each group, reserved in the group's region
+  int32_t* first = sm;  // [NW][G] chunk counts, then each chunk's first row
+  // 1. this CTA's rows of each group, reserved in the group's region; the
+  // rows of chunk v follow those of chunks 0 .. v-1 (token order). A group
+  // whose rows were not reserved gets a negative first row in every chunk.
   for (int g = tid; g < G; g += NT) {
     int n = 0;
 #pragma unroll
-    for (int v = 0; v < NW; ++v) n += cnt_s[v * G + g];
+    for (int v = 0; v < NW; ++v) n += first[v * G + g];
     int base = -1;
     if (n > 0) {
       base = atomicAdd(a.fill + g, n);
@@ -389,30 +391,44 @@ __device__ void group_rows(const GroupArgs& a, int tid, int t0, const uint32_t* 
         base = -1;
       }
     }
-    base_s[g] = base;
+    int o = base < 0 ? -(1 << 30) : base;
+#pragma unroll
+    for (int v = 0; v < NW; ++v) {
+      const int c = first[v * G + g];
+      first[v * G + g] = o;
+      o += c;
+    }
   }
   named_bar(bar, NT);
-  // 2. the rows, in token order: a thread takes the rows of one group from
-  // one 32-token chunk (after the rows of the group's earlier chunks)
-  for (int idx = tid; idx < G * NW; idx += NT) {
-    const int g = idx / NW, c = idx - g * NW;
-    const int base = base_s[g];
-    if (base < 0) continue;
-    int off = 0;
-#pragma unroll
-    for (int v = 0; v < NW; ++v) off += v < c ? cnt_s[v * G + g] : 0;
-    const int e = g / B, blk = g - e * B;
-    const int wcol = e == 0 ? 2 * a.K : e - 1;
-    const size_t r0 = (size_t)g * a.region + base + off;
-    int32_t* tok = a.row_tok + r0;
-    float* wt = a.row_w + r0;
-    const uint32_t sh = masks[c * 128 + blk];
-    uint32_t m = e == 0 ? sh : (masks[c * 128 + 64 + e - 1] & ~sh);
-    for (int r = 0; m != 0u; ++r) {
-      const int i = c * 32 + __ffs(m) - 1;
-      m &= m - 1u;
-      tok[r] = t0 + i;
-      wt[r] = dec_s[i * dec_stride + wcol];
+  // 2. the token's rows: its row in group g is the chunk's first row of g
+  // plus the number of lower lanes of the chunk that are also in g
+  const int c = tid >> 5;
+  const uint32_t lt = (1u << (tid & 31)) - 1u;
+  const int32_t* fc = first + c * G;
+  const uint32_t* mk = masks + c * 128;
+  const float* ds = dec_s + tid * dec_stride;
+  const int tok = t0 + tid;
+  const float alpha = ds[2 * a.K];
+  for (uint64_t rem = shr; rem != 0ull; rem &= rem - 1ull) {  // shared blocks (e = 0)
+    const int blk = __ffsll((long long)rem) - 1;
+    const int r = fc[blk] + __popc(mk[blk] & lt);
+    if (r >= 0) {
+      a.row_tok[(size_t)blk * a.region + r] = tok;
+      a.row_w[(size_t)blk * a.region + r] = alpha;
+    }
+  }
+  const uint64_t comp = ~shr & (B >= 64 ? ~0ull : ((1ull << B) - 1ull));
+  for (uint64_t rj = em; rj != 0ull; rj &= rj - 1ull) {  // residual experts
+    const int j = __ffsll((long long)rj) - 1;
+    const uint32_t mj = mk[64 + j];
+    const float w = ds[j];
+    for (uint64_t rb = comp; rb != 0ull; rb &= rb - 1ull) {  // their complementary blocks
+      const int blk = __ffsll((long long)rb) - 1, g = (j + 1) * B + blk;
+      const int r = fc[g] + __popc(mj & ~mk[blk] & lt);
+      if (r >= 0) {
+        a.row_tok[(size_t)g * a.region + r] = tok;
+        a.row_w[(size_t)g * a.region + r] = w;
+      }
     }
   }
 }

@@ -518,7 +518,7 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
       named_bar(1, 128);
       if (row == 0) misc_s[7] = *abort_flag;  // one reading for all four warps
       named_bar(1, 128);
-      if (!misc_s[7]) group_rows<4>(p.grp, row, t0, cscr, ss, 2 * K + 1, gsm, 1);
+      if (!misc_s[7]) group_rows<4>(p.grp, row, t0, shr, em, cscr, ss, 2 * K + 1, gsm, 1);
     }
   }
   __syncwarp();  // every warp converged before the CTA barrier
