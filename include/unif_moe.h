@@ -79,8 +79,9 @@ UNIF_MOE_API void unif_moe_default_thresholds(unif_moe_thresholds* th);
 enum {
   UNIF_MOE_FEATURE_NORM_FIRST = 1, /* unif_moe_sublayer_forward with norm_first:
                                       a [max_tokens][d] buffer for LN(x) */
-  UNIF_MOE_FEATURE_HOST_IO = 2,    /* unif_moe_forward_host: device staging
-                                      buffers for x, y, the mask and the counts */
+  UNIF_MOE_FEATURE_HOST_IO = 2,    /* unif_moe_forward_host(_async): two slots
+                                      of device staging buffers for x, y, the
+                                      mask and the counts, two copy streams */
   UNIF_MOE_FEATURE_BACKWARD = 4,   /* unif_moe_backward: transposed copies of the
                                       expert weights and per-row gradient buffers
                                       (bf16 layers, d % 128 == 0) */
@@ -200,6 +201,34 @@ UNIF_MOE_API int unif_moe_sublayer_forward(unif_moe_t h, const void* x_dev, void
 UNIF_MOE_API int unif_moe_forward_host(unif_moe_t h, const void* x_host, void* out_host, int T,
                           const uint8_t* token_mask_host, int32_t* shared_counts_host,
                           int32_t* residual_counts_host, void* stream);
+
+/* Pipelined forwards from host buffers, for a stream of batches: enqueues
+ * the forward of x_host and returns without waiting. Arguments and results
+ * as unif_moe_forward_host (the same Eqs. 16-30; out_host [T][d] and the
+ * counts receive this call's results), but the copies overlap other calls'
+ * kernels: calls alternate between the handle's two staging slots, and a
+ * call's input copy runs on a copy stream of the handle while the previous
+ * call's kernels run on `stream`, its output copy on a second copy stream
+ * while the next call's kernels run. A slot is refilled only after the
+ * kernels two calls back have read it and their output has been copied out.
+ * Ownership: the caller keeps x_host and token_mask_host unchanged, and does
+ * not read out_host or the counts, until unif_moe_forward_host_wait has
+ * returned; host buffers must be pinned (page-locked) for the copies to
+ * overlap (pageable ones are still correct). Consecutive calls on one handle
+ * pass the same `stream`; unif_moe_forward_host, unif_moe_get_routing and
+ * the other calls that read the last forward's state come after
+ * unif_moe_forward_host_wait. Errors: as unif_moe_forward_host (ERR_STATE
+ * without UNIF_MOE_FEATURE_HOST_IO); a kernel timeout surfaces through
+ * unif_moe_sync_status. Nothing is allocated. */
+UNIF_MOE_API int unif_moe_forward_host_async(unif_moe_t h, const void* x_host, void* out_host,
+                                             int T, const uint8_t* token_mask_host,
+                                             int32_t* shared_counts_host,
+                                             int32_t* residual_counts_host, void* stream);
+
+/* Blocks until every forward enqueued by unif_moe_forward_host_async has
+ * its output and counts in host memory. Errors: ERR_ARG (NULL handle),
+ * ERR_STATE (handle without UNIF_MOE_FEATURE_HOST_IO), ERR_CUDA. */
+UNIF_MOE_API int unif_moe_forward_host_wait(unif_moe_t h);
 
 /* Backward pass of the last forward for training (Sec. III-E): given
  * dL/dy, the gradients of L with respect to x and to every parameter of

@@ -34,7 +34,8 @@ EXPORTS = ["unif_moe_default_thresholds", "unif_moe_default_options", "unif_moe_
            "unif_moe_create_ex", "unif_moe_load_weights",
            "unif_moe_load_upcycled", "unif_moe_forward", "unif_moe_sublayer_forward",
            "unif_moe_backward", "unif_moe_value_alignment", "unif_moe_functional_demand",
-           "unif_moe_forward_host", "unif_moe_get_routing",
+           "unif_moe_forward_host", "unif_moe_forward_host_async",
+           "unif_moe_forward_host_wait", "unif_moe_get_routing",
            "unif_moe_get_groups", "unif_moe_max_rows", "unif_moe_pass_tokens",
            "unif_moe_kernels_per_forward",
            "unif_moe_set_stage_events",
@@ -88,6 +89,8 @@ def lib(path: str = LIB_PATH) -> C.CDLL:
         L.unif_moe_value_alignment.argtypes = [P, C.c_float, P, P]
         L.unif_moe_functional_demand.argtypes = [P, P, I, P, C.c_float, C.c_float, P, P, P, P]
         L.unif_moe_forward_host.argtypes = [P, P, P, I, P, P, P, P]
+        L.unif_moe_forward_host_async.argtypes = [P, P, P, I, P, P, P, P]
+        L.unif_moe_forward_host_wait.argtypes = [P]
         L.unif_moe_get_routing.argtypes = [P, P, P, P, P, P, P]
         L.unif_moe_get_groups.argtypes = [P, P, P, P, P, C.POINTER(C.c_int64), P]
         L.unif_moe_max_rows.argtypes = [P]
@@ -266,6 +269,23 @@ class Layer:
                                            _ptr(residual_counts_host), _stream(stream)))
         self.last_T = T
         return out_host
+
+    def forward_host_async(self, x_host: torch.Tensor, out_host: torch.Tensor,
+                           mask_host: Optional[torch.Tensor] = None,
+                           shared_counts_host: Optional[torch.Tensor] = None,
+                           residual_counts_host: Optional[torch.Tensor] = None, stream=None):
+        """Enqueues a forward of host tensors and returns at once (the copies
+        overlap other calls' kernels); results are in out_host (and the
+        counts) after forward_host_wait()."""
+        T = x_host.shape[0]
+        _check(lib().unif_moe_forward_host_async(self._h, _ptr(x_host), _ptr(out_host), T,
+                                                 _ptr(mask_host), _ptr(shared_counts_host),
+                                                 _ptr(residual_counts_host), _stream(stream)))
+        self.last_T = T
+        return out_host
+
+    def forward_host_wait(self):
+        _check(lib().unif_moe_forward_host_wait(self._h))
 
     def routing(self, stream=None) -> dict:
         """Decisions of the last forward, as CUDA tensors."""

@@ -75,12 +75,13 @@ struct Workspace {
   float* y32 = nullptr;          // [max_tokens][d]
   // Host-buffer forward staging.
   void* xn = nullptr;             // [max_tokens][d] LN(x) of a norm-first sublayer
-  // Staging buffers of the host-buffer forward.
-  void* x_stage = nullptr;
-  void* out_stage = nullptr;
-  uint8_t* mask_stage = nullptr;
-  int32_t* b_stage = nullptr;
-  int32_t* k_stage = nullptr;
+  // Staging buffers of the host-buffer forwards, two slots (the pipelined
+  // forward alternates between them; the synchronous one uses slot 0).
+  void* x_stage[2] = {nullptr, nullptr};
+  void* out_stage[2] = {nullptr, nullptr};
+  uint8_t* mask_stage[2] = {nullptr, nullptr};
+  int32_t* b_stage[2] = {nullptr, nullptr};
+  int32_t* k_stage[2] = {nullptr, nullptr};
   int* status = nullptr;         // device status word
   // Backward pass (UNIF_MOE_FEATURE_BACKWARD).
   void* w_upT = nullptr;         // [K+1][d][H] keys transposed (layer dtype)
@@ -163,6 +164,14 @@ struct unif_moe_layer {
   CUtensorMap tm_da_q;      // da, boxes of 64 x 32 (weight-gradient operand)
   CUtensorMap tm_hw_q;      // hw, boxes of 64 x 32
   uint32_t bwd_hidden_smem = 0, bwd_wgrad_smem = 0;
+  // Pipelined host-buffer forwards (UNIF_MOE_FEATURE_HOST_IO): the handle's
+  // copy streams, and per staging slot the events that order its reuse
+  // (input landed, kernels done, output copied out).
+  cudaStream_t copy_in = nullptr, copy_out = nullptr;
+  cudaEvent_t ev_in[2] = {nullptr, nullptr};
+  cudaEvent_t ev_comp[2] = {nullptr, nullptr};
+  cudaEvent_t ev_out[2] = {nullptr, nullptr};
+  int host_slot = 0;  // slot of the next pipelined forward
   // Optional caller-owned timing events recorded at the stage boundaries.
   cudaEvent_t stage_ev[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
 };

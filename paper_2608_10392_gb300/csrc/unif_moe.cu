@@ -68,14 +68,23 @@ void free_all(unif_moe_layer* L) {
                   L->ws.shr_mask, L->ws.exp_mask, L->ws.s, L->ws.chunk_cnt,
                   L->ws.grp_cnt, L->ws.grp_off, L->ws.n_tiles, L->ws.tile_group,
                   L->ws.tile_row0, L->ws.row_tok, L->ws.row_w, L->ws.hbuf, L->ws.y32,
-                  L->ws.xn, L->ws.x_stage, L->ws.out_stage, L->ws.mask_stage, L->ws.b_stage,
-                  L->ws.k_stage, L->ws.status, L->ws.grp_fill,
+                  L->ws.xn, L->ws.x_stage[0], L->ws.out_stage[0], L->ws.mask_stage[0],
+                  L->ws.b_stage[0], L->ws.k_stage[0], L->ws.x_stage[1], L->ws.out_stage[1],
+                  L->ws.mask_stage[1], L->ws.b_stage[1], L->ws.k_stage[1], L->ws.status,
+                  L->ws.grp_fill,
                   L->ws.tile_rows, L->ws.w_upT, L->ws.w_downT, L->ws.da, L->ws.hw,
                   L->ws.dwt, L->ws.dz, L->ws.wrT, L->ws.gram, L->ws.diag_sets,
                   L->ws.diag_counts, L->ws.diag_pair, L->ws.diag_wts, L->ws.diag_q,
                   L->ws.diag_E, L->ws.diag_ES};
   for (void* q : ptrs)
     if (q) cudaFree(q);
+  for (int i = 0; i < 2; ++i) {
+    if (L->ev_in[i]) cudaEventDestroy(L->ev_in[i]);
+    if (L->ev_comp[i]) cudaEventDestroy(L->ev_comp[i]);
+    if (L->ev_out[i]) cudaEventDestroy(L->ev_out[i]);
+  }
+  if (L->copy_in) cudaStreamDestroy(L->copy_in);
+  if (L->copy_out) cudaStreamDestroy(L->copy_out);
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -242,9 +251,23 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
     if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.xn), es * T * d_model);
   }
   if (o.features & UNIF_MOE_FEATURE_HOST_IO) {
-    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.x_stage), es * T * d_model);
-    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.out_stage), es * T * d_model);
-    ALLOC(w.mask_stage, T); ALLOC(w.b_stage, T); ALLOC(w.k_stage, T);
+    for (int i = 0; i < 2; ++i) {
+      if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.x_stage[i]), es * T * d_model);
+      if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.out_stage[i]), es * T * d_model);
+      ALLOC(w.mask_stage[i], T); ALLOC(w.b_stage[i], T); ALLOC(w.k_stage[i], T);
+    }
+    // the pipelined forward's copy streams and slot events
+    bool ok = rc == UNIF_MOE_OK &&
+              cudaStreamCreateWithFlags(&L->copy_in, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaStreamCreateWithFlags(&L->copy_out, cudaStreamNonBlocking) == cudaSuccess;
+    for (int i = 0; i < 2 && ok; ++i)
+      ok = cudaEventCreateWithFlags(&L->ev_in[i], cudaEventDisableTiming) == cudaSuccess &&
+           cudaEventCreateWithFlags(&L->ev_comp[i], cudaEventDisableTiming) == cudaSuccess &&
+           cudaEventCreateWithFlags(&L->ev_out[i], cudaEventDisableTiming) == cudaSuccess;
+    if (rc == UNIF_MOE_OK && !ok) {
+      set_error("creating the host-buffer copy streams or events failed");
+      rc = UNIF_MOE_ERR_CUDA;
+    }
   }
   if (o.features & UNIF_MOE_FEATURE_BACKWARD) {
     if (rc == UNIF_MOE_OK && (dtype != UNIF_MOE_BF16 || !L->fused_group || d_model % 128 != 0)) {
@@ -596,25 +619,93 @@ int unif_moe_forward_host(unif_moe_t L, const void* x_host, void* out_host, int 
   unif::Workspace& w = L->ws;
   const size_t es = elt_size(L);
   const size_t xb = es * (size_t)T * L->d;
-  CK(cudaMemcpyAsync(w.x_stage, x_host, xb, cudaMemcpyHostToDevice, s));
-  if (mask_host) CK(cudaMemcpyAsync(w.mask_stage, mask_host, (size_t)T, cudaMemcpyHostToDevice, s));
+  // slot 0 may still be in use by pipelined forwards
+  CK(cudaStreamSynchronize(L->copy_in));
+  CK(cudaStreamSynchronize(L->copy_out));
+  CK(cudaMemcpyAsync(w.x_stage[0], x_host, xb, cudaMemcpyHostToDevice, s));
+  if (mask_host) CK(cudaMemcpyAsync(w.mask_stage[0], mask_host, (size_t)T, cudaMemcpyHostToDevice, s));
   // Outputs in pinned host memory that the device can address are written
   // there by the kernels themselves (the combine, the router), without a
   // staging buffer and a copy back.
   void* out_dev = mapped_host(out_host);
   int32_t* b_dev = static_cast<int32_t*>(mapped_host(b_host));
   int32_t* k_dev = static_cast<int32_t*>(mapped_host(k_host));
-  int rc = unif_moe_forward(L, w.x_stage, out_dev ? out_dev : w.out_stage, T,
-                            mask_host ? w.mask_stage : nullptr,
-                            b_host ? (b_dev ? b_dev : w.b_stage) : nullptr,
-                            k_host ? (k_dev ? k_dev : w.k_stage) : nullptr, stream);
+  int rc = unif_moe_forward(L, w.x_stage[0], out_dev ? out_dev : w.out_stage[0], T,
+                            mask_host ? w.mask_stage[0] : nullptr,
+                            b_host ? (b_dev ? b_dev : w.b_stage[0]) : nullptr,
+                            k_host ? (k_dev ? k_dev : w.k_stage[0]) : nullptr, stream);
   if (rc != UNIF_MOE_OK) return rc;
-  if (!out_dev) CK(cudaMemcpyAsync(out_host, w.out_stage, xb, cudaMemcpyDeviceToHost, s));
+  if (!out_dev) CK(cudaMemcpyAsync(out_host, w.out_stage[0], xb, cudaMemcpyDeviceToHost, s));
   if (b_host && !b_dev)
-    CK(cudaMemcpyAsync(b_host, w.b_stage, sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
+    CK(cudaMemcpyAsync(b_host, w.b_stage[0], sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
   if (k_host && !k_dev)
-    CK(cudaMemcpyAsync(k_host, w.k_stage, sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
+    CK(cudaMemcpyAsync(k_host, w.k_stage[0], sizeof(int32_t) * T, cudaMemcpyDeviceToHost, s));
   CK(cudaStreamSynchronize(s));
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_forward_host_async(unif_moe_t L, const void* x_host, void* out_host, int T,
+                                const uint8_t* mask_host, int32_t* b_host, int32_t* k_host,
+                                void* stream) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (T < 0 || T > L->max_tokens) {
+    set_error("T=%d outside [0, max_tokens=%d]", T, L->max_tokens);
+    return T < 0 ? UNIF_MOE_ERR_ARG : UNIF_MOE_ERR_CAPACITY;
+  }
+  if (!L->loaded) { set_error("forward before load_weights"); return UNIF_MOE_ERR_STATE; }
+  if (!(L->features & UNIF_MOE_FEATURE_HOST_IO)) {
+    set_error("host-buffer forward on a handle created without UNIF_MOE_FEATURE_HOST_IO");
+    return UNIF_MOE_ERR_STATE;
+  }
+  if (T == 0) return UNIF_MOE_OK;
+  if (!x_host || !out_host) { set_error("x or out is NULL"); return UNIF_MOE_ERR_ARG; }
+  DeviceGuard dg(L->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unif::Workspace& w = L->ws;
+  const int i = L->host_slot;
+  const size_t xb = elt_size(L) * (size_t)T * L->d;
+  // input, on the copy-in stream: once the kernels that read this slot two
+  // calls ago are done, so that it overlaps the previous call's kernels
+  CK(cudaStreamWaitEvent(L->copy_in, L->ev_comp[i], 0));
+  CK(cudaMemcpyAsync(w.x_stage[i], x_host, xb, cudaMemcpyHostToDevice, L->copy_in));
+  if (mask_host)
+    CK(cudaMemcpyAsync(w.mask_stage[i], mask_host, (size_t)T, cudaMemcpyHostToDevice, L->copy_in));
+  CK(cudaEventRecord(L->ev_in[i], L->copy_in));
+  // kernels, on the caller's stream: after this slot's input has landed and
+  // its previous output (and counts) have been copied out
+  CK(cudaStreamWaitEvent(s, L->ev_in[i], 0));
+  CK(cudaStreamWaitEvent(s, L->ev_out[i], 0));
+  const int rc = unif_moe_forward(L, w.x_stage[i], w.out_stage[i], T,
+                                  mask_host ? w.mask_stage[i] : nullptr,
+                                  b_host ? w.b_stage[i] : nullptr, k_host ? w.k_stage[i] : nullptr,
+                                  stream);
+  if (rc != UNIF_MOE_OK) return rc;
+  CK(cudaEventRecord(L->ev_comp[i], s));
+  // output, on the copy-out stream, overlapping the next call's kernels
+  CK(cudaStreamWaitEvent(L->copy_out, L->ev_comp[i], 0));
+  CK(cudaMemcpyAsync(out_host, w.out_stage[i], xb, cudaMemcpyDeviceToHost, L->copy_out));
+  if (b_host)
+    CK(cudaMemcpyAsync(b_host, w.b_stage[i], sizeof(int32_t) * T, cudaMemcpyDeviceToHost,
+                       L->copy_out));
+  if (k_host)
+    CK(cudaMemcpyAsync(k_host, w.k_stage[i], sizeof(int32_t) * T, cudaMemcpyDeviceToHost,
+                       L->copy_out));
+  CK(cudaEventRecord(L->ev_out[i], L->copy_out));
+  L->host_slot = i ^ 1;
+  return UNIF_MOE_OK;
+}
+
+int unif_moe_forward_host_wait(unif_moe_t L) {
+  unif::g_err[0] = 0;
+  if (!L) { set_error("NULL handle"); return UNIF_MOE_ERR_ARG; }
+  if (!(L->features & UNIF_MOE_FEATURE_HOST_IO)) {
+    set_error("host-buffer forward on a handle created without UNIF_MOE_FEATURE_HOST_IO");
+    return UNIF_MOE_ERR_STATE;
+  }
+  DeviceGuard dg(L->device);
+  CK(cudaStreamSynchronize(L->copy_in));
+  CK(cudaStreamSynchronize(L->copy_out));
   return UNIF_MOE_OK;
 }
 

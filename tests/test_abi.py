@@ -80,6 +80,9 @@ def test_argument_errors_without_gpu(lib):
     assert lib.unif_moe_functional_demand(None, None, 4, None, 0.98, 0.05, None, None, None,
                                           None) == -1
     assert lib.unif_moe_sync_status(None, None) == -1
+    assert lib.unif_moe_forward_host(None, None, None, 4, None, None, None, None) == -1
+    assert lib.unif_moe_forward_host_async(None, None, None, 4, None, None, None, None) == -1
+    assert lib.unif_moe_forward_host_wait(None) == -1
     assert lib.unif_moe_max_rows(None) == -1
     assert lib.unif_moe_kernels_per_forward(None) == -1
     lib.unif_moe_destroy(None)

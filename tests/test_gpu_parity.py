@@ -390,6 +390,51 @@ def test_forward_host_pageable_buffers():
     assert np.array_equal(b.numpy(), g.b) and np.array_equal(k.numpy(), g.k)
 
 
+def test_forward_host_async_pipeline():
+    """Pipelined host-buffer forwards: four different batches (different
+    sizes, a padding mask on two) enqueued back to back, so that both staging
+    slots are refilled while earlier calls' kernels and copies are in flight;
+    each call's output and counts match the device forward of its batch, and
+    a synchronous host-buffer forward afterwards is unaffected."""
+    base = workloads.make_workload(small(tokens=700))
+    layer = run_gpu(base).layer
+    dev = torch.device("cuda")
+    gen = torch.Generator().manual_seed(5)
+    batches = []
+    for i, T in enumerate([700, 513, 640, 128]):
+        idx = torch.randperm(700, generator=gen)[:T]
+        x = (base.x[idx].float() * (1.0 + 0.1 * i)).to(base.x.dtype)
+        m = None if i % 2 == 0 else (torch.rand(T, generator=gen) > 0.2).to(torch.uint8)
+        b = torch.empty(T, dtype=torch.int32, device=dev)
+        k = torch.empty(T, dtype=torch.int32, device=dev)
+        y = layer.forward(x.to(dev), mask=None if m is None else m.to(dev), shared_counts=b,
+                          residual_counts=k)
+        torch.cuda.synchronize()
+        batches.append((x, m, y.float().cpu(), b.cpu(), k.cpu()))
+    pending = []
+    for x, m, *_ in batches:
+        T = x.shape[0]
+        xh = x.pin_memory()
+        mh = None if m is None else m.pin_memory()
+        oh = torch.full_like(xh, float("nan")).pin_memory()
+        bh = torch.full((T,), -7, dtype=torch.int32).pin_memory()
+        kh = torch.full((T,), -7, dtype=torch.int32).pin_memory()
+        layer.forward_host_async(xh, oh, mh, bh, kh)
+        pending.append((xh, mh, oh, bh, kh))
+    layer.forward_host_wait()
+    torch.cuda.synchronize()
+    assert layer.sync_status() == 0
+    for (x, m, y, b, k), (_, _, oh, bh, kh) in zip(batches, pending):
+        np.testing.assert_allclose(oh.float().numpy(), y.numpy(), rtol=1e-2, atol=1e-6)
+        assert np.array_equal(bh.numpy(), b.numpy()) and np.array_equal(kh.numpy(), k.numpy())
+    x, m, y, b, k = batches[1]
+    out = torch.empty_like(x).pin_memory()
+    bh = torch.empty(x.shape[0], dtype=torch.int32).pin_memory()
+    layer.forward_host(x.pin_memory(), out, m.pin_memory(), shared_counts_host=bh)
+    np.testing.assert_allclose(out.float().numpy(), y.numpy(), rtol=1e-2, atol=1e-6)
+    assert np.array_equal(bh.numpy(), b.numpy())
+
+
 # ------------------------------------------- GEMM kernel variants
 
 @pytest.mark.parametrize("kernels", ["weight_stationary", "streaming"])
