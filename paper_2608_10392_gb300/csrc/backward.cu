@@ -551,81 +551,187 @@ bwd_wgrad_kernel(const __grid_constant__ CUtensorMap tm_da, const __grid_constan
 // ---------------------------------------------------------------------------
 // Router gradients (Eqs. 17, 18, 24)
 // ---------------------------------------------------------------------------
-// One warp per token: dL/dz_0 = dL/dalpha (1 - 2 tau) sigma(z_0)(1 - sigma(z_0))
+// dL/dz of token t into z[0..KC) (K + 1 <= KC values, the rest and a padding
+// token's all zero): dL/dz_0 = dL/dalpha (1 - 2 tau) sigma(z_0)(1 - sigma(z_0))
 // (adaptive alpha; sigma(z_0) = (alpha - tau) / (1 - 2 tau) from the stored
-// alpha), dL/dz_{1+j} = s_j (dL/ds_j - sum_l s_l dL/ds_l); then dx[t] +=
-// dL/dz W*^T, with W*^T the router's first K+1 columns transposed (fp32
-// [K+1][d], so that the lanes read consecutive features). Lane l keeps
-// dL/dz_c for c = l, l + 32, l + 64 in registers.
-// dL/dz of token t and its share of dL/dx (one warp, `lane` its lane).
-__device__ __forceinline__ void router_grad_token(int t, int K, int d, float tau, int adaptive,
-                                                  const uint8_t* __restrict__ mask,
-                                                  const float* __restrict__ alpha,
-                                                  const float* __restrict__ s,
-                                                  const float* __restrict__ dwt,
-                                                  const float* __restrict__ wrT,
-                                                  float* __restrict__ dz,
-                                                  float* __restrict__ dx, int lane) {
+// alpha), dL/dz_{1+j} = s_j (dL/ds_j - sum_l s_l dL/ds_l), from the pathway
+// weights' gradients dL/dalpha, dL/ds_j that the hidden kernel accumulated.
+// All of the token's loads go out before the arithmetic.
+template <int KC>
+__device__ __forceinline__ void router_token_dz(int t, int K, float tau, int adaptive,
+                                                const uint8_t* __restrict__ mask,
+                                                const float* __restrict__ alpha,
+                                                const float* __restrict__ s,
+                                                const float* __restrict__ dwt, float (&z)[KC]) {
   const int K1 = K + 1;
-  float* dzt = dz + (size_t)t * K1;
-  if (mask && !mask[t]) {
-    for (int c = lane; c < K1; c += 32) dzt[c] = 0.f;
-    return;
-  }
+  const bool valid = !mask || mask[t];
   const float* st = s + (size_t)t * K;
   const float* gt = dwt + (size_t)t * K1;
-  float part = 0.f;
-  for (int j = lane; j < K; j += 32) part += st[j] * gt[1 + j];
+  float sv[KC], gv[KC];
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-  float zc[3];  // dL/dz_c for c = lane + 32 u
-#pragma unroll
-  for (int u = 0; u < 3; ++u) {
-    const int c = lane + 32 * u;
-    float v = 0.f;
-    if (c == 0) {
-      if (adaptive && tau < 0.5f) {
-        const float sg = (alpha[t] - tau) / (1.0f - 2.0f * tau);
-        v = gt[0] * (1.0f - 2.0f * tau) * sg * (1.0f - sg);
-      }
-    } else if (c < K1) {
-      v = st[c - 1] * (gt[c] - part);
-    }
-    zc[u] = v;
-    if (c < K1) dzt[c] = v;
+  for (int j = 0; j < KC; ++j) {
+    sv[j] = valid && j < K ? st[j] : 0.f;
+    gv[j] = valid && j < K1 ? gt[j] : 0.f;
   }
-  float* dxt = dx + (size_t)t * d;
-  for (int i0 = 0; i0 < d; i0 += 32) {
-    const int i = i0 + lane;
-    float acc = 0.f;
-    for (int c = 0; c < K1; ++c) {
-      const float zv = __shfl_sync(0xffffffffu, zc[c >> 5], c & 31);
-      if (i < d) acc = fmaf(zv, wrT[(size_t)c * d + i], acc);
+  const float al = valid ? alpha[t] : 0.f;
+  float part = 0.f;
+#pragma unroll
+  for (int j = 0; j + 1 < KC; ++j) part += sv[j] * gv[1 + j];
+  z[0] = 0.f;
+  if (valid && adaptive && tau < 0.5f) {
+    const float sg = (al - tau) / (1.0f - 2.0f * tau);
+    z[0] = gv[0] * (1.0f - 2.0f * tau) * sg * (1.0f - sg);
+  }
+#pragma unroll
+  for (int j = 0; j + 1 < KC; ++j) z[1 + j] = sv[j] * (gv[1 + j] - part);
+}
+
+// dL/dz of every token into dz [T][K+1] (a thread per token).
+template <int KC>
+__global__ void __launch_bounds__(256)
+router_dz_kernel(int T, int K, float tau, int adaptive, const uint8_t* __restrict__ mask,
+                 const float* __restrict__ alpha, const float* __restrict__ s,
+                 const float* __restrict__ dwt, float* __restrict__ dz) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  float z[KC];
+  router_token_dz<KC>(t, K, tau, adaptive, mask, alpha, s, dwt, z);
+  float* o = dz + (size_t)t * (K + 1);
+#pragma unroll
+  for (int c = 0; c < KC; ++c)
+    if (c <= K) o[c] = z[c];
+}
+
+// dx[t][8 f .. 8 f + 8) += sum_c dL/dz_c(t) W*^T[c][8 f .. 8 f + 8) for the
+// two tokens t = 2 p, 2 p + 1: a thread per (token pair, 8 features), so that
+// each W*^T load serves both tokens. W*^T is the router's first K+1 columns
+// as fp32 [K+1][d]; d % 128 == 0; padding tokens have dL/dz = 0 and keep dx.
+__global__ void __launch_bounds__(256)
+router_dx_kernel(int T, int K1, int d, const float* __restrict__ dz,
+                 const float* __restrict__ wrT, float* __restrict__ dx) {
+  const int per = d / 8;
+  const int n = ((T + 1) / 2) * per;
+  for (int it = blockIdx.x * blockDim.x + threadIdx.x; it < n; it += gridDim.x * blockDim.x) {
+    const int p = it / per, f8 = it - p * per;
+    const int ta = 2 * p, tb = min(2 * p + 1, T - 1);  // (tb == ta: the last odd token)
+    float4* pa = reinterpret_cast<float4*>(dx + (size_t)ta * d + 8 * f8);
+    float4* pb = reinterpret_cast<float4*>(dx + (size_t)tb * d + 8 * f8);
+    const float4 xa0 = pa[0], xa1 = pa[1], xb0 = pb[0], xb1 = pb[1];  // added at the end
+    const float* za = dz + (size_t)ta * K1;
+    const float* zb = dz + (size_t)tb * K1;
+    float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f), a1 = a0, b0 = a0, b1 = a0;
+    // four columns at a time: their loads go out together
+    for (int cb = 0; cb < K1; cb += 4) {
+      float4 w0[4], w1[4];
+      float u[4], v[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int c = cb + k;
+        if (c < K1) {
+          const float4* wc = reinterpret_cast<const float4*>(wrT + (size_t)c * d + 8 * f8);
+          w0[k] = wc[0];
+          w1[k] = wc[1];
+          u[k] = za[c];
+          v[k] = zb[c];
+        } else {
+          w0[k] = w1[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+          u[k] = v[k] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        a0.x = fmaf(u[k], w0[k].x, a0.x); a0.y = fmaf(u[k], w0[k].y, a0.y);
+        a0.z = fmaf(u[k], w0[k].z, a0.z); a0.w = fmaf(u[k], w0[k].w, a0.w);
+        a1.x = fmaf(u[k], w1[k].x, a1.x); a1.y = fmaf(u[k], w1[k].y, a1.y);
+        a1.z = fmaf(u[k], w1[k].z, a1.z); a1.w = fmaf(u[k], w1[k].w, a1.w);
+        b0.x = fmaf(v[k], w0[k].x, b0.x); b0.y = fmaf(v[k], w0[k].y, b0.y);
+        b0.z = fmaf(v[k], w0[k].z, b0.z); b0.w = fmaf(v[k], w0[k].w, b0.w);
+        b1.x = fmaf(v[k], w1[k].x, b1.x); b1.y = fmaf(v[k], w1[k].y, b1.y);
+        b1.z = fmaf(v[k], w1[k].z, b1.z); b1.w = fmaf(v[k], w1[k].w, b1.w);
+      }
     }
-    if (i < d) dxt[i] += acc;
+    a0.x += xa0.x; a0.y += xa0.y; a0.z += xa0.z; a0.w += xa0.w;
+    a1.x += xa1.x; a1.y += xa1.y; a1.z += xa1.z; a1.w += xa1.w;
+    b0.x += xb0.x; b0.y += xb0.y; b0.z += xb0.z; b0.w += xb0.w;
+    b1.x += xb1.x; b1.y += xb1.y; b1.z += xb1.z; b1.w += xb1.w;
+    pa[0] = a0;
+    pa[1] = a1;
+    if (tb != ta) {
+      pb[0] = b0;
+      pb[1] = b1;
+    }
   }
 }
 
-
-// The block's warps take tokens in turn; W*^T is staged in shared memory
-// when it fits (wrT_smem), else read from global memory.
+// dL/dW*[i][c] = sum_t x[t][i] dL/dz_c(t) and dL/dbias[c] = sum_t dL/dz_c(t):
+// block (fc, j, cc) takes features [128 fc, 128 fc + 128), the tokens of
+// slice j (kRwSlice tokens) and columns [16 cc, 16 cc + 16); 32 tokens at a
+// time, the tile of x (16-byte loads; zero rows for padding tokens, whose x
+// may hold anything) and of dL/dz go to shared memory (the next tile's
+// loads run while the current tile is summed), then thread (g, q)
+// adds x[t][2 q .. 2 q + 2) times dL/dz_{16 cc + 4 g .. + 4}(t) into its
+// 2 x 4 partial sums (one 4-byte and one 16-byte shared load per 8 FMAs),
+// which go out with one atomic add each.
+constexpr int kRwSlice = 128;
 __global__ void __launch_bounds__(256)
-router_grad_kernel(int T, int K, int d, float tau, int adaptive,
-                   const uint8_t* __restrict__ mask, const float* __restrict__ alpha,
-                   const float* __restrict__ s, const float* __restrict__ dwt,
-                   const float* __restrict__ wrT_g, float* __restrict__ dz,
-                   float* __restrict__ dx, int wrT_smem) {
-  extern __shared__ float wrT_s[];
-  const int K1 = K + 1;
-  if (wrT_smem) {
-    for (int k = threadIdx.x; k < K1 * d; k += blockDim.x) wrT_s[k] = wrT_g[k];
+router_dw_kernel(int T, int K1, int d, const uint8_t* __restrict__ mask,
+                 const __nv_bfloat16* __restrict__ x, const float* __restrict__ dz,
+                 float* __restrict__ dw_router, float* __restrict__ dbias) {
+  __shared__ __align__(16) __nv_bfloat16 xs[32][128];
+  __shared__ __align__(16) float zs[32][16];
+  const int i0 = blockIdx.x * 128, c0 = blockIdx.z * 16;
+  const int t_begin = blockIdx.y * kRwSlice, t_end = min(T, t_begin + kRwSlice);
+  const int q = threadIdx.x & 63, g = threadIdx.x >> 6;
+  const int lq = threadIdx.x & 15, lr = threadIdx.x >> 4;
+  float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+  float bacc[4] = {0.f, 0.f, 0.f, 0.f};
+  // this thread's share of a tile: 16-byte chunk lq of x rows lr, lr + 16
+  // and column c0 + lq of dL/dz for the same two tokens; the next tile's
+  // share is loaded into registers while the current one is summed
+  uint4 xr[2];
+  float zr[2];
+  auto load = [&](int tt) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int t = tt + lr + 16 * k, c = c0 + lq;
+      xr[k] = make_uint4(0u, 0u, 0u, 0u);
+      if (t < t_end && (!mask || mask[t]))
+        xr[k] = reinterpret_cast<const uint4*>(x + (size_t)t * d + i0)[lq];
+      zr[k] = t < t_end && c < K1 ? dz[(size_t)t * K1 + c] : 0.f;
+    }
+  };
+  load(t_begin);
+  for (int tt = t_begin; tt < t_end; tt += 32) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      reinterpret_cast<uint4*>(&xs[lr + 16 * k][0])[lq] = xr[k];
+      zs[lr + 16 * k][lq] = zr[k];
+    }
+    __syncthreads();
+    if (tt + 32 < t_end) load(tt + 32);
+    const int nr = min(32, t_end - tt);
+    for (int r = 0; r < nr; ++r) {
+      const float2 xv = __bfloat1622float2(reinterpret_cast<const __nv_bfloat162*>(&xs[r][0])[q]);
+      const float4 z = reinterpret_cast<const float4*>(&zs[r][0])[g];
+      acc[0][0] = fmaf(xv.x, z.x, acc[0][0]); acc[0][1] = fmaf(xv.x, z.y, acc[0][1]);
+      acc[0][2] = fmaf(xv.x, z.z, acc[0][2]); acc[0][3] = fmaf(xv.x, z.w, acc[0][3]);
+      acc[1][0] = fmaf(xv.y, z.x, acc[1][0]); acc[1][1] = fmaf(xv.y, z.y, acc[1][1]);
+      acc[1][2] = fmaf(xv.y, z.z, acc[1][2]); acc[1][3] = fmaf(xv.y, z.w, acc[1][3]);
+      if (q == 0) {
+        bacc[0] += z.x; bacc[1] += z.y; bacc[2] += z.z; bacc[3] += z.w;
+      }
+    }
     __syncthreads();
   }
-  const float* wrT = wrT_smem ? wrT_s : wrT_g;
-  const int lane = threadIdx.x & 31;
-  const int warps = gridDim.x * (blockDim.x >> 5);
-  for (int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); t < T; t += warps)
-    router_grad_token(t, K, d, tau, adaptive, mask, alpha, s, dwt, wrT, dz, dx, lane);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int c = c0 + 4 * g + e;
+    if (c < K1) {
+      atomicAdd(dw_router + (size_t)(i0 + 2 * q) * K1 + c, acc[0][e]);
+      atomicAdd(dw_router + (size_t)(i0 + 2 * q + 1) * K1 + c, acc[1][e]);
+      if (dbias && blockIdx.x == 0 && q == 0) atomicAdd(dbias + c, bacc[e]);
+    }
+  }
 }
 
 // W*^T: the router's first K+1 columns (fp32 [d][Cp]) as [K+1][d].
@@ -635,62 +741,6 @@ __global__ void router_transpose_kernel(int K1, int d, int Cp, const float* __re
   if (k < K1 * d) {
     const int c = k / d, i = k % d;
     wrT[k] = wr[(size_t)i * Cp + c];
-  }
-}
-
-// dL/dW*[i][c] = sum_t x[t][i] dL/dz[t][c] and dL/dbias[c] = sum_t dL/dz[t][c]:
-// block (32 features x 8 token lanes) of one token slice; the 8 lanes'
-// partial sums are added in shared memory, then once per block into the
-// outputs (which start at zero).
-constexpr int kRgSlices = 128;
-__global__ void __launch_bounds__(256)
-router_wgrad_kernel(int T, int K1, int d, const uint8_t* __restrict__ mask,
-                    const __nv_bfloat16* __restrict__ x, const float* __restrict__ dz,
-                    float* __restrict__ dw_router, float* __restrict__ dbias) {
-  __shared__ float red[8][32][17];
-  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-  const int i = blockIdx.x * 32 + tx;
-  const int per = (T + gridDim.y - 1) / gridDim.y;
-  const int t_begin = blockIdx.y * per, t_end = min(T, t_begin + per);
-  for (int c0 = 0; c0 < K1; c0 += 16) {
-    float acc[16], bacc[16];
-#pragma unroll
-    for (int u = 0; u < 16; ++u) acc[u] = bacc[u] = 0.f;
-    for (int t = t_begin + ty; t < t_end; t += 8) {
-      if (mask && !mask[t]) continue;
-      const float xv = i < d ? __bfloat162float(x[(size_t)t * d + i]) : 0.f;
-      const float* zt = dz + (size_t)t * K1 + c0;
-#pragma unroll
-      for (int u = 0; u < 16; ++u)
-        if (c0 + u < K1) {
-          const float zv = zt[u];
-          acc[u] = fmaf(xv, zv, acc[u]);
-          bacc[u] += zv;
-        }
-    }
-#pragma unroll
-    for (int u = 0; u < 16; ++u) red[ty][tx][u] = acc[u];
-    __syncthreads();
-    if (ty == 0 && i < d) {
-      for (int u = 0; u < 16 && c0 + u < K1; ++u) {
-        float v = 0.f;
-#pragma unroll
-        for (int w = 0; w < 8; ++w) v += red[w][tx][u];
-        atomicAdd(dw_router + (size_t)i * K1 + c0 + u, v);
-      }
-    }
-    __syncthreads();
-    if (dbias && blockIdx.x == 0) {  // the bias sums, from lane 0 of each token lane
-#pragma unroll
-      for (int u = 0; u < 16; ++u) red[ty][tx][u] = tx == 0 ? bacc[u] : 0.f;
-      __syncthreads();
-      if (threadIdx.x < 16 && c0 + (int)threadIdx.x < K1) {
-        float v = 0.f;
-        for (int w = 0; w < 8; ++w) v += red[w][0][threadIdx.x];
-        atomicAdd(dbias + c0 + threadIdx.x, v);
-      }
-      __syncthreads();
-    }
   }
 }
 
@@ -781,7 +831,7 @@ int backward_setup(unif_moe_layer* L) {
   if (cudaFuncSetAttribute(bwd_hidden_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)L->bwd_hidden_smem) != cudaSuccess ||
       cudaFuncSetAttribute(bwd_wgrad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)L->bwd_wgrad_smem) != cudaSuccess) {
+                           (int)L->bwd_wgrad_smem) != cudaSuccess ) {
     set_error("cudaFuncSetAttribute failed for the backward kernels");
     return UNIF_MOE_ERR_CUDA;
   }
@@ -857,20 +907,32 @@ int backward_run(unif_moe_layer* L, const void* x, const void* dy, int T, const 
     bwd_wgrad_kernel<<<L->n_sm, kThreads, L->bwd_wgrad_smem, s>>>(L->tm_da_q, L->tm_hw_q, p);
     CKB(cudaGetLastError());
   }
-  // router: W*^T, dL/dz, its share of dL/dx, dL/dW*, dL/dbias
+  // router: W*^T, then dL/dz, its share of dL/dx, dL/dW* and dL/dbias
   router_transpose_kernel<<<(K1 * L->d + 255) / 256, 256, 0, s>>>(K1, L->d, L->router_cols_pad,
                                                                    L->wr, w.wrT);
   CKB(cudaGetLastError());
-  const int adaptive = isnan(L->th.alpha_fixed) ? 1 : 0;
-  const size_t wrT_bytes = sizeof(float) * (size_t)K1 * L->d;
-  const int wrT_smem = wrT_bytes <= 48 * 1024 ? 1 : 0;
-  const int rg_blocks = min((T + 7) / 8, L->n_sm * 8);
-  router_grad_kernel<<<rg_blocks, 256, wrT_smem ? wrT_bytes : 0, s>>>(
-      T, L->K, L->d, L->tau, adaptive, mask, w.alpha, w.s, w.dwt, w.wrT, w.dz, dx, wrT_smem);
-  CKB(cudaGetLastError());
-  router_wgrad_kernel<<<dim3((L->d + 31) / 32, kRgSlices), 256, 0, s>>>(
-      T, K1, L->d, mask, static_cast<const __nv_bfloat16*>(x), w.dz, dw_router, dbias);
-  CKB(cudaGetLastError());
+  {
+    const int adaptive = isnan(L->th.alpha_fixed) ? 1 : 0;
+    const int dz_blocks = (T + 255) / 256;
+    if (K1 <= 16)
+      router_dz_kernel<16><<<dz_blocks, 256, 0, s>>>(T, L->K, L->tau, adaptive, mask, w.alpha,
+                                                     w.s, w.dwt, w.dz);
+    else if (K1 <= 32)
+      router_dz_kernel<32><<<dz_blocks, 256, 0, s>>>(T, L->K, L->tau, adaptive, mask, w.alpha,
+                                                     w.s, w.dwt, w.dz);
+    else
+      router_dz_kernel<65><<<dz_blocks, 256, 0, s>>>(T, L->K, L->tau, adaptive, mask, w.alpha,
+                                                     w.s, w.dwt, w.dz);
+    CKB(cudaGetLastError());
+    const int items = (T + 1) / 2 * (L->d / 8);
+    router_dx_kernel<<<std::min((items + 255) / 256, 8 * L->n_sm), 256, 0, s>>>(T, K1, L->d,
+                                                                                 w.dz, w.wrT, dx);
+    CKB(cudaGetLastError());
+    router_dw_kernel<<<dim3(L->d / 128, (T + kRwSlice - 1) / kRwSlice, (K1 + 15) / 16), 256, 0,
+                       s>>>(T, K1, L->d, mask, static_cast<const __nv_bfloat16*>(x), w.dz,
+                            dw_router, dbias);
+    CKB(cudaGetLastError());
+  }
   if (lambda_div != 0.f || l_div) {
     gram_kernel<<<K1 * K1, 128, 0, s>>>(K1, L->d, w.wrT, w.gram);
     CKB(cudaGetLastError());

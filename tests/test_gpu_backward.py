@@ -117,6 +117,13 @@ def test_backward_router_bias_many_experts():
     check(wl, got, ref)
 
 
+def test_backward_sixteen_experts():
+    """K = 16 residual experts (17 router columns, as ViT-B's layer), 300
+    tokens: the router gradients' kernel instance for up to 32 columns."""
+    wl, got, ref, _ = run_case(small(tokens=300, n_experts=16))
+    check(wl, got, ref)
+
+
 def test_backward_gram_regulariser():
     """lambda_div = 0.01 (the paper's choice): dW* gains lambda dL_div/dW*,
     and L_div itself is returned."""
