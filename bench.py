@@ -275,6 +275,9 @@ def main():
     ap.add_argument("--workload", default="vit_s")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--gemm-kernels", default="auto",
+                    choices=["auto", "grouped", "streaming", "expert_tile"],
+                    help="expert GEMM kernel family (unif_moe_options.gemm_kernels)")
     ap.add_argument("--routing", default="adaptive", choices=sorted(ROUTINGS),
                     help="routing variant (Table IV ablations, fixed thresholds)")
     ap.add_argument("--train", action="store_true",
@@ -323,7 +326,8 @@ def main():
     layer = Layer(s.d_model, s.d_ff, s.n_experts, s.n_blocks, dtype=s.dtype, max_tokens=T,
                   tau=s.tau, alpha_fixed=s.alpha_fixed, beta_fixed=s.beta_fixed,
                   topk_fixed=s.topk_fixed, prefix_blocks=s.prefix_blocks,
-                  features=FEATURES_DEFAULT | (FEATURE_BACKWARD if args.train else 0))
+                  features=FEATURES_DEFAULT | (FEATURE_BACKWARD if args.train else 0),
+                  gemm_kernels=args.gemm_kernels)
     layer.load_weights(w_router.to(dev), w_up.to(dev), w_down.to(dev),
                        None if bias is None else bias.to(dev))
     xd = x.to(dev)
@@ -498,8 +502,19 @@ def main():
     hbm_nominal = 8000.0
     # roofline of the dominant kernel (the larger grouped GEMM), timed in the
     # per-kernel pass
-    dom = "up_gemm" if stage_ms["up_gemm"] >= stage_ms["down_gemm"] else "down_gemm"
-    ach = stage_flops / (stage_ms[dom] / 1e3) / 1e12
+    # the expert-tile FFN (three kernels per forward) runs both projections
+    # in one launch: its stage is the up stage (the down stage is the empty
+    # gap between two events), its work the activated flops of both
+    # projections, 4 d M C_B per token (Eq. 35); the masked blocks it also
+    # computes are not counted
+    expert_tile = layer.kernels_per_forward() == 3
+    if expert_tile:
+        dom = "ffn"
+        ffn_ms = stage_ms["up_gemm"] + stage_ms["down_gemm"]
+        ach = 2.0 * stage_flops / (ffn_ms / 1e3) / 1e12
+    else:
+        dom = "up_gemm" if stage_ms["up_gemm"] >= stage_ms["down_gemm"] else "down_gemm"
+        ach = stage_flops / (stage_ms[dom] / 1e3) / 1e12
     traffic = measured_traffic(s.name, dom)
     # algorithmic bytes of the memory-bound kernels (per forward): the router
     # reads x and writes each token's records (alpha, b, k, two masks, K
@@ -507,8 +522,15 @@ def main():
     # one (token, weight) row per pair; the permute writes those rows; the
     # combine reads the fp32 accumulator and writes the output
     fused = layer.kernels_per_forward() <= 5 and s.dtype == "bf16"
+    # (grouped by expert: one row per (token, expert), 1[b > 0] + k per token)
+    n_rows_last = cb_last
+    if expert_tile:
+        rows_t = (b_h > 0).long() + k_h
+        if mask is not None:
+            rows_t = rows_t * mask.long()
+        n_rows_last = int(rows_t[last0:].sum())
     router_bytes = (T_last * d * elt + T_last * (4 * 3 + 8 * 2 + 4 * s.n_experts + 8) +
-                    (8 * cb_last if fused else 0))
+                    (8 * n_rows_last if fused else 0))
     combine_bytes = T_last * d * (4 + elt)
     permute_bytes = cb_last * 8
 
@@ -521,11 +543,16 @@ def main():
         "router": hbm_stage(stage_ms["router"], router_bytes),
         "permute": (hbm_stage(stage_ms["permute"], permute_bytes) if not fused else
                     {"ms": 0.0, "fused_into": "router", "event_gap_ms": stage_ms["permute"]}),
-        "up_gemm": {"ms": stage_ms["up_gemm"], "TFLOP/s": stage_flops / stage_ms["up_gemm"] / 1e9,
-                    "frac_of_burst_bf16": stage_flops / stage_ms["up_gemm"] / 1e9 / peak_tf},
-        "down_gemm": {"ms": stage_ms["down_gemm"],
-                      "TFLOP/s": stage_flops / stage_ms["down_gemm"] / 1e9,
-                      "frac_of_burst_bf16": stage_flops / stage_ms["down_gemm"] / 1e9 / peak_tf},
+        **({"ffn": {"ms": ffn_ms, "TFLOP/s": ach, "frac_of_burst_bf16": ach / peak_tf,
+                    "kernel": "expert-tile FFN (both projections, rows grouped by expert)",
+                    "event_gap_ms": stage_ms["down_gemm"]}} if expert_tile else {
+            "up_gemm": {"ms": stage_ms["up_gemm"],
+                        "TFLOP/s": stage_flops / stage_ms["up_gemm"] / 1e9,
+                        "frac_of_burst_bf16": stage_flops / stage_ms["up_gemm"] / 1e9 / peak_tf},
+            "down_gemm": {"ms": stage_ms["down_gemm"],
+                          "TFLOP/s": stage_flops / stage_ms["down_gemm"] / 1e9,
+                          "frac_of_burst_bf16":
+                              stage_flops / stage_ms["down_gemm"] / 1e9 / peak_tf}}),
         "timed_pass": {"passes_per_forward": n_pass, "pass_tokens": P,
                        "tokens": [last0, T]},
         "combine": hbm_stage(stage_ms["combine"], combine_bytes),

@@ -91,15 +91,29 @@ enum {
   UNIF_MOE_FEATURES_DEFAULT = 3,   /* what unif_moe_create allocates */
   UNIF_MOE_FEATURES_ALL = 15
 };
-/* Grouped GEMM kernels: the library picks the weight-stationary kernels
- * where a group's weight slice fits in shared memory, else the streaming
- * ones (AUTO); STREAMING always takes the streaming ones (both compute the
- * same products; the fp32 sums into the output differ only in order). */
-enum { UNIF_MOE_GEMM_AUTO = 0, UNIF_MOE_GEMM_STREAMING = 1 };
+/* Expert GEMM kernels (all compute the same products; the fp32 sums into
+ * the output differ only in order):
+ * - EXPERT_TILE: rows grouped by expert, both projections of Eq. 16 in one
+ *   kernel with h kept on chip, each (token, expert) added into the output
+ *   once; bf16, d a multiple of 128 up to 384, H a multiple of 128, M a
+ *   multiple of 64, a handle without UNIF_MOE_FEATURE_BACKWARD (otherwise
+ *   as GROUPED).
+ * - GROUPED: rows grouped by (expert, block) pair (Eq. 35's C_B pairs per
+ *   token), an up and a down projection kernel with h in device memory;
+ *   weight-stationary kernels where a group's weight slice fits in shared
+ *   memory, else the streaming ones.
+ * - STREAMING: as GROUPED, always the streaming kernels.
+ * - AUTO: GROUPED. */
+enum {
+  UNIF_MOE_GEMM_AUTO = 0,
+  UNIF_MOE_GEMM_STREAMING = 1,
+  UNIF_MOE_GEMM_GROUPED = 2,
+  UNIF_MOE_GEMM_EXPERT_TILE = 3
+};
 
 typedef struct {
   unsigned int features; /* UNIF_MOE_FEATURE_* bits */
-  int gemm_kernels;      /* UNIF_MOE_GEMM_AUTO or UNIF_MOE_GEMM_STREAMING */
+  int gemm_kernels;      /* UNIF_MOE_GEMM_AUTO, _STREAMING, _GROUPED, _EXPERT_TILE */
 } unif_moe_options;
 
 /* Fills *opts with the defaults of unif_moe_create: UNIF_MOE_FEATURES_DEFAULT

@@ -60,7 +60,7 @@ class Options(C.Structure):
 
 FEATURE_NORM_FIRST, FEATURE_HOST_IO, FEATURE_BACKWARD, FEATURE_DIAGNOSTICS = 1, 2, 4, 8
 FEATURES_DEFAULT, FEATURES_ALL = 3, 15
-GEMM_KERNELS = {"auto": 0, "streaming": 1}
+GEMM_KERNELS = {"auto": 0, "streaming": 1, "grouped": 2, "expert_tile": 3}
 
 
 _lib = None
@@ -132,8 +132,11 @@ class Layer:
     """One UniF-MoE layer (Sec. III): K residual experts plus one shared
     expert, FFN width H split into B blocks. dtype "bf16" (tensor cores) or
     "f32" (CUDA-core FMA). `features` (FEATURE_* bits) picks the optional
-    workspaces allocated at create time; `gemm_kernels` "auto" or
-    "streaming"."""
+    workspaces allocated at create time; `gemm_kernels` "grouped" ((expert,
+    block) groups, weight-stationary kernels where they fit), "streaming"
+    ((expert, block) groups, streaming kernels), "expert_tile" (rows grouped
+    by expert, both projections in one kernel, where it applies) or "auto"
+    (as "grouped")."""
 
     def __init__(self, d_model: int, d_ff: int, n_experts: int, n_blocks: int,
                  dtype: str = "bf16", max_tokens: int = 65536, tau: float = math.nan,

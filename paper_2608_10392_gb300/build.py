@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 LIBDIR = os.path.join(HERE, "lib")
 LIB = os.path.join(LIBDIR, "libunif_moe.so")
 SOURCES = ["unif_moe.cu", "route_permute.cu", "gemm_simt.cu", "gemm_tc.cu", "gemm_ws.cu",
-           "backward.cu", "diagnostics.cu"]
+           "backward.cu", "diagnostics.cu", "gemm_fused.cu"]
 HEADERS = ["internal.cuh", "decide.cuh", "tc_common.cuh", os.path.join("..", "..", "include", "unif_moe.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -433,6 +433,80 @@ __device__ void group_rows(const GroupArgs& a, int tid, int t0, uint64_t shr, ui
   }
 }
 
+// Expert-major grouping (the fused expert-tile FFN): group e = expert e
+// (G = K + 1), one row per (token, expert) the token runs: the shared expert
+// for every token with b > 0 (weight alpha, Eq. 28), each selected residual
+// expert j (weight s_j, Eq. 29). The blocks a row runs follow from the
+// token's shared block set (expert_blocks). Lane masks: masks[0] = lanes
+// with b > 0, masks[64 + j] = lanes selecting residual expert j; counts
+// out[e * stride] per expert.
+__device__ __forceinline__ void count_chunk_experts(int K, int lane, uint64_t shr, uint64_t em,
+                                                    uint32_t* scratch, int32_t* out, int stride) {
+  const uint32_t m0 = __ballot_sync(0xffffffffu, shr != 0ull);
+  if (lane == 0) scratch[0] = m0;
+  for (int e = 0; e < K; ++e) {
+    const uint32_t m = __ballot_sync(0xffffffffu, (em >> e) & 1ull);
+    if (lane == 0) scratch[64 + e] = m;
+  }
+  __syncwarp();
+  for (int g = lane; g <= K; g += 32)
+    out[(size_t)g * stride] = __popc(g == 0 ? scratch[0] : scratch[64 + g - 1]);
+  __syncwarp();
+}
+
+// group_rows for the expert-major grouping (the same reservation, then each
+// thread writes its token's 1 + k rows; arguments as group_rows, G = K + 1).
+template <int NW>
+__device__ void group_rows_expert(const GroupArgs& a, int tid, int t0, uint64_t shr, uint64_t em,
+                                  const uint32_t* masks, const float* dec_s, int dec_stride,
+                                  int32_t* sm, uint32_t bar) {
+  constexpr int NT = NW * 32;
+  const int G = a.G;
+  int32_t* first = sm;
+  for (int g = tid; g < G; g += NT) {
+    int n = 0;
+#pragma unroll
+    for (int v = 0; v < NW; ++v) n += first[v * G + g];
+    int base = -1;
+    if (n > 0) {
+      base = atomicAdd(a.fill + g, n);
+      if (base + n > a.region) {
+        atomicOr(a.status, kStatusBadIndex);
+        base = -1;
+      }
+    }
+    int o = base < 0 ? -(1 << 30) : base;
+#pragma unroll
+    for (int v = 0; v < NW; ++v) {
+      const int c = first[v * G + g];
+      first[v * G + g] = o;
+      o += c;
+    }
+  }
+  named_bar(bar, NT);
+  const int c = tid >> 5;
+  const uint32_t lt = (1u << (tid & 31)) - 1u;
+  const int32_t* fc = first + c * G;
+  const uint32_t* mk = masks + c * 128;
+  const float* ds = dec_s + tid * dec_stride;
+  const int tok = t0 + tid;
+  if (shr != 0ull) {
+    const int r = fc[0] + __popc(mk[0] & lt);
+    if (r >= 0) {
+      a.row_tok[r] = tok;
+      a.row_w[r] = ds[2 * a.K];
+    }
+  }
+  for (uint64_t rj = em; rj != 0ull; rj &= rj - 1ull) {
+    const int j = __ffsll((long long)rj) - 1;
+    const int r = fc[j + 1] + __popc(mk[64 + j] & lt);
+    if (r >= 0) {
+      a.row_tok[(size_t)(j + 1) * a.region + r] = tok;
+      a.row_w[(size_t)(j + 1) * a.region + r] = ds[j];
+    }
+  }
+}
+
 // The tiles of the groups whose sizes are fill[0..G) (each clamped to the
 // region): first_s[g] = first tile of group g (first_s[G] = all tiles),
 // cnt_s[g] = its size. Run by one warp; shared arrays of G + 1 and G ints.

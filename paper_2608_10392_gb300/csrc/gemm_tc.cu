@@ -389,7 +389,8 @@ __host__ __device__ constexpr int router_overlay_bytes(int Cp, int K, int G, boo
 struct RouterTcParams {
   DecideArgs dec;
   GroupArgs grp;
-  int fused;     // 1: the router also lays out the group rows (group_rows)
+  int fused;     // 1: the router also lays out the group rows by (expert, block)
+                 // (group_rows); 2: by expert (group_rows_expert)
   int d, Cp;
   uint32_t tmem_cols;
   int* status;
@@ -508,7 +509,10 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
       } else {
         // per-chunk counts stay in shared memory (chunk q = tokens
         // 32 q .. 32 q + 31 of this CTA); alpha joins the affinities
-        count_chunk_pairs(p.dec, lane, shr, em, cscr + q * 128, gsm + q * G, 1);
+        if (p.fused == 2)
+          count_chunk_experts(K, lane, shr, em, cscr + q * 128, gsm + q * G, 1);
+        else
+          count_chunk_pairs(p.dec, lane, shr, em, cscr + q * 128, gsm + q * G, 1);
         sv[2 * K] = alpha;
       }
     }
@@ -518,7 +522,12 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
       named_bar(1, 128);
       if (row == 0) misc_s[7] = *abort_flag;  // one reading for all four warps
       named_bar(1, 128);
-      if (!misc_s[7]) group_rows<4>(p.grp, row, t0, shr, em, cscr, ss, 2 * K + 1, gsm, 1);
+      if (!misc_s[7]) {
+        if (p.fused == 2)
+          group_rows_expert<4>(p.grp, row, t0, shr, em, cscr, ss, 2 * K + 1, gsm, 1);
+        else
+          group_rows<4>(p.grp, row, t0, shr, em, cscr, ss, 2 * K + 1, gsm, 1);
+      }
     }
   }
   __syncwarp();  // every warp converged before the CTA barrier
@@ -625,13 +634,18 @@ int gemm_tc_setup(unif_moe_layer* L) {
     return UNIF_MOE_ERR_CUDA;
   }
   const int rc = gemm_ws_setup(L);
-  L->tile_list = L->fused_group && !(L->up_ws && L->down_ws);
+  L->tile_list = L->fused_group && !L->ffn_fused && !(L->up_ws && L->down_ws);
   return rc;
 }
 
 cudaError_t launch_gemms_tc(unif_moe_layer* L, const void* x, int T, cudaEvent_t mid,
                             cudaStream_t s) {
   (void)T;
+  if (L->ffn_fused) {  // both projections in one kernel (the down stage takes no time)
+    cudaError_t e = launch_ffn_fused(L, x, s);
+    if (e == cudaSuccess && mid) e = cudaEventRecord(mid, s);
+    return e;
+  }
   tc::Params p;
   p.n_tiles = L->ws.n_tiles; p.tile_group = L->ws.tile_group; p.tile_row0 = L->ws.tile_row0;
   p.tile_rows = L->ws.tile_rows;
@@ -712,11 +726,11 @@ cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* ma
   if (!tc::encode_2d(&tm_x, x, L->d, (uint64_t)T, tc::kBK, tc::kBM)) return cudaErrorInvalidValue;
   tc::RouterTcParams p;
   p.dec = decide_args(L, mask, T, b_out, k_out);
-  p.fused = L->fused_group ? 1 : 0;
+  p.fused = L->fused_group ? (L->ffn_fused ? 2 : 1) : 0;
   if (L->fused_group) {
     Workspace& w = L->ws;
     GroupArgs& g = p.grp;
-    g.G = L->G; g.K = L->K; g.B = L->B;
+    g.G = L->ffn_fused ? L->K + 1 : L->G; g.K = L->K; g.B = L->B;
     g.region = L->region_rows;
     g.fill = w.grp_fill;
     g.row_tok = w.row_tok; g.row_w = w.row_w;

@@ -73,6 +73,9 @@ struct Workspace {
   // output accumulator.
   void* hbuf = nullptr;          // [max_rows][M] (layer dtype)
   float* y32 = nullptr;          // [max_tokens][d]
+  // Expert weights repacked into the expert-tile FFN's 16 KB operand slabs.
+  void* wk_slabs = nullptr;      // K_e: [K+1][H/128][d/64] slabs
+  void* wv_slabs = nullptr;      // V_e: [K+1][H/128][2][d/128] slabs
   // Host-buffer forward staging.
   void* xn = nullptr;             // [max_tokens][d] LN(x) of a norm-first sublayer
   // Staging buffers of the host-buffer forwards, two slots (the pipelined
@@ -157,6 +160,11 @@ struct unif_moe_layer {
   // number of output column slices run as separate work items
   int ws_down_bn = 0, ws_down_nsub = 0, down_slices = 1;
   CUtensorMap tm_wdown_ws;  // w_down slabs of ws_down_bn rows
+  // Expert-tile FFN (both projections in one kernel, rows grouped by
+  // expert): its weight maps (128 x 64 slabs), shared memory and ring depth.
+  bool ffn_fused = false;
+  int ffn_per_cta = 0, ffn_slots = 0;
+  uint32_t ffn_smem = 0;
   // backward: transposed weights and the per-row gradient buffers
   CUtensorMap tm_wdownT;    // w_downT [(K+1) H][d], boxes of 64 x up_bn
   CUtensorMap tm_wupT;      // w_upT [(K+1) d][H], boxes of 64 x down_bn
@@ -212,6 +220,10 @@ cudaError_t launch_timeout_probe(unif_moe_layer* L, int timeout_us, cudaStream_t
 int gemm_ws_setup(unif_moe_layer* L);  // picks the weight-stationary kernels where they fit
 cudaError_t launch_up_ws(unif_moe_layer* L, const void* x, cudaStream_t s);
 cudaError_t launch_down_ws(unif_moe_layer* L, cudaStream_t s);
+bool ffn_fused_fits(int d, int H, int M);
+int gemm_fused_setup(unif_moe_layer* L);  // the expert-tile FFN's maps and shared memory
+cudaError_t launch_ffn_fused(unif_moe_layer* L, const void* x, cudaStream_t s);
+cudaError_t launch_repack_slabs(unif_moe_layer* L, cudaStream_t s);  // after the weights load
 long long gemm_wait_limit();
 bool encode_bf16_map(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
                      uint32_t box_cols, uint32_t box_rows, int swizzle_bytes);  // clock cycles before a bounded wait gives up

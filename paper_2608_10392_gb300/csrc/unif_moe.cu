@@ -75,7 +75,7 @@ void free_all(unif_moe_layer* L) {
                   L->ws.tile_rows, L->ws.w_upT, L->ws.w_downT, L->ws.da, L->ws.hw,
                   L->ws.dwt, L->ws.dz, L->ws.wrT, L->ws.gram, L->ws.diag_sets,
                   L->ws.diag_counts, L->ws.diag_pair, L->ws.diag_wts, L->ws.diag_q,
-                  L->ws.diag_E, L->ws.diag_ES};
+                  L->ws.diag_E, L->ws.diag_ES, L->ws.wk_slabs, L->ws.wv_slabs};
   for (void* q : ptrs)
     if (q) cudaFree(q);
   for (int i = 0; i < 2; ++i) {
@@ -128,7 +128,8 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   unif_moe_default_options(&o);
   if (opts) o = *opts;
   if ((o.features & ~(unsigned)UNIF_MOE_FEATURES_ALL) != 0u ||
-      (o.gemm_kernels != UNIF_MOE_GEMM_AUTO && o.gemm_kernels != UNIF_MOE_GEMM_STREAMING)) {
+      (o.gemm_kernels != UNIF_MOE_GEMM_AUTO && o.gemm_kernels != UNIF_MOE_GEMM_STREAMING &&
+       o.gemm_kernels != UNIF_MOE_GEMM_GROUPED && o.gemm_kernels != UNIF_MOE_GEMM_EXPERT_TILE)) {
     set_error("bad options: features 0x%x, gemm_kernels %d", o.features, o.gemm_kernels);
     return UNIF_MOE_ERR_ARG;
   }
@@ -237,6 +238,10 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   L->fused_group = dtype == UNIF_MOE_BF16 && L->router_cols_pad <= 160 &&
                    unif::router_can_group(L->router_cols_pad, L->K, L->G);
   L->region_rows = (L->pass_tokens + 127) / 128 * 128;
+  // rows grouped by expert for the expert-tile FFN (where it applies; the
+  // backward pass reads the (expert, block) groups and h of a forward)
+  L->ffn_fused = L->fused_group && o.gemm_kernels == UNIF_MOE_GEMM_EXPERT_TILE &&
+                 !(o.features & UNIF_MOE_FEATURE_BACKWARD) && unif::ffn_fused_fits(d_model, d_ff, M);
   const size_t row_cap = L->fused_group ? (size_t)L->G * L->region_rows : (size_t)L->max_rows;
   ALLOC(w.row_tok, row_cap); ALLOC(w.row_w, row_cap);
   if (L->fused_group) ALLOC(w.grp_fill, (size_t)L->G);
@@ -244,6 +249,10 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&hb), es * (size_t)L->max_rows * M);
   w.hbuf = hb;
   ALLOC(w.y32, (size_t)L->pass_tokens * d_model);
+  if (L->ffn_fused) {  // the expert weights as the expert-tile FFN's operand slabs
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.wk_slabs), es * E * d_ff * d_model);
+    if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.wv_slabs), es * E * d_ff * d_model);
+  }
   ALLOC(w.status, 1);
   // optional features: every buffer a later call needs, so that no later
   // call allocates
@@ -305,6 +314,7 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
     rc = UNIF_MOE_ERR_CUDA;
   }
   if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::gemm_tc_setup(L);
+  if (rc == UNIF_MOE_OK && L->ffn_fused) rc = unif::gemm_fused_setup(L);
   if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::router_tc_setup(L);
   if (rc == UNIF_MOE_OK && (o.features & UNIF_MOE_FEATURE_BACKWARD)) rc = unif::backward_setup(L);
   if (rc != UNIF_MOE_OK) {
@@ -327,6 +337,7 @@ int unif_moe_load_weights(unif_moe_t L, const void* w_router, const void* w_up,
   CK(cudaMemcpyAsync(L->w_down, w_down, bytes, cudaMemcpyDeviceToDevice, s));
   CK(unif::launch_prototypes(L, w_router, router_bias, s));
   if (L->features & UNIF_MOE_FEATURE_BACKWARD) CK(unif::launch_transpose_weights(L, s));
+  if (L->ffn_fused) CK(unif::launch_repack_slabs(L, s));
   L->loaded = true;
   return UNIF_MOE_OK;
 }
@@ -456,6 +467,7 @@ int unif_moe_load_upcycled(unif_moe_t L, const void* w_router, const void* w_up_
   }
   CK(unif::launch_prototypes(L, w_router, router_bias, s));
   if (L->features & UNIF_MOE_FEATURE_BACKWARD) CK(unif::launch_transpose_weights(L, s));
+  if (L->ffn_fused) CK(unif::launch_repack_slabs(L, s));
   L->loaded = true;
   return UNIF_MOE_OK;
 }
@@ -740,7 +752,52 @@ int unif_moe_get_groups(unif_moe_t L, int32_t* counts, int32_t* offsets, int32_t
   if (L->last_T > 0 && !L->fused_group)
     CK(cudaMemcpyAsync(&total, L->ws.grp_off + L->G, sizeof(int32_t), dh, s));
   CK(cudaStreamSynchronize(s));
-  if (L->last_T > 0 && L->fused_group) {
+  if (L->last_T > 0 && L->ffn_fused) {
+    // the device grouped the rows by expert; the (expert, block) table of
+    // the forward's last pass follows from its routing records: token t
+    // runs blocks shr(t) of the shared expert (weight alpha) and the
+    // complementary blocks of each selected residual expert j (weight s_j)
+    const int tok_base = L->last_T - L->last_pass_T;
+    const size_t n = (size_t)L->last_pass_T, K = (size_t)L->K;
+    std::vector<float> al(n), sv(n * K);
+    std::vector<uint64_t> sh(n), em(n);
+    CK(cudaMemcpyAsync(al.data(), L->ws.alpha + tok_base, sizeof(float) * n, dh, s));
+    CK(cudaMemcpyAsync(sh.data(), L->ws.shr_mask + tok_base, sizeof(uint64_t) * n, dh, s));
+    CK(cudaMemcpyAsync(em.data(), L->ws.exp_mask + tok_base, sizeof(uint64_t) * n, dh, s));
+    CK(cudaMemcpyAsync(sv.data(), L->ws.s + (size_t)tok_base * K, sizeof(float) * n * K, dh, s));
+    CK(cudaStreamSynchronize(s));
+    const int B = L->B;
+    const uint64_t full = B >= 64 ? ~0ull : ((1ull << B) - 1ull);
+    std::vector<int32_t> cnt(L->G, 0), off(L->G + 1), pos(L->G);
+    for (int pass = 0; pass < 2; ++pass) {
+      if (pass == 1) {
+        off[0] = 0;
+        for (int g = 0; g < L->G; ++g) off[g + 1] = off[g] + (cnt[g] + 127) / 128 * 128;
+        for (int g = 0; g < L->G; ++g) pos[g] = off[g];
+      }
+      for (size_t t = 0; t < n; ++t) {
+        for (int e = 0; e <= L->K; ++e) {
+          uint64_t bl = e == 0 ? sh[t] : (((em[t] >> (e - 1)) & 1ull) ? (~sh[t] & full) : 0ull);
+          const float w = e == 0 ? al[t] : sv[t * K + e - 1];
+          for (; bl != 0ull; bl &= bl - 1ull) {
+            const int g = e * B + (__builtin_ffsll((long long)bl) - 1);
+            if (pass == 0) { ++cnt[g]; continue; }
+            if (row_token) row_token[pos[g]] = tok_base + (int32_t)t;
+            if (row_weight) row_weight[pos[g]] = w;
+            ++pos[g];
+          }
+        }
+      }
+    }
+    total = off[L->G];
+    for (int g = 0; g < L->G; ++g)
+      for (int r = pos[g]; r < off[g + 1]; ++r) {
+        if (row_token) row_token[r] = -1;
+        if (row_weight) row_weight[r] = 0.f;
+      }
+    if (counts) memcpy(counts, cnt.data(), sizeof(int32_t) * L->G);
+    if (offsets) memcpy(offsets, off.data(), sizeof(int32_t) * (L->G + 1));
+  } else if (L->last_T > 0 && L->fused_group) {
     // rows live in per-group regions on the device, each group's rows in the
     // order the router CTAs reserved them: gather them group by group into
     // the contiguous padded layout, in token order
@@ -799,6 +856,7 @@ int unif_moe_pass_tokens(unif_moe_t L) { return L ? L->pass_tokens : -1; }
 
 int unif_moe_kernels_per_forward(unif_moe_t L) {
   if (!L) return -1;
+  if (L->ffn_fused) return 3;  // router, expert-tile FFN, combine
   return L->fused_group ? (L->tile_list ? 5 : 4) : 6;
 }
 

@@ -66,7 +66,7 @@ def test_argument_errors_without_gpu(lib):
     opts = pkg.Options()
     lib.unif_moe_default_options(C.byref(opts))
     assert opts.features == pkg.FEATURES_DEFAULT and opts.gemm_kernels == 0
-    for o in (pkg.Options(16, 0), pkg.Options(3, 2), pkg.Options(3, -1)):  # unknown bit / kind
+    for o in (pkg.Options(16, 0), pkg.Options(3, 4), pkg.Options(3, -1)):  # unknown bit / kind
         assert lib.unif_moe_create_ex(C.byref(h), 64, 256, 4, 4, None, 1, 16, C.byref(o)) == -1
     assert b"options" in lib.unif_moe_last_error()
     assert lib.unif_moe_forward(None, None, None, 4, None, None, None, None) == -1

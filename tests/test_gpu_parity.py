@@ -143,6 +143,10 @@ def test_smaller_then_larger_forward_on_one_handle():
 def test_kernels_per_forward():
     s = small(tokens=500)
     assert make_layer(s).kernels_per_forward() == 4   # grouping inside the router
+    # router, expert-tile FFN, combine
+    assert make_layer(s, gemm_kernels="expert_tile").kernels_per_forward() == 3
+    assert make_layer(small(tokens=500, d_model=192, d_ff=768),
+                      gemm_kernels="expert_tile").kernels_per_forward() == 4  # d % 128 != 0
     assert make_layer(small("f32", tokens=64)).kernels_per_forward() == 6
 
 
@@ -211,9 +215,13 @@ def test_f32_variants():
 
 # ------------------------------------------------------------ group table
 
-def test_group_table_matches_oracle():
+@pytest.mark.parametrize("kernels", ["expert_tile", "grouped"])
+def test_group_table_matches_oracle(kernels):
+    """The (expert, block) group table: read from the device grouping
+    ("grouped"), or derived from the routing records when the device
+    grouped the rows by expert (the expert-tile FFN)."""
     wl = workloads.make_workload(small(tokens=1500, n_experts=6, n_blocks=8, d_ff=1024))
-    g = run_gpu(wl)
+    g = run_gpu(wl, gemm_kernels=kernels)
     counts, offsets, tok, w = g.layer.groups()
     r = oracle.with_decisions(compare_routing(wl), g.shr, g.em, wl.spec.n_blocks)
     c_ref, tok_ref, w_ref = oracle.groups(r, wl.spec.n_experts, wl.spec.n_blocks)
@@ -437,14 +445,33 @@ def test_forward_host_async_pipeline():
 
 # ------------------------------------------- GEMM kernel variants
 
-@pytest.mark.parametrize("kernels", ["weight_stationary", "streaming"])
+GEMM_FAMILY = {"expert_tile": "expert_tile", "weight_stationary": "grouped",
+               "streaming": "streaming"}
+
+
+@pytest.mark.parametrize("kernels", list(GEMM_FAMILY))
 def test_gemm_variants_many_group_runs(kernels):
     """Enough tiles that every CTA walks several group runs (weight slabs
-    reloaded mid-run), on both GEMM kernel families."""
+    reloaded mid-run; several expert tiles per CTA), on every GEMM kernel
+    family."""
     wl = workloads.make_workload(small(tokens=6000, d_model=128, d_ff=512, n_experts=8,
                                        n_blocks=4))
-    g = run_gpu(wl, gemm_kernels="auto" if kernels == "weight_stationary" else "streaming")
+    g = run_gpu(wl, gemm_kernels=GEMM_FAMILY[kernels])
     assert_parity(wl, g, compare(wl, g, label=kernels))
+
+
+@pytest.mark.parametrize("shape", [
+    dict(d_model=128, d_ff=384, n_experts=3, n_blocks=6),     # M = 64: two blocks per chunk
+    dict(d_model=256, d_ff=1536, n_experts=8, n_blocks=8),    # M = 192: blocks across chunks
+    dict(d_model=384, d_ff=1024, n_experts=2, n_blocks=16),   # M = 64, B = 16
+])
+def test_expert_tile_shapes(shape):
+    """The expert-tile FFN where blocks and 128-channel chunks do not line
+    up, on ragged token counts (partial last tiles of every expert)."""
+    wl = workloads.make_workload(small(tokens=1111, **shape))
+    g = run_gpu(wl, gemm_kernels="expert_tile")
+    assert g.layer.kernels_per_forward() == 3
+    assert_parity(wl, g, compare(wl, g, label="expert_tile"))
 
 
 def test_vit_s_streaming_kernels():
@@ -455,8 +482,9 @@ def test_vit_s_streaming_kernels():
 
 
 def test_repeated_forwards_match_streaming_kernels():
-    """Ten forwards of the ViT-S layer through the weight-stationary kernels
-    agree with the streaming kernels token by token (the two differ only in
+    """Ten forwards of the ViT-S layer through the expert-tile FFN, and ten
+    through the weight-stationary kernels, agree with the streaming kernels
+    token by token (the two differ only in
     the order of the fp32 additions into the accumulator): catches
     synchronisation races that corrupt a tile now and then."""
     s = workloads.spec("vit_s")
@@ -470,13 +498,14 @@ def test_repeated_forwards_match_streaming_kernels():
 
     x = wl.x.to(dev)
     ref = layer("streaming").forward(x).float()
-    L = layer("auto")
-    for _ in range(10):
-        y = L.forward(x).float()
-        torch.cuda.synchronize()
-        assert L.sync_status() == 0
-        rel = (y - ref).abs().amax(1) / ref.abs().amax(1).clamp_min(1e-6)
-        assert float(rel.max()) < 1e-2, int((rel >= 1e-2).sum())
+    for kernels in ("expert_tile", "grouped"):
+        L = layer(kernels)
+        for _ in range(10):
+            y = L.forward(x).float()
+            torch.cuda.synchronize()
+            assert L.sync_status() == 0
+            rel = (y - ref).abs().amax(1) / ref.abs().amax(1).clamp_min(1e-6)
+            assert float(rel.max()) < 1e-2, (kernels, int((rel >= 1e-2).sum()))
 
 
 def test_repeated_forwards_sliced_down_projection():
