@@ -103,7 +103,7 @@ enum {
  *   weight-stationary kernels where a group's weight slice fits in shared
  *   memory, else the streaming ones.
  * - STREAMING: as GROUPED, always the streaming kernels.
- * - AUTO: GROUPED. */
+ * - AUTO: EXPERT_TILE where it applies, else GROUPED. */
 enum {
   UNIF_MOE_GEMM_AUTO = 0,
   UNIF_MOE_GEMM_STREAMING = 1,

@@ -136,7 +136,7 @@ class Layer:
     block) groups, weight-stationary kernels where they fit), "streaming"
     ((expert, block) groups, streaming kernels), "expert_tile" (rows grouped
     by expert, both projections in one kernel, where it applies) or "auto"
-    (as "grouped")."""
+    (expert_tile where it applies, else grouped)."""
 
     def __init__(self, d_model: int, d_ff: int, n_experts: int, n_blocks: int,
                  dtype: str = "bf16", max_tokens: int = 65536, tau: float = math.nan,

@@ -163,7 +163,9 @@ struct unif_moe_layer {
   // Expert-tile FFN (both projections in one kernel, rows grouped by
   // expert): its weight maps (128 x 64 slabs), shared memory and ring depth.
   bool ffn_fused = false;
-  int ffn_per_cta = 0, ffn_slots = 0;
+  CUtensorMap tm_fk, tm_fv;  // the repacked K_e / V_e slabs, boxes of one half-slab
+  int ffn_pairs = 0;         // CTA pairs launched (clusters of two)
+  int ffn_per_cta = 0, ffn_slots = 0;  // pair tiles per pair (run table), ring half-slabs
   uint32_t ffn_smem = 0;
   // backward: transposed weights and the per-row gradient buffers
   CUtensorMap tm_wdownT;    // w_downT [(K+1) H][d], boxes of 64 x up_bn

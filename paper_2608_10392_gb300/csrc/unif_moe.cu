@@ -240,7 +240,9 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   L->region_rows = (L->pass_tokens + 127) / 128 * 128;
   // rows grouped by expert for the expert-tile FFN (where it applies; the
   // backward pass reads the (expert, block) groups and h of a forward)
-  L->ffn_fused = L->fused_group && o.gemm_kernels == UNIF_MOE_GEMM_EXPERT_TILE &&
+  L->ffn_fused = L->fused_group &&
+                 (o.gemm_kernels == UNIF_MOE_GEMM_EXPERT_TILE ||
+                  o.gemm_kernels == UNIF_MOE_GEMM_AUTO) &&
                  !(o.features & UNIF_MOE_FEATURE_BACKWARD) && unif::ffn_fused_fits(d_model, d_ff, M);
   const size_t row_cap = L->fused_group ? (size_t)L->G * L->region_rows : (size_t)L->max_rows;
   ALLOC(w.row_tok, row_cap); ALLOC(w.row_w, row_cap);

@@ -142,9 +142,9 @@ def test_smaller_then_larger_forward_on_one_handle():
 
 def test_kernels_per_forward():
     s = small(tokens=500)
-    assert make_layer(s).kernels_per_forward() == 4   # grouping inside the router
-    # router, expert-tile FFN, combine
+    assert make_layer(s).kernels_per_forward() == 3   # router, expert-tile FFN, combine
     assert make_layer(s, gemm_kernels="expert_tile").kernels_per_forward() == 3
+    assert make_layer(s, gemm_kernels="grouped").kernels_per_forward() == 4  # up, down
     assert make_layer(small(tokens=500, d_model=192, d_ff=768),
                       gemm_kernels="expert_tile").kernels_per_forward() == 4  # d % 128 != 0
     assert make_layer(small("f32", tokens=64)).kernels_per_forward() == 6
