@@ -122,6 +122,8 @@ def measured_traffic(workload, kernel):
     if not os.path.exists(path):
         return None
     rec = json.load(open(path)).get(workload, {})
+    if isinstance(rec.get(kernel), dict):  # a kernel with its own record and sources
+        rec = dict(rec[kernel], **{kernel: rec[kernel].get("bytes")})
     csrc = os.path.join(ROOT, "paper_2608_10392_gb300", "csrc")
     h = hashlib.sha1()
     for f in rec.get("sources", []):

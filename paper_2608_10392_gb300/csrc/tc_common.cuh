@@ -243,16 +243,16 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
   return r;
 }
 // Arrive on an mbarrier of any CTA of the cluster (default semantics, as
-// for a local arrive; a .release.cluster arrive costs ~0.5-1 us per call
-// on GB300, measured, and is not needed where the waiting side only issues
-// tcgen05 work on data this thread's fences already ordered).
+// for a local arrive: the waiting side only issues tcgen05 work on data
+// this thread's own fences already ordered; with .release.cluster the
+// peer CTA's arrivals in the expert-tile FFN came 0.5-1 us later, measured
+// on GB300).
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 // wait_warp for a barrier that the peer CTA of a pair also arrives on (its
-// arrivals follow a tcgen05 fence or a proxy fence of their own; a wait with
-// .acquire.cluster semantics costs ~0.3 us per call on GB300, measured, and
-// serialised the MMA issue behind it).
+// arrivals follow a tcgen05 fence or a proxy fence of their own), with the
+// default semantics of the arrivals it pairs with.
 static __device__ __forceinline__ bool wait_warp_cluster(uint32_t bar, uint32_t parity,
                                                          volatile int* abort_flag, int* status,
                                                          long long limit) {
