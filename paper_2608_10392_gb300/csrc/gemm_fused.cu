@@ -73,7 +73,7 @@ constexpr int kEpiWarps = 8;
 constexpr int kFirstDrain = 14;
 constexpr int kDrainWarps = 4;
 constexpr int kThreads = 32 * (kFirstDrain + kDrainWarps);  // 576
-constexpr uint32_t kStaging = kDrainWarps * 32u * 128u;       // 32 x 32 fp32 per drain warp
+constexpr uint32_t kStaging = kDrainWarps * 32u * 128u;  // per TMEM lane quarter 4 KB: two 32 x 16 fp32 tiles
 constexpr uint32_t kBarBytes = 512;
 constexpr uint32_t kMaxSmem = 232448;
 constexpr int kPairRows = 256;        // rows of a pair tile
@@ -215,7 +215,7 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
       mbar_init(hsempty(h), 1);
     }
     mbar_init(dfull, 1);
-    mbar_init(dempty, 2 * kDrainWarps);
+    mbar_init(dempty, 2 * (kDrainWarps + kGatherWarps));
     mbar_init(mma_done, 1);
     mbar_init(fin, 1);
     *abort_flag = 0;
@@ -270,6 +270,50 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     r0 = run_s[p.per_pair + i] + kBM * (int)rank;
     rows = min(kBM, max(0, run_s[2 * p.per_pair + i] - kBM * (int)rank));
   };
+  // y[tok] += w D over columns [c_begin, c_end) of tile i's D, for the 32
+  // rows of TMEM lane quarter warp % 4 (thread = row). 16 columns per
+  // pass: the thread stages its row's 64 scaled bytes in the warp's 2 KB
+  // tile (16-byte chunk c at c ^ ((r >> 1) & 3)), then 4 lanes per row add
+  // 8 rows x 64 contiguous bytes per instruction. Returns false if a wait
+  // gave up. The D reads end with the arrival on dempty.
+  auto drain = [&](int i, int c_begin, int c_end, float* stf) {
+    const int q = warp & 3;
+    const int r = 32 * q + lane;
+    int r0, rows;
+    my_rows(i, r0, rows);
+    const int tok = r < rows ? p.row_tok[r0 + r] : -1;
+    const float w = r < rows ? p.row_w[r0 + r] : 0.f;
+    if (!wait_warp(dfull, (uint32_t)i & 1u, abort_flag, p.status, p.wait_limit)) return false;
+    tc_fence_after();
+    const uint32_t t_row = tmem_base + ((uint32_t)(32 * q) << 16);
+    const int r_sub = lane >> 2, c4 = lane & 3;
+    const uint32_t sw = (uint32_t)(lane >> 1) & 3u;
+#pragma unroll 1
+    for (int c = c_begin; c < c_end; c += 16) {
+      float v[16];
+      tmem_ld16(t_row + (uint32_t)c, v);
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj)
+        *reinterpret_cast<float4*>(stf + lane * 16 + ((jj ^ sw) << 2)) =
+            make_float4(w * v[4 * jj], w * v[4 * jj + 1], w * v[4 * jj + 2], w * v[4 * jj + 3]);
+      __syncwarp();
+#pragma unroll
+      for (int ii = 0; ii < 4; ++ii) {
+        const int rr = 8 * ii + r_sub;
+        const int tr = __shfl_sync(0xffffffffu, tok, rr);
+        const float4 val = *reinterpret_cast<const float4*>(
+            stf + rr * 16 + ((c4 ^ ((rr >> 1) & 3)) << 2));
+        if (tr >= 0)
+          atomicAdd(reinterpret_cast<float4*>(p.y32 + (size_t)tr * DD + c + c4 * 4), val);
+      }
+      __syncwarp();
+    }
+    // D has been read: the next tile's down MMAs may overwrite it
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) arrive_leader(dempty);
+    return true;
+  };
 
   if (warp < kGatherWarps) {
     // ---------------- this CTA's x rows of the tile -------------------------
@@ -278,6 +322,7 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     // commit group per 64-column block, so the first up MMAs can start on
     // the first block while the rest arrive
     const int j8 = lane & 7, rsub = lane >> 3;
+    float* stg_gather = reinterpret_cast<float*>(stg_base + (size_t)warp * 4096 + 2048);
     bool ok = true;
     for (int i = 0; i < n_run && ok; ++i) {
       int r0, rows;
@@ -306,7 +351,11 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         __syncwarp();
         if (lane == 0) arrive_leader(xfull(kb));
       }
+      // idle until the next tile's rows are wanted: drain the second half
+      // of the previous tile's D columns beside the drain warps
+      if (i > 0) ok = drain(i - 1, DD / 2, DD, stg_gather);
     }
+    if (ok && n_run > 0) drain(n_run - 1, DD / 2, DD, stg_gather);
   } else if (warp == kLoaderWarp) {
     // ---------------- this CTA's weight half-slabs, in MMA order ------------
     // Half `rank` of slab u = rows 128 u + 64 rank .. + 63 of the repacked
@@ -519,48 +568,11 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
       }
     }
   } else {
-    // ---------------- drain: y[tok] += w D -----------------------------------
-    // Thread = row 32 q + lane of this CTA's rows; 32 columns per pass: the
-    // thread stages its row's 128 scaled bytes (chunk c at c ^ (r & 7)),
-    // then 8 lanes per row add 4 rows x 128 contiguous bytes per
-    // instruction.
-    const int q = warp & 3;
-    const int r = 32 * q + lane;
-    float* stf = reinterpret_cast<float*>(stg_base + (size_t)(warp - kFirstDrain) * 32 * 128);
-    const int r_sub = lane >> 3, c8 = lane & 7;
-    for (int i = 0; i < n_run; ++i) {
-      int r0, rows;
-      my_rows(i, r0, rows);
-      const int tok = r < rows ? p.row_tok[r0 + r] : -1;
-      const float w = r < rows ? p.row_w[r0 + r] : 0.f;
-      if (!wait_warp(dfull, (uint32_t)i & 1u, abort_flag, p.status, p.wait_limit)) break;
-      tc_fence_after();
-      const uint32_t t_row = tmem_base + ((uint32_t)(32 * q) << 16);
-#pragma unroll 1
-      for (int c = 0; c < DD; c += 32) {
-        float v[32];
-        tmem_ld32(t_row + (uint32_t)c, v);
-#pragma unroll
-        for (int jj = 0; jj < 8; ++jj)
-          *reinterpret_cast<float4*>(stf + lane * 32 + ((jj ^ (lane & 7)) << 2)) =
-              make_float4(w * v[4 * jj], w * v[4 * jj + 1], w * v[4 * jj + 2], w * v[4 * jj + 3]);
-        __syncwarp();
-#pragma unroll
-        for (int ii = 0; ii < 8; ++ii) {
-          const int rr = 4 * ii + r_sub;
-          const int tr = __shfl_sync(0xffffffffu, tok, rr);
-          const float4 val =
-              *reinterpret_cast<const float4*>(stf + rr * 32 + ((c8 ^ (rr & 7)) << 2));
-          if (tr >= 0)
-            atomicAdd(reinterpret_cast<float4*>(p.y32 + (size_t)tr * DD + c + c8 * 4), val);
-        }
-        __syncwarp();
-      }
-      // D has been read: the next tile's down MMAs may overwrite it
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) arrive_leader(dempty);
-    }
+    // ---------------- drain: y[tok] += w D, the first half of the columns ---
+    // (the gather warps, idle between their tiles' gathers, take the second)
+    float* stf = reinterpret_cast<float*>(stg_base + (size_t)(warp & 3) * 4096);
+    for (int i = 0; i < n_run; ++i)
+      if (!drain(i, 0, DD / 2, stf)) break;
   }
   // every warp converged before the CTA barrier; then each CTA tells its
   // peer that it is done with the pair's TMEM (the leader after its MMAs
