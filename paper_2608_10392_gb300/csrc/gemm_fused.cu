@@ -89,6 +89,8 @@ struct Params {
   int n_chunks, num_kb, n_pieces, slots;
   const __nv_bfloat16* x;  // [T][d] the pass's tokens
   float* y32;              // [T][d] fp32 output accumulator of the pass
+  float* y32_next;         // the other accumulator, zeroed here for the next pass
+  long long next_f4;       // its float4 count
   int* status;
   long long wait_limit;
 };
@@ -508,6 +510,16 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         __syncwarp();
         wait_settle(mma_done, 0u, p.wait_limit);
       }
+    } else {
+      // The peer's MMA warp has no MMAs to issue: it zeroes its pair's share
+      // of the other accumulator, which the next pass adds into (the
+      // combine only reads this pass's). It waits for nothing, so a pass
+      // whose other roles gave up still leaves the next one clean.
+      float4* z = reinterpret_cast<float4*>(p.y32_next);
+      const long long per = (p.next_f4 + n_pairs - 1) / n_pairs;
+      const long long z0 = (long long)pair * per;
+      const long long z1 = min(p.next_f4, z0 + per);
+      for (long long k = z0 + lane; k < z1; k += 32) z[k] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
     __syncwarp();
   } else if (warp < kFirstDrain) {
@@ -733,7 +745,9 @@ cudaError_t launch_ffn_fused(unif_moe_layer* L, const void* x, cudaStream_t s) {
   p.n_pieces = L->d / tc::fused::kPiece;
   p.slots = L->ffn_slots;
   p.x = static_cast<const __nv_bfloat16*>(x);
-  p.y32 = L->ws.y32;
+  p.y32 = acc_cur(L);
+  p.y32_next = L->acc_sel ? L->ws.y32 : L->ws.y32_b;
+  p.next_f4 = (long long)L->pass_tokens * L->d / 4;
   p.status = L->ws.status;
   p.wait_limit = gemm_wait_limit();
   cudaLaunchConfig_t cfg = {};

@@ -73,6 +73,10 @@ struct Workspace {
   // output accumulator.
   void* hbuf = nullptr;          // [max_rows][M] (layer dtype)
   float* y32 = nullptr;          // [max_tokens][d]
+  // The expert-tile FFN's second accumulator: a pass adds into one of the
+  // two and zeroes the other for the next pass, so that the combine only
+  // reads (acc_sel names the one the next pass adds into).
+  float* y32_b = nullptr;        // [pass_tokens][d]
   // Expert weights repacked into the expert-tile FFN's 16 KB operand slabs.
   void* wk_slabs = nullptr;      // K_e: [K+1][H/128][d/64] slabs
   void* wv_slabs = nullptr;      // V_e: [K+1][H/128][2][d/128] slabs
@@ -163,6 +167,7 @@ struct unif_moe_layer {
   // Expert-tile FFN (both projections in one kernel, rows grouped by
   // expert): its weight maps (128 x 64 slabs), shared memory and ring depth.
   bool ffn_fused = false;
+  int acc_sel = 0;  // expert-tile FFN: the accumulator the next pass adds into (0: y32, 1: y32_b)
   CUtensorMap tm_fk, tm_fv;  // the repacked K_e / V_e slabs, boxes of one half-slab
   int ffn_pairs = 0;         // CTA pairs launched (clusters of two)
   int ffn_per_cta = 0, ffn_slots = 0;  // pair tiles per pair (run table), ring half-slabs
@@ -198,6 +203,8 @@ cudaError_t launch_router(unif_moe_layer* L, const void* x, const uint8_t* mask,
                           int32_t* b_out, int32_t* k_out, cudaStream_t s);
 cudaError_t launch_permute(unif_moe_layer* L, int T, cudaStream_t s);
 cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s);
+// The fp32 accumulator the pass being launched adds into.
+inline float* acc_cur(const unif_moe_layer* L);
 cudaError_t launch_layernorm(unif_moe_layer* L, const void* x, void* out, const uint8_t* mask,
                              const void* gamma, const void* beta, float eps, int T,
                              cudaStream_t s);
@@ -248,5 +255,9 @@ int backward_run(unif_moe_layer* L, const void* x, const void* dy, int T, const 
 int diag_alignment(unif_moe_layer* L, float delta, float* rho, cudaStream_t s);
 int diag_demand(unif_moe_layer* L, const void* x, int T, const void* w_res, float delta,
                 float eps, int32_t* k_eps, float* err, int32_t* pair_out, cudaStream_t s);
+
+inline float* acc_cur(const unif_moe_layer* L) {
+  return L->ffn_fused && L->acc_sel ? L->ws.y32_b : L->ws.y32;
+}
 
 }  // namespace unif

@@ -508,12 +508,14 @@ __global__ void tile_list_kernel(const int32_t* __restrict__ fill, int G, int re
 // ---------------------------------------------------------------------------
 
 // The fp32 accumulator is all zero between forwards: each combine zeroes
-// the rows it reads (the down projection of the next forward adds into
-// them). Also copies the router's group fill counters (n_fill ints, the
-// group sizes) to the group table's counts and zeroes them for the next
-// forward: every kernel that reads them has finished.
+// the rows it reads (zero != 0; the down projection of the next forward
+// adds into them), or the expert-tile FFN zeroed the other of its two
+// accumulators for the next pass (zero == 0). Also copies the router's
+// group fill counters (n_fill ints, the group sizes) to the group table's
+// counts and zeroes them for the next forward: every kernel that reads
+// them has finished.
 __global__ void cast_out_bf16(float4* __restrict__ y, uint2* __restrict__ out, size_t n4,
-                              int32_t* fill, int32_t* counts, int n_fill, int region) {
+                              int32_t* fill, int32_t* counts, int n_fill, int region, int zero) {
   grid_dep_wait();  // the down projection's sums are complete
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i < n_fill; i += blockDim.x) {
@@ -540,7 +542,7 @@ __global__ void cast_out_bf16(float4* __restrict__ y, uint2* __restrict__ out, s
       o.x = *reinterpret_cast<unsigned*>(&lo);
       o.y = *reinterpret_cast<unsigned*>(&hi);
       out[i] = o;
-      y[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (zero) y[i] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
   }
 }
@@ -645,14 +647,14 @@ layernorm_rows(const T* __restrict__ x, T* __restrict__ out, const uint8_t* __re
 
 // The sublayer's combine: v = y + x (accumulator row plus the residual
 // input), out = LN(v) (NORM) or v; padding rows give 0. Zeroes the
-// accumulator rows and, in block 0, hands the group sizes on and zeroes the
-// grouping counters, as cast_out_bf16 does.
+// accumulator rows (zero != 0) and, in block 0, hands the group sizes on
+// and zeroes the grouping counters, as cast_out_bf16 does.
 template <typename T, bool NORM>
 __global__ void __launch_bounds__(256)
 combine_residual(float* __restrict__ y, const T* __restrict__ x, T* __restrict__ out,
                  const uint8_t* __restrict__ mask, const T* __restrict__ gamma,
                  const T* __restrict__ beta, float eps, int n_rows, int d, int32_t* fill,
-                 int32_t* counts, int n_fill, int region) {
+                 int32_t* counts, int n_fill, int region, int zero) {
   grid_dep_wait();  // the down projection's sums are complete
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i < n_fill; i += blockDim.x) {
@@ -661,7 +663,7 @@ combine_residual(float* __restrict__ y, const T* __restrict__ x, T* __restrict__
     }
   const int lane = threadIdx.x & 31;
   const int warps = gridDim.x * (blockDim.x >> 5);
-  const float zero[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  const float zeros[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n_rows; r += warps) {
     const size_t base = (size_t)r * d;
     const bool pad = mask != nullptr && mask[r] == 0;
@@ -686,7 +688,7 @@ combine_residual(float* __restrict__ y, const T* __restrict__ x, T* __restrict__
       const int f = 8 * (32 * j + lane);
       if (f < d) {
         store8(out + base + f, v[j]);
-        store8(y + base + f, zero);
+        if (zero) store8(y + base + f, zeros);
       }
     }
   }
@@ -847,20 +849,21 @@ cudaError_t launch_combine_residual(unif_moe_layer* L, const void* x, void* out,
                                     float eps, bool norm, int T, cudaStream_t s) {
   const int grid = std::min((T + 7) / 8, L->n_sm * 8);
   const int n_fill = L->fused_group ? L->G : 0;
-  float* y = L->ws.y32;
+  float* y = acc_cur(L);
+  const int zero = L->ffn_fused ? 0 : 1;  // the expert-tile FFN zeroed the other accumulator
   if (L->dtype == UNIF_MOE_BF16) {
     using B = __nv_bfloat16;
     auto k = norm ? combine_residual<B, true> : combine_residual<B, false>;
     return launch_dependent(k, dim3(grid), dim3(256), 0, s, y, static_cast<const B*>(x),
                             static_cast<B*>(out), mask, static_cast<const B*>(gamma),
                             static_cast<const B*>(beta), eps, T, L->d, L->ws.grp_fill,
-                            L->ws.grp_cnt, n_fill, L->region_rows);
+                            L->ws.grp_cnt, n_fill, L->region_rows, zero);
   }
   auto k = norm ? combine_residual<float, true> : combine_residual<float, false>;
   return launch_dependent(k, dim3(grid), dim3(256), 0, s, y, static_cast<const float*>(x),
                           static_cast<float*>(out), mask, static_cast<const float*>(gamma),
                           static_cast<const float*>(beta), eps, T, L->d, L->ws.grp_fill,
-                          L->ws.grp_cnt, n_fill, L->region_rows);
+                          L->ws.grp_cnt, n_fill, L->region_rows, zero);
 }
 
 cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s) {
@@ -868,9 +871,9 @@ cudaError_t launch_combine(unif_moe_layer* L, void* out, int T, cudaStream_t s) 
   const int grid = L->n_sm * 8;
   if (L->dtype == UNIF_MOE_BF16)
     return launch_dependent(cast_out_bf16, dim3(grid), dim3(256), 0, s,
-                            reinterpret_cast<float4*>(L->ws.y32), static_cast<uint2*>(out),
+                            reinterpret_cast<float4*>(acc_cur(L)), static_cast<uint2*>(out),
                             n4, L->ws.grp_fill, L->ws.grp_cnt, L->fused_group ? L->G : 0,
-                            L->region_rows);
+                            L->region_rows, L->ffn_fused ? 0 : 1);
   else
     copy_out_f32<<<grid, 256, 0, s>>>(reinterpret_cast<float4*>(L->ws.y32),
                                       static_cast<float4*>(out), n4);

@@ -75,7 +75,7 @@ void free_all(unif_moe_layer* L) {
                   L->ws.tile_rows, L->ws.w_upT, L->ws.w_downT, L->ws.da, L->ws.hw,
                   L->ws.dwt, L->ws.dz, L->ws.wrT, L->ws.gram, L->ws.diag_sets,
                   L->ws.diag_counts, L->ws.diag_pair, L->ws.diag_wts, L->ws.diag_q,
-                  L->ws.diag_E, L->ws.diag_ES, L->ws.wk_slabs, L->ws.wv_slabs};
+                  L->ws.diag_E, L->ws.diag_ES, L->ws.wk_slabs, L->ws.wv_slabs, L->ws.y32_b};
   for (void* q : ptrs)
     if (q) cudaFree(q);
   for (int i = 0; i < 2; ++i) {
@@ -251,6 +251,7 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&hb), es * (size_t)L->max_rows * M);
   w.hbuf = hb;
   ALLOC(w.y32, (size_t)L->pass_tokens * d_model);
+  if (L->ffn_fused) ALLOC(w.y32_b, (size_t)L->pass_tokens * d_model);
   if (L->ffn_fused) {  // the expert weights as the expert-tile FFN's operand slabs
     if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.wk_slabs), es * E * d_ff * d_model);
     if (rc == UNIF_MOE_OK) rc = dalloc(reinterpret_cast<char**>(&w.wv_slabs), es * E * d_ff * d_model);
@@ -303,6 +304,8 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
   if (rc == UNIF_MOE_OK && (cudaMemset(w.status, 0, sizeof(int)) != cudaSuccess ||
                             cudaMemset(w.y32, 0, sizeof(float) * L->pass_tokens * d_model) !=
                                 cudaSuccess ||
+                            (w.y32_b && cudaMemset(w.y32_b, 0, sizeof(float) * L->pass_tokens *
+                                                                   d_model) != cudaSuccess) ||
                             (L->fused_group &&
                              (cudaMemset(w.grp_fill, 0, sizeof(int32_t) * L->G) != cudaSuccess ||
                               // rows hold token indices from the start, also any row a
@@ -392,6 +395,8 @@ static int forward_pass(unif_moe_t L, const void* x, void* out, int T, int t0,
   // launching its combine leaves them dirty: clear them first.
   if (L->y_dirty) {
     CK(cudaMemsetAsync(L->ws.y32, 0, sizeof(float) * (size_t)L->pass_tokens * L->d, s));
+    if (L->ws.y32_b)
+      CK(cudaMemsetAsync(L->ws.y32_b, 0, sizeof(float) * (size_t)L->pass_tokens * L->d, s));
     if (L->fused_group) CK(cudaMemsetAsync(L->ws.grp_fill, 0, sizeof(int32_t) * L->G, s));
   }
   L->y_dirty = true;
@@ -418,6 +423,8 @@ static int forward_pass(unif_moe_t L, const void* x, void* out, int T, int t0,
   else
     CK(unif::launch_combine(L, out, T, s));
   L->y_dirty = false;
+  // the expert-tile FFN zeroed the other accumulator for the next pass
+  if (L->ffn_fused) L->acc_sel ^= 1;
   if (ev[5]) CK(cudaEventRecord(ev[5], s));
   return UNIF_MOE_OK;
 }
