@@ -9,10 +9,12 @@
 // pair computes
 //   U = x K_e[c]^T                        (M=256, N=128, K=d; TMEM)
 //   h = bf16(GeLU(U)), zero in the columns of blocks the row does not run
-//   D += h V_e[:, c]^T                    (M=256, N=d in 128-column pieces)
+//   D += h V_e[:, c]^T                    (M=256, N=d: 256-column pieces,
+//                                          then a 128-column remainder)
 // with tcgen05.mma.cta_group::2 issued by the even CTA: each CTA holds the
 // A rows of its own 128 rows (x, then h) and half of every B operand (64 of
-// the 128 rows of each weight slab), and each CTA's TMEM the D and U rows of
+// the 128 rows of each weight slab; for a 256-column piece, one whole slab
+// each), and each CTA's TMEM the D and U rows of
 // its own 128 rows. After the last chunk each CTA adds w D into the fp32
 // output accumulator, once per (token, expert) instead of once per (token,
 // expert, block). Each token's x row is gathered once per expert it runs,
@@ -166,6 +168,26 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
   constexpr int num_kb = DD / kBK, npc = DD / kPiece;
   static_assert(num_kb % kStageHalves == 0 && (2 * npc) % kStageHalves == 0,
                 "stages never straddle an up or a down projection");
+  // The down projection of a chunk: D[:, 256 P .. 256 P + 255] for each
+  // 256-column piece P as N = 256 MMAs, each reading h once for 256 output
+  // columns (three N = 128 pieces read h three times per chunk, and shared
+  // memory bandwidth is what the chunk loop runs against), then the
+  // 128-column remainder (d = 128, 384) as N = 128 MMAs. Stages in MMA
+  // order: piece P for h half 0, the remainder (both halves), piece P for
+  // h half 1, so that h half 0 is released after the second stage as
+  // before. Each stage is kStageHalves half-slabs of this CTA.
+  constexpr int n256 = DD / 256, kRem = DD % 256 ? 1 : 0;
+  constexpr int kDownStages = 2 * n256 + kRem;
+  static_assert(kDownStages * kStageHalves == 2 * npc, "the down stages hold the chunk's slabs");
+  // true: 256-column piece P of h half hh; false: the remainder piece
+  auto down_stage = [](int st, int& hh, int& P) {
+    if (st < n256) { hh = 0; P = st; return true; }
+    if (kRem && st == n256) { hh = 0; P = 0; return false; }
+    hh = 1; P = st - n256 - kRem;
+    return true;
+  };
+  // the last down stage that reads h half 0
+  constexpr int kH0Last = kRem ? n256 : n256 - 1;
   const int nch = p.n_chunks;
   const uint32_t sX = smem_u32(smem);
   const uint32_t sH = sX + (uint32_t)num_kb * kXBlock;
@@ -373,7 +395,9 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     uint32_t ph = 0;
     long long issued = 0;
     bool ok = true;
-    auto stage = [&](const CUtensorMap* m, long long slab0) {
+    // lane j < kStageHalves loads the 64 repacked rows starting at row_j
+    // into half-slab slot j of the stage
+    auto stage = [&](const CUtensorMap* m, long long row0, long long row1) {
       if (!ok) return;
       // the whole warp waits (lanes parked at a shuffle while one lane
       // waits cost the warp hundreds of cycles to reconverge)
@@ -385,19 +409,35 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
       __syncwarp();
       if (lane < kStageHalves)
         tma_load_2d_pair(sW + (uint32_t)(s * kStageHalves + lane) * kHalf, m, at_leader(wfull(s)),
-                         0, (int)((slab0 + lane) * 128 + 64 * (long long)rank));
+                         0, (int)(lane == 0 ? row0 : row1));
       ++issued;
       if (++s == n_stages) { s = 0; ph ^= 1u; }
     };
+    // Down stages of chunk c in MMA order (down_stage): a 256-column piece
+    // P for h half hh holds this CTA's 128 of its rows, i.e. all of slab
+    // (hh, np = 2 P + rank); the 128-column remainder piece holds this
+    // CTA's 64-row halves of slabs (0, npc - 1) and (1, npc - 1).
     auto load_down = [&](int e, int c) {
       const long long v0 = (long long)(e * nch + chunk_of(c)) * 2 * npc;
-      for (int j = 0; j < 2 * npc; j += kStageHalves) stage(&tmV, v0 + j);
+#pragma unroll
+      for (int st = 0; st < kDownStages; ++st) {
+        int hh, P;
+        if (down_stage(st, hh, P)) {
+          const long long row = (v0 + hh * npc + 2 * P + rank) * 128;
+          stage(&tmV, row, row + 64);
+        } else {
+          const long long row = (v0 + npc - 1) * 128 + 64 * (long long)rank;
+          stage(&tmV, row, row + (long long)npc * 128);
+        }
+      }
     };
     for (int i = 0; i < n_run && ok; ++i) {
       const int e = run_s[i];
       for (int c = 0; c < nch; ++c) {
         const long long u0 = (long long)(e * nch + chunk_of(c)) * num_kb;
-        for (int kb = 0; kb < num_kb; kb += kStageHalves) stage(&tmK, u0 + kb);
+        for (int kb = 0; kb < num_kb; kb += kStageHalves)
+          stage(&tmK, (u0 + kb) * 128 + 64 * (long long)rank,
+                (u0 + kb + 1) * 128 + 64 * (long long)rank);
         if (c > 0) load_down(e, c - 1);
       }
       load_down(e, nch - 1);
@@ -412,6 +452,7 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     // ---------------- MMA issue (the leader CTA) ----------------------------
     if (leader) {
       const uint32_t idesc = idesc_bf16(2 * kBM, kChunk);  // M = 256 over the pair, N = 128
+      const uint32_t idesc256 = idesc_bf16(2 * kBM, 256);   // the down projection's wide pieces
       const uint16_t both = 3;
       const uint32_t tU = tmem_base + kUCol;
       const int n_stages = p.slots / kStageHalves;
@@ -456,7 +497,7 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         ++uc;
         return true;
       };
-      // down items j = hh * npc + np: h half hh times V_e rows of piece np
+      // down stages in the order of down_stage (the loader's order)
       auto down = [&](int i, int c) {
         if (c == 0) {
           if (!wait_warp_cluster(dempty, ((uint32_t)i & 1u) ^ 1u, abort_flag, p.status,
@@ -465,26 +506,41 @@ ffn_fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
           tc_fence_after();
         }
 #pragma unroll
-        for (int j0 = 0; j0 < 2 * npc; j0 += kStageHalves) {
-#pragma unroll
-          for (int j = j0; j < j0 + kStageHalves; ++j)
-            if (j % npc == 0 &&
-                !wait_warp_cluster(hsfull(j / npc), dc & 1u, abort_flag, p.status, p.wait_limit))
-              return false;
+        for (int st = 0; st < kDownStages; ++st) {
+          int hh, P;
+          const bool wide = down_stage(st, hh, P);
+          if (st == 0 &&
+              !wait_warp_cluster(hsfull(0), dc & 1u, abort_flag, p.status, p.wait_limit))
+            return false;
+          if (st == n256 &&
+              !wait_warp_cluster(hsfull(1), dc & 1u, abort_flag, p.status, p.wait_limit))
+            return false;
           if (!wait_warp_cluster(wfull(s), ph, abort_flag, p.status, p.wait_limit)) return false;
           tc_fence_after();
           if (elect_one()) {
-#pragma unroll
-            for (int jj = 0; jj < kStageHalves; ++jj) {
-              const int j = j0 + jj, hh = j / npc, np = j - hh * npc;
+            const uint32_t w0 = sW + (uint32_t)(s * kStageHalves) * kHalf;
+            if (wide) {
+              // N = 256: this CTA's 128 rows of the piece span the stage's
+              // two half-slab slots (contiguous, 8-row groups 1 KB apart)
               const uint64_t a = sw128_desc(sH + (uint32_t)hh * kXBlock);
-              const uint64_t b = sw128_desc(sW + (uint32_t)(s * kStageHalves + jj) * kHalf);
+              const uint64_t b = sw128_desc(w0);
 #pragma unroll
               for (int k = 0; k < kBK / 16; ++k)
-                umma_bf16_pair(tmem_base + (uint32_t)(np * kPiece), a + 2 * k, b + 2 * k, idesc,
+                umma_bf16_pair(tmem_base + (uint32_t)(P * 256), a + 2 * k, b + 2 * k, idesc256,
                                (c | hh | k) != 0 ? 1u : 0u);
-              if (np == npc - 1) umma_commit_pair(hsempty(hh), both);
+            } else {
+#pragma unroll
+              for (int jj = 0; jj < kStageHalves; ++jj) {
+                const uint64_t a = sw128_desc(sH + (uint32_t)jj * kXBlock);
+                const uint64_t b = sw128_desc(w0 + (uint32_t)jj * kHalf);
+#pragma unroll
+                for (int k = 0; k < kBK / 16; ++k)
+                  umma_bf16_pair(tmem_base + (uint32_t)(n256 * 256), a + 2 * k, b + 2 * k, idesc,
+                                 (c | jj | k) != 0 ? 1u : 0u);
+              }
             }
+            if (st == kH0Last) umma_commit_pair(hsempty(0), both);
+            if (st == kDownStages - 1) umma_commit_pair(hsempty(1), both);
             umma_commit_pair(wempty(s), both);
           }
           __syncwarp();
