@@ -367,11 +367,12 @@ __global__ void timeout_probe_kernel(int* status, long long limit) {
 // ---------------------------------------------------------------------------
 // Router on the tensor cores (bf16 layers)
 // ---------------------------------------------------------------------------
-// One CTA per 128 tokens: z = x [W_shr | W_g | mu] as a 128 x Cp x d MMA
-// (Eqs. 17, 21), TMA-fed, fp32 accumulator in TMEM. Each of the four decision
-// warps then owns 32 tokens = 32 TMEM lanes: a thread reads its token's Cp
-// logits, takes the decisions of Eqs. 18-27 and the warp counts its chunk's
-// (expert, block) pairs.
+// One CTA per R tokens (R = 32, 64, 96 or 128, chosen per call so that the
+// grid fits on the SMs in one wave): z = x [W_shr | W_g | mu] as a 128 x Cp
+// x d MMA (Eqs. 17, 21; rows past R are computed and never read), TMA-fed,
+// fp32 accumulator in TMEM. Each decision warp then owns 32 tokens = 32
+// TMEM lanes: a thread reads its token's Cp logits, takes the decisions of
+// Eqs. 18-27 and the warp counts its chunk's (expert, block) pairs.
 constexpr int kRtThreads = 192;   // warp 0 TMA, warp 1 TMEM + MMA, warps 2-5 decisions
 constexpr int kRtStages = 6;
 constexpr uint32_t kRtStageB = 160u * kBK * 2;  // up to 160 router columns
@@ -392,6 +393,8 @@ struct RouterTcParams {
   int fused;     // 1: the router also lays out the group rows by (expert, block)
                  // (group_rows); 2: by expert (group_rows_expert)
   int d, Cp;
+  int rows;      // tokens per CTA: 32, 64, 96 or 128 (the MMA always spans 128
+                 // rows; the rows past the tile are never read back)
   uint32_t tmem_cols;
   int* status;
   long long wait_limit;
@@ -414,7 +417,8 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kRtStages + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int t0 = blockIdx.x * kBM;
+  const int R = p.rows;
+  const int t0 = blockIdx.x * R;
   const int Cp = p.Cp, K = p.dec.K;
   // the up projection may start its prologue on SMs this grid leaves free
   grid_dep_launch();
@@ -442,7 +446,7 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      const uint32_t bytes = kStageA + (uint32_t)Cp * kBK * 2;
+      const uint32_t bytes = (uint32_t)(R + Cp) * kBK * 2;  // the x box (R rows) and the router box
       for (int kb = 0; kb < num_kb; ++kb) {
         if (!wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.status, p.wait_limit)) break;
         mbar_expect_tx(full_bar(stage), bytes);
@@ -490,20 +494,25 @@ router_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant
     const int G = p.grp.G;
     int32_t* gsm = reinterpret_cast<int32_t*>(cscr + 4 * 128);  // group_rows' counters
     int32_t* misc_s = gsm + group_rows_smem_ints(4, G) - 8;
+    // a warp whose quarter lies past the CTA's R tokens takes no decisions
+    // (those token indices belong to the next CTA) and counts nothing
+    const bool in_tile = q * 32 < R;
     if (wait_warp(accf, 0u, abort_flag, p.status, p.wait_limit)) {
       tc_fence_after();
-      float* z = zs + row * (Cp + 1);
-      for (int c = 0; c < Cp; c += 32) {
-        float v[32];
-        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + c, v);
+      if (in_tile) {
+        float* z = zs + row * (Cp + 1);
+        for (int c = 0; c < Cp; c += 32) {
+          float v[32];
+          tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + c, v);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) z[c + i] = v[i];
+          for (int i = 0; i < 32; ++i) z[c + i] = v[i];
+        }
+        const bool valid = t < p.dec.T && (p.dec.mask == nullptr || p.dec.mask[t] != 0);
+        decide_token(p.dec, t, valid, z, sv, shr, em, alpha);
       }
-      const bool valid = t < p.dec.T && (p.dec.mask == nullptr || p.dec.mask[t] != 0);
-      decide_token(p.dec, t, valid, z, sv, shr, em, alpha);
-      const int chunk = blockIdx.x * (kBM / 32) + q;
+      const int chunk = blockIdx.x * (R / 32) + q;
       if (!p.fused) {
-        if (chunk < p.dec.n_chunks)
+        if (in_tile && chunk < p.dec.n_chunks)
           count_chunk_pairs(p.dec, lane, shr, em, cscr + q * 128,
                             p.dec.chunk_cnt + chunk, p.dec.n_chunks);
       } else {
@@ -722,8 +731,14 @@ int router_tc_setup(unif_moe_layer* L) {
 
 cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* mask, int T,
                              int32_t* b_out, int32_t* k_out, cudaStream_t s) {
+  // Tokens per CTA: the smallest multiple of 32 whose grid still fits in one
+  // wave on the SMs (the x load is bound per SM: spreading the tokens over
+  // more SMs shortens it), else 128.
+  int R = tc::kBM;
+  for (int r = 32; r < tc::kBM; r += 32)
+    if ((T + r - 1) / r <= L->n_sm) { R = r; break; }
   CUtensorMap tm_x;
-  if (!tc::encode_2d(&tm_x, x, L->d, (uint64_t)T, tc::kBK, tc::kBM)) return cudaErrorInvalidValue;
+  if (!tc::encode_2d(&tm_x, x, L->d, (uint64_t)T, tc::kBK, (uint32_t)R)) return cudaErrorInvalidValue;
   tc::RouterTcParams p;
   p.dec = decide_args(L, mask, T, b_out, k_out);
   p.fused = L->fused_group ? (L->ffn_fused ? 2 : 1) : 0;
@@ -738,10 +753,11 @@ cudaError_t launch_router_tc(unif_moe_layer* L, const void* x, const uint8_t* ma
   }
   p.d = L->d;
   p.Cp = L->router_cols_pad;
+  p.rows = R;
   p.tmem_cols = p.Cp <= 32 ? 32u : (p.Cp <= 64 ? 64u : (p.Cp <= 128 ? 128u : 256u));
   p.status = L->ws.status;
   p.wait_limit = tc::g_wait_limit;
-  tc::router_tc_kernel<<<(T + tc::kBM - 1) / tc::kBM, tc::kRtThreads, tc::kRtSmem, s>>>(
+  tc::router_tc_kernel<<<(T + R - 1) / R, tc::kRtThreads, tc::kRtSmem, s>>>(
       tm_x, L->tm_wr, p);
   return cudaGetLastError();
 }
