@@ -531,6 +531,7 @@ def main():
         if mask is not None:
             rows_t = rows_t * mask.long()
         n_rows_last = int(rows_t[last0:].sum())
+    exec_tf = (4.0 * d * s.d_ff * n_rows_last / (ffn_ms / 1e3) / 1e12) if expert_tile else None
     router_bytes = (T_last * d * elt + T_last * (4 * 3 + 8 * 2 + 4 * s.n_experts + 8) +
                     (8 * n_rows_last if fused else 0))
     combine_bytes = T_last * d * (4 + elt)
@@ -547,6 +548,11 @@ def main():
                     {"ms": 0.0, "fused_into": "router", "event_gap_ms": stage_ms["permute"]}),
         **({"ffn": {"ms": ffn_ms, "TFLOP/s": ach, "frac_of_burst_bf16": ach / peak_tf,
                     "kernel": "expert-tile FFN (both projections, rows grouped by expert)",
+                    # the tensor work the kernel issues: both projections over
+                    # all H channels of every (token, expert) row, the blocks
+                    # the row does not run included (masked)
+                    "executed_TFLOP/s": exec_tf,
+                    "executed_frac_of_burst_bf16": exec_tf / peak_tf,
                     "event_gap_ms": stage_ms["down_gemm"]}} if expert_tile else {
             "up_gemm": {"ms": stage_ms["up_gemm"],
                         "TFLOP/s": stage_flops / stage_ms["up_gemm"] / 1e9,

@@ -59,7 +59,7 @@ namespace tc {
 namespace fused {
 
 constexpr int kChunk = 128;           // H channels per chunk (the up MMA's N)
-constexpr int kPiece = 128;           // output columns per down MMA (its N)
+constexpr int kPiece = 128;           // d rows per repacked V_e slab (an N = 128 MMA's B; N = 256 takes two)
 constexpr uint32_t kSlab = 16384;     // a weight slab: 128 rows x 64 bf16
 constexpr uint32_t kHalf = 8192;      // the half of a slab one CTA of the pair holds
 constexpr uint32_t kXBlock = 16384;   // 128 rows x 64 bf16 of x or h
@@ -151,7 +151,7 @@ __device__ __forceinline__ void pair_tile_table(const int32_t* fill, int G, int 
 }
 
 // DD = d (128, 256 or 384): the x tile's 64-column blocks and the down
-// projection's 128-column pieces are compile-time counts, so that the MMA
+// projection's stages and pieces are compile-time counts, so that the MMA
 // warp's per-stage control is a few instructions (it shares its scheduler
 // with epilogue warps running GeLU, and a runtime division per stage
 // measurably delayed every stage)
