@@ -104,6 +104,32 @@ def test_ragged_token_counts(T):
     assert_parity(wl, g, compare(wl, g))
 
 
+def _router_rows(T, n_sm):
+    """Tokens per router CTA the library picks for T tokens: the smallest
+    multiple of 32 whose grid fits on the SMs, else 128."""
+    for r in (32, 64, 96):
+        if (T + r - 1) // r <= n_sm:
+            return r
+    return 128
+
+
+@pytest.mark.parametrize("where", ["R=32 last", "R=64 first", "R=64 last", "R=96 first",
+                                   "R=96 last", "R=128 first"])
+def test_router_tile_heights(where):
+    """Token counts at each switch of the tensor-core router's tokens per CTA
+    (32, 64, 96, 128 with the grid in one wave): every token's decisions and
+    output against the oracle, with a ragged last CTA on both sides."""
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    R, side = where.split()
+    R = int(R[2:])
+    prev = {32: 0, 64: 32, 96: 64, 128: 96}[R]
+    T = prev * n_sm + 1 if side == "first" else R * n_sm - 5
+    assert _router_rows(T, n_sm) == R
+    wl = workloads.make_workload(small(tokens=T, d_model=128, d_ff=256, n_experts=4, n_blocks=4))
+    g = run_gpu(wl)
+    assert_parity(wl, g, compare(wl, g))
+
+
 def test_zero_tokens_is_noop():
     wl = workloads.make_workload(small(tokens=16))
     layer = make_layer(wl.spec)
