@@ -113,15 +113,15 @@ def _router_rows(T, n_sm):
     return 128
 
 
-@pytest.mark.parametrize("where", ["R=32 last", "R=64 first", "R=64 last", "R=96 first",
-                                   "R=96 last", "R=128 first"])
+@pytest.mark.parametrize("where", ["R32-last", "R64-first", "R64-last", "R96-first",
+                                   "R96-last", "R128-first"])
 def test_router_tile_heights(where):
     """Token counts at each switch of the tensor-core router's tokens per CTA
     (32, 64, 96, 128 with the grid in one wave): every token's decisions and
     output against the oracle, with a ragged last CTA on both sides."""
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
-    R, side = where.split()
-    R = int(R[2:])
+    R, side = where.split("-")
+    R = int(R[1:])
     prev = {32: 0, 64: 32, 96: 64, 128: 96}[R]
     T = prev * n_sm + 1 if side == "first" else R * n_sm - 5
     assert _router_rows(T, n_sm) == R
