@@ -33,12 +33,15 @@
 // tiles. TMEM (512 columns): D in columns [0, d), U in [384, 512).
 //
 // Roles (each CTA, 18 warps):
-//   warps 0-3    gather this CTA's x rows (16-byte cp.async, 32 rows each)
+//   warps 0-3    gather this CTA's x rows (16-byte cp.async, 32 rows each),
+//                then drain the previous tile's D columns [d/2, d)
 //   warp 4       this CTA's weight half-slabs by TMA, in MMA order
-//   warp 5       TMEM allocation (both CTAs); MMA issue (even CTA, one lane)
+//   warp 5       TMEM allocation (both CTAs); MMA issue (even CTA, one lane);
+//                in the odd CTA, zeroing of the next pass's accumulator
 //   warps 6-13   chunk epilogue: U -> GeLU -> masked bf16 h in shared memory
 //                (warp w: TMEM lane quarter w % 4, 64-column half (w-6)/4)
-//   warps 14-17  drain: w D -> fp32 atomic adds into the accumulator
+//   warps 14-17  drain: w D columns [0, d/2) -> fp32 atomic adds into the
+//                accumulator
 // The even CTA's barriers collect both CTAs' arrivals (x rows, h, U and D
 // read) and both halves of each slab (TMA with cta_group::2 completes on
 // them); its MMA commits arrive on both CTAs' barriers (multicast). Order
