@@ -775,10 +775,15 @@ int gemm_fused_setup(unif_moe_layer* L) {
   L->ffn_per_cta = (int)((max_tiles + clusters - 1) / clusters);  // pair tiles per pair
   if (L->ffn_per_cta > per_pair_guess) {  // fewer pairs than SMs / 2: a longer run table
     L->ffn_smem = smem_bytes(num_kb, slots, G, L->ffn_per_cta);
-    if (L->ffn_smem > kMaxSmem) {
+    while (L->ffn_smem > kMaxSmem && slots > 2 * kStageHalves) {
       slots -= kStageHalves;
       L->ffn_slots = slots;
       L->ffn_smem = smem_bytes(num_kb, slots, G, L->ffn_per_cta);
+    }
+    if (L->ffn_smem > kMaxSmem) {
+      set_error("expert-tile FFN: a run of %d pair tiles per pair does not fit in shared memory",
+                L->ffn_per_cta);
+      return UNIF_MOE_ERR_SHAPE;
     }
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)L->ffn_smem) != cudaSuccess) {

@@ -1,8 +1,9 @@
 // Host side of the UniF-MoE C ABI declared in include/unif_moe.h: argument
 // checks, workspace allocation at create time, and the launch sequence of a
 // forward pass
-//   router (Eqs. 17-27) -> permute (groups of Eqs. 28-29) ->
-//   grouped up/down GEMMs (Eq. 16) -> combine (Eq. 30).
+//   router (Eqs. 17-27; bf16 layers also group the rows, Eqs. 28-29) ->
+//   [fp32 layers: permute] -> expert-tile FFN (bf16, d <= 384) or grouped
+//   up/down GEMMs (Eq. 16) -> combine (Eq. 30).
 #include <algorithm>
 #include <math.h>
 #include <stdarg.h>
@@ -319,7 +320,18 @@ int unif_moe_create_ex(unif_moe_t* out, int d_model, int d_ff, int n_experts, in
     rc = UNIF_MOE_ERR_CUDA;
   }
   if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::gemm_tc_setup(L);
-  if (rc == UNIF_MOE_OK && L->ffn_fused) rc = unif::gemm_fused_setup(L);
+  if (rc == UNIF_MOE_OK && L->ffn_fused) {
+    rc = unif::gemm_fused_setup(L);
+    // AUTO falls back to the grouped kernels (their workspace is allocated
+    // either way) when the expert-tile kernel cannot be set up here; an
+    // explicit EXPERT_TILE request fails instead
+    if (rc != UNIF_MOE_OK && o.gemm_kernels == UNIF_MOE_GEMM_AUTO) {
+      L->ffn_fused = false;
+      L->tile_list = L->fused_group && !(L->up_ws && L->down_ws);
+      cudaGetLastError();  // a failed attribute call must not surface at a later launch
+      rc = UNIF_MOE_OK;
+    }
+  }
   if (rc == UNIF_MOE_OK && dtype == UNIF_MOE_BF16) rc = unif::router_tc_setup(L);
   if (rc == UNIF_MOE_OK && (o.features & UNIF_MOE_FEATURE_BACKWARD)) rc = unif::backward_setup(L);
   if (rc != UNIF_MOE_OK) {
