@@ -500,6 +500,23 @@ def test_expert_tile_shapes(shape):
     assert_parity(wl, g, compare(wl, g, label="expert_tile"))
 
 
+def test_expert_tile_padding_mask():
+    """Text-style batch (valid lengths uniform per sequence, padding tokens
+    NaN-filled and masked) through the expert-tile FFN: padding tokens get no
+    rows, their outputs are exactly zero, the NaNs reach no valid token, and
+    every valid token's decisions and output match the oracle."""
+    s = workloads.spec("bert_base").with_(tokens=2048, d_model=256, d_ff=1024, n_experts=8,
+                                          n_blocks=8)
+    wl = workloads.make_workload(s)
+    g = run_gpu(wl)
+    assert g.layer.kernels_per_forward() == 3
+    m = wl.mask.numpy()
+    assert 0 < int(m.sum()) < s.tokens
+    assert (g.b[m == 0] == 0).all() and (g.k[m == 0] == 0).all()
+    assert (g.y[m == 0] == 0).all() and np.isfinite(g.y).all()
+    assert_parity(wl, g, compare(wl, g, label="expert_tile, padding"))
+
+
 def test_vit_s_streaming_kernels():
     """The ViT-S layer through the streaming GEMMs agrees with the oracle too."""
     wl = workloads.make_workload(workloads.spec("vit_s", tokens=4000))
